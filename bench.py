@@ -1,0 +1,519 @@
+"""Throughput of the policy-loss hot path on the multi-turn agent workload.
+
+Workload (the configuration the headline metric is quoted on): 16 groups x 8
+trajectories with lengths U{256..2048} (about 147K packed tokens), ~40% of the
+tokens masked in spans, rewards Bernoulli(0.3), vocabulary V = 151,936, bf16
+logits ~ N(0, 2^2), 16,384-row microbatches. The whole batch's logits and
+gradient stay resident in HBM (about 90 GB, far above the 129 MB L2, so no L2
+flush is needed between steps).
+
+One step = rl_group_advantages over the batch, then rl_policy_loss_fwd_bwd over
+every microbatch (the loss accumulates on the device; its value is read back
+once after the timed region).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+Prints one JSON line. With N > 1 (launched by torchrun) every rank runs its own
+replica of the workload; the step time is the maximum over ranks.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import multiprocessing as mp
+import os
+import re
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2608_16798_gb300 import workloads as W  # noqa: E402
+
+METRIC = "policy-loss fwd+bwd tokens/s at V=151,936 and % of HBM roofline (1 GB300)"
+UNIT = "tokens/s"
+WORKLOAD = W.WORKLOADS["multiturn"]
+PROFILE = os.path.join(ROOT, "profiles", "rows_kernel_multiturn.md")
+KERNEL_SRC = os.path.join(ROOT, "paper_2608_16798_gb300", "csrc", "rl_rows.cu")
+FALLBACK_HBM_GBS = 6800.0
+
+
+def workload_config(T, n_mb):
+    w = WORKLOAD
+    return {"workload": f"multiturn: {w.n_groups} groups x {w.group_size} trajectories, lengths U{{256..2048}}, "
+                        f"~40% masked in spans, V={w.vocab}, bf16 logits N(0,2^2), {w.microbatch}-row microbatches",
+            "tokens_per_step": int(T), "microbatches": int(n_mb), "vocab": w.vocab, "logits": "bf16",
+            "l2": "no flush: resident inputs (logits + gradient) far larger than L2",
+            "parallelism": "replicas"}
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return FALLBACK_HBM_GBS, "fallback"
+
+
+def profiled_traffic():
+    """Per-launch DRAM bytes of the rows kernel from the committed ncu summary, if it was taken
+    on the current kernel source (else None)."""
+    if not os.path.exists(PROFILE):
+        return None
+    txt = open(PROFILE).read()
+    m_b = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", txt)
+    m_h = re.search(r"kernel_source_sha256:\s*([0-9a-f]{64})", txt)
+    if not m_b or not m_h:
+        return None
+    cur = hashlib.sha256(open(KERNEL_SRC, "rb").read()).hexdigest()
+    return float(m_b.group(1)) if cur == m_h.group(1) else None
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling during the timed region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index  # nvidia-smi --id value: the GPU's UUID when torch reports one
+        self.proc = None
+        self.path = os.path.join("/tmp", f"bench_clocks_{os.getpid()}.csv")
+
+    def start(self):
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.f.close()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        os.remove(self.path)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+# ----------------------------------------------------------------------------- device workload
+
+class DeviceBatch:
+    def __init__(self, torch, R, dev, seed=0):
+        w = WORKLOAD
+        self.lay = W.make_layout(w, seed)
+        self.T = self.lay.n_tokens
+        self.V = w.vocab
+        self.mbs = W.microbatches(self.lay, w.microbatch)
+        t = torch
+        self.logits = t.empty((self.T, self.V), dtype=t.bfloat16, device=dev)
+        W.logits_rows_torch(w, seed, 0, self.T, self.logits)
+        self.ids = W.sample_tokens_torch(self.logits, seed, 0, w)
+        self.grad = t.empty_like(self.logits)
+        d = lambda x: t.from_numpy(np.ascontiguousarray(x)).to(dev)  # noqa: E731
+        self.mask = d(self.lay.mask)
+        self.rewards = d(self.lay.rewards)
+        self.group_offsets = d(self.lay.group_offsets)
+        self.traj_offsets = d(self.lay.traj_offsets)
+        self.valid = d(self.lay.traj_valid)
+        self.params = R.make_params(W.CLIP_EPS_LOW, W.CLIP_EPS_HIGH, 0.0, 0, 0.0, 0.0, 1e-6, 0)
+        self.ws = R.new_workspace(w.microbatch, self.V, device=dev)
+        # pi_old as the training engine recomputes it: this library's forward log-probs, plus noise
+        logp = t.empty(self.T, dtype=t.float32, device=dev)
+        for lo, hi in self.mbs:
+            R.rl_token_logprobs(self.logits[lo:hi], self.ids[lo:hi], self.ws, logp_out=logp[lo:hi])
+        self.old = d(W.old_logp_from(logp.cpu().numpy(), w, seed))
+        self.adv = t.empty(self.lay.n_traj, dtype=t.float32, device=dev)
+        self.coef = t.empty_like(self.adv)
+        self.n_tok = t.empty(self.lay.n_traj, dtype=t.int32, device=dev)
+        self.token_traj = t.empty(self.T, dtype=t.int32, device=dev)
+        self.loss = t.zeros(1, dtype=t.float64, device=dev)
+        m = self.lay.mask.astype(np.int64)
+        es = 2
+        # algorithmic bytes per microbatch launch: trainable rows read + write, other rows write only
+        self.mb_bytes = [int(((m[lo:hi] + 1) * self.V * es).sum()) for lo, hi in self.mbs]
+
+    def step(self, R, events=None):
+        R.rl_group_advantages(self.group_offsets, self.rewards, self.traj_offsets, self.mask, self.params, self.ws,
+                              traj_valid=self.valid, adv_out=self.adv, coef_out=self.coef, n_tok_out=self.n_tok,
+                              token_traj_out=self.token_traj)
+        for k, (lo, hi) in enumerate(self.mbs):
+            if events is not None:
+                events[k][0].record()
+            R.rl_policy_loss_fwd_bwd(self.logits[lo:hi], self.ids[lo:hi], self.mask[lo:hi], self.token_traj[lo:hi],
+                                     self.adv, self.coef, self.old[lo:hi], self.params, self.ws, self.loss,
+                                     grad_out=self.grad[lo:hi])
+            if events is not None:
+                events[k][1].record()
+
+    def launches_per_step(self):
+        return 2 + 2 * len(self.mbs)
+
+
+def e2e_run(torch, R, batch, dev, steps, warmup):
+    """Same step through host buffers: every step copies its inputs from pinned host memory
+    (metadata + each microbatch's logits) and reads back the gradient and the loss.
+
+    Host memory holds a ring of two microbatches of logits and gradient (pinned), reused
+    cyclically; copies and kernels overlap on two streams."""
+    t = torch
+    w = WORKLOAD
+    V, mb = batch.V, w.microbatch
+    host_logits = [t.empty((mb, V), dtype=t.bfloat16, pin_memory=True) for _ in range(2)]
+    host_grad = [t.empty((mb, V), dtype=t.bfloat16, pin_memory=True) for _ in range(2)]
+    for k in range(2):
+        lo, hi = batch.mbs[k % len(batch.mbs)]
+        host_logits[k][:hi - lo].copy_(batch.logits[lo:hi])
+    meta_host = {n: getattr(batch, n).cpu().pin_memory() for n in
+                 ("ids", "mask", "old", "rewards", "group_offsets", "traj_offsets", "valid")}
+    meta_dev = {n: t.empty_like(getattr(batch, n)) for n in meta_host}
+    dev_logits = [t.empty((mb, V), dtype=t.bfloat16, device=dev) for _ in range(2)]
+    dev_grad = [t.empty((mb, V), dtype=t.bfloat16, device=dev) for _ in range(2)]
+    loss_host = t.zeros(1, dtype=t.float64, pin_memory=True)
+    copy_in, copy_out = t.cuda.Stream(dev), t.cuda.Stream(dev)
+    comp = t.cuda.current_stream(dev)
+    adv, coef = t.empty_like(batch.adv), t.empty_like(batch.coef)
+    n_tok, tt = t.empty_like(batch.n_tok), t.empty_like(batch.token_traj)
+    loss = t.zeros(1, dtype=t.float64, device=dev)
+    h2d = sum(v.numel() * v.element_size() for v in meta_host.values())
+    h2d += sum((hi - lo) * V * 2 for lo, hi in batch.mbs)
+    d2h = sum((hi - lo) * V * 2 for lo, hi in batch.mbs) + 8
+
+    def one_step():
+        for n, h in meta_host.items():
+            meta_dev[n].copy_(h, non_blocking=True)
+        R.rl_group_advantages(meta_dev["group_offsets"], meta_dev["rewards"], meta_dev["traj_offsets"],
+                              meta_dev["mask"], batch.params, batch.ws, traj_valid=meta_dev["valid"], adv_out=adv,
+                              coef_out=coef, n_tok_out=n_tok, token_traj_out=tt)
+        loaded = [None, None]
+        freed = [None, None]
+        for k, (lo, hi) in enumerate(batch.mbs):
+            s = k & 1
+            n = hi - lo
+            with t.cuda.stream(copy_in):
+                if freed[s] is not None:
+                    copy_in.wait_event(freed[s])
+                dev_logits[s][:n].copy_(host_logits[s][:n], non_blocking=True)
+                loaded[s] = t.cuda.Event()
+                loaded[s].record(copy_in)
+            comp.wait_event(loaded[s])
+            R.rl_policy_loss_fwd_bwd(dev_logits[s][:n], meta_dev["ids"][lo:hi], meta_dev["mask"][lo:hi], tt[lo:hi],
+                                     adv, coef, meta_dev["old"][lo:hi], batch.params, batch.ws, loss,
+                                     grad_out=dev_grad[s][:n], stream=comp)
+            done = t.cuda.Event()
+            done.record(comp)
+            with t.cuda.stream(copy_out):
+                copy_out.wait_event(done)
+                host_grad[s][:n].copy_(dev_grad[s][:n], non_blocking=True)
+                freed[s] = t.cuda.Event()
+                freed[s].record(copy_out)
+        comp.wait_stream(copy_out)
+        loss_host.copy_(loss, non_blocking=True)
+
+    for _ in range(warmup):
+        one_step()
+    t.cuda.synchronize(dev)
+    e0, e1 = t.cuda.Event(enable_timing=True), t.cuda.Event(enable_timing=True)
+    e0.record(comp)
+    for _ in range(steps):
+        one_step()
+    e1.record(comp)
+    e1.synchronize()
+    t.cuda.synchronize(dev)
+    ms = e0.elapsed_time(e1)
+    return ms, h2d, d2h
+
+
+# ----------------------------------------------------------------------------- oracle (CPU) legs
+
+_W = {}
+
+
+def _oracle_init(shm_name, shape, ids, mask, tt, adv, coef, old):
+    from multiprocessing import shared_memory
+
+    sys.path.insert(0, ROOT)
+    shm = shared_memory.SharedMemory(name=shm_name)
+    _W.update(shm=shm, raw=np.ndarray(shape, dtype=np.uint16, buffer=shm.buf), ids=ids, mask=mask, tt=tt, adv=adv,
+              coef=coef, old=old)
+
+
+def _oracle_rows(span):
+    import oracle.grpo_objective as O
+
+    lo, hi = span
+    O.policy_loss_fwd_bwd(_W["raw"][lo:hi], "bf16", _W["ids"][lo:hi], _W["mask"][lo:hi], _W["tt"][lo:hi], _W["adv"],
+                          _W["coef"], _W["old"][lo:hi], O.LossParams())
+    return hi - lo
+
+
+def oracle_sample_inputs(batch_host):
+    """Inputs of the CPU oracle for a sample of the workload: the first packed tokens.
+
+    old_logp is placed near the sampled token's log-probability from the logit law
+    (lse ~ ln V + sigma^2 / 2 for N(0, sigma^2) logits), which keeps the timing leg
+    independent of the CUDA library's outputs."""
+    import oracle.grpo_objective as O
+
+    w = WORKLOAD
+    lay = batch_host["layout"]
+    raw = batch_host["raw"]
+    ids = batch_host["ids"]
+    rows = raw.shape[0]
+    z_a = (raw[np.arange(rows), ids].astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    logp_hat = z_a - (math.log(w.vocab) + w.logit_std ** 2 / 2)
+    old = W.old_logp_from(logp_hat, w, 0)
+    P = O.LossParams()
+    adv, coef, L, tt = O.advantages_and_coefficients(lay.rewards, lay.group_offsets, lay.traj_offsets, lay.mask,
+                                                     lay.traj_valid, P)
+    return raw, ids, lay.mask[:rows], tt[:rows], adv, coef, old
+
+
+class OraclePool:
+    """The float64 oracle, as it stands, over a spawn pool of all host cores.
+
+    The sample's logits sit in shared memory; each job is a 16-row span of the sample.
+    ``run(seconds)`` cycles over the sample's spans for about that long and returns
+    rows per second."""
+
+    CHUNK = 16
+
+    def __init__(self, batch_host):
+        from multiprocessing import shared_memory
+
+        self.cores = len(os.sched_getaffinity(0))
+        raw, ids, mask, tt, adv, coef, old = oracle_sample_inputs(batch_host)
+        self.rows = raw.shape[0]
+        self.shm = shared_memory.SharedMemory(create=True, size=raw.nbytes)
+        np.ndarray(raw.shape, dtype=np.uint16, buffer=self.shm.buf)[:] = raw
+        self.spans = [(i, min(self.rows, i + self.CHUNK)) for i in range(0, self.rows, self.CHUNK)]
+        self.pool = mp.get_context("spawn").Pool(self.cores, initializer=_oracle_init,
+                                                 initargs=(self.shm.name, raw.shape, ids, mask, tt, adv, coef, old))
+        self.pool.map(_oracle_rows, self.spans[:self.cores], chunksize=1)   # imports and first touch
+        t0 = time.perf_counter()
+        n = sum(self.pool.map(_oracle_rows, [self.spans[j % len(self.spans)] for j in range(self.cores)],
+                              chunksize=1))
+        self.rate = n / max(time.perf_counter() - t0, 1e-6)
+        self.done = 0
+        self.wall = 0.0
+
+    def run(self, seconds):
+        n_jobs = max(self.cores, int(self.rate * seconds / self.CHUNK))
+        jobs = [self.spans[(self.done // self.CHUNK + j) % len(self.spans)] for j in range(n_jobs)]
+        t0 = time.perf_counter()
+        done = sum(self.pool.map(_oracle_rows, jobs, chunksize=1))
+        dt = time.perf_counter() - t0
+        self.done += done
+        self.wall += dt
+        return done / dt
+
+    def describe(self):
+        return {"unit": UNIT, "cores": self.cores, "kind": "oracle",
+                "sample": f"{self.done} token rows cycled over the first {self.rows} packed tokens of the batch "
+                          f"(masked rows included), float64 numpy oracle on {self.cores} spawn workers, "
+                          f"{self.wall:.1f} s wall"}
+
+    def close(self):
+        self.pool.close()
+        self.pool.join()
+        self.shm.close()
+        self.shm.unlink()
+
+
+def time_oracle(batch_host, target_s=15.0):
+    """One bounded timing of the oracle on a sample of the workload (about target_s of wall time)."""
+    op = OraclePool(batch_host)
+    try:
+        v = op.run(target_s)
+        d = op.describe()
+    finally:
+        op.close()
+    d["value"] = v
+    return d
+
+
+def host_sample(torch, batch, rows):
+    """Copy a sample of the device workload (torch-drawn logits and ids) to the host."""
+    raw = batch.logits[:rows].view(torch.int16).cpu().numpy().view(np.uint16)
+    ids = batch.ids[:rows].cpu().numpy()
+    return {"layout": batch.lay, "raw": raw, "ids": ids}
+
+
+def host_sample_np(rows):
+    """A host-only sample of the same workload (numpy generator), for runs without a GPU."""
+    lay = W.make_layout(WORKLOAD, 0)
+    raw, vals = W.logits_rows_np(WORKLOAD, 0, 0, rows)
+    ids = W.sample_tokens_np(vals, 0, 0, WORKLOAD)
+    return {"layout": lay, "raw": raw, "ids": ids}
+
+
+# ----------------------------------------------------------------------------- main
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    return int(os.environ.get("RANK", "0")), ws, int(os.environ.get("LOCAL_RANK", "0"))
+
+
+def run_reference(args):
+    """The oracle timed on the host cores, on the same workload, metric and unit: each step is a
+    bounded sample sized so that the whole run stays within a few minutes."""
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    lay = W.make_layout(WORKLOAD, 0)
+    n_mb = len(W.microbatches(lay, WORKLOAD.microbatch))
+    op = OraclePool(host_sample_np(min(lay.n_tokens, 512)))
+    per_step = max(0.3, 150.0 / max(1, args.steps + args.warmup))
+    vals = []
+    try:
+        for i in range(args.warmup + args.steps):
+            v = op.run(per_step)
+            if i >= args.warmup:
+                vals.append(v)
+        cb = op.describe()
+    finally:
+        op.close()
+    v = statistics.median(vals)
+    cb["value"] = v
+    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": lay.n_tokens / v * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": workload_config(lay.n_tokens, n_mb), "cpu_baseline": cb,
+            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="cuda", choices=["cuda", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=5)
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    args.warmup = max(3, args.warmup)
+
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_16798_gb300 import build as B
+
+    B.build()
+    import paper_2608_16798_gb300.rl_loss as R
+
+    rank, world, local = dist_env()
+    if world > 1:
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    dev = torch.device("cuda", local if world > 1 else 0)
+    torch.cuda.set_device(dev)
+    R.lib()
+
+    batch = DeviceBatch(torch, R, dev)
+    n_mb = len(batch.mbs)
+    for _ in range(args.warmup):
+        batch.step(R)
+    torch.cuda.synchronize(dev)
+
+    # timed region: K steps, barrier + synchronize on both sides
+    evs = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_mb)]
+           for _ in range(args.steps)]
+    props = torch.cuda.get_device_properties(dev)
+    uuid = str(getattr(props, "uuid", "") or "")
+    sampler = ClockSampler(("GPU-" + uuid) if uuid and not uuid.startswith("GPU-") else (uuid or str(dev.index)))
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    sampler.start()
+    time.sleep(0.3)
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for k in range(args.steps):
+        batch.step(R, evs[k])
+    t1.record()
+    torch.cuda.synchronize(dev)
+    clocks = sampler.stop()
+    if world > 1:
+        dist.barrier()
+    ms = t0.elapsed_time(t1)
+    kern_ms = [a.elapsed_time(b) for step in evs for (a, b) in step]
+    st, word = R.rl_query_status(batch.ws)
+    if word != 0:
+        raise RuntimeError(f"device status word {word} after the timed region")
+    if world > 1:
+        tt = torch.tensor([ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+    ms_step = ms / args.steps
+    value = batch.T * world / (ms / 1e3 / args.steps)
+
+    peak, peak_kind = measured_peaks()
+    per_launch_bytes = sum(batch.mb_bytes) / n_mb
+    avg_launch_ms = sum(kern_ms) / len(kern_ms)
+    achieved = per_launch_bytes / (avg_launch_ms * 1e-3) / 1e9
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                "traffic": profiled_traffic(), "peak_source": peak_kind,
+                "kernel": "rows_kernel<bf16> via rl_policy_loss_fwd_bwd (+ 1-CTA loss reduction)",
+                "algorithmic_bytes_per_launch": per_launch_bytes, "avg_launch_ms": avg_launch_ms}
+
+    e2e = None
+    if not args.no_e2e:
+        e_ms, h2d, d2h = e2e_run(torch, R, batch, dev, args.e2e_steps, 1)
+        e2e = {"value": batch.T / (e_ms / 1e3 / args.e2e_steps) * world, "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "steps": args.e2e_steps}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = time_oracle(host_sample(torch, batch, 2048))
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+                "vs_baseline": None, "dtype": "f32", "data": "synthetic", "config": workload_config(batch.T, n_mb),
+                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks,
+                "gpu_launches": batch.launches_per_step() * args.steps,
+                "loss_per_step": float(batch.loss.item()) / (args.warmup + args.steps)}
+        print(json.dumps(line))
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

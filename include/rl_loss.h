@@ -1,0 +1,213 @@
+/*
+ * rl_loss.h -- C ABI of the GB300 (sm_103a) policy-loss library.
+ *
+ * The library computes the token-level, group-relative clipped policy-gradient
+ * objective of black-box agent RL (ClawGym II, arXiv 2608.16798) over packed,
+ * ragged trajectories, and its gradient with respect to the logits:
+ *
+ *   - group-relative advantages A_i = (R_i - mu_g) / (sigma_g + eps) with the
+ *     population standard deviation (Sec. 2.3.2, GRPO advantage equation;
+ *     Sec. 3.2.3 for groups of rollouts; Sec. 3.3 for task-harness groups);
+ *   - the masked objective (1/G) sum_i (1 / sum_t M_it) sum_t M_it [min(rho A,
+ *     clip(rho, 1-eps, 1+eps) A) - beta KL] (Sec. 2.3.2, GRPO objective; the
+ *     mask M_t of Sec. 2.3.1 excludes harness / tool-observation tokens);
+ *   - the token-level truncated importance weight w_t = min(exp(log pi_old -
+ *     log pi_rollout), c-bar) (Sec. 3.2.4, TIS equation);
+ *   - log pi(a_t | s_t) of the sampled token, a log-softmax over the vocabulary
+ *     (Sec. 2.3, the policy pi_theta(a_t | s_t)).
+ *
+ * Conventions shared by every entry point:
+ *   - Array arguments are DEVICE pointers owned by the caller. The library
+ *     never allocates, frees or synchronises (except rl_query_status, which
+ *     synchronises the given stream). All work is enqueued on `stream`
+ *     (a cudaStream_t; NULL is the legacy default stream).
+ *   - Argument errors that the host can see return a status before anything is
+ *     launched; rl_last_error_message() then describes the problem.
+ *   - Errors that only the device can see (a token id outside [0, V), a
+ *     trajectory index outside [0, n_traj), inconsistent offsets, a bounded
+ *     wait that ran out) set bits of a status word kept in the workspace;
+ *     kernels never trap. Read it with rl_query_status().
+ *   - The loss returned is the NEGATED objective (the paper maximises the
+ *     objective; the library gives a loss to minimise and its gradient).
+ *   - Logits rows are dense, row-major, row r starting at element r * ld.
+ *     bf16 values are IEEE bfloat16 bit patterns.
+ */
+#ifndef RL_LOSS_H
+#define RL_LOSS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same object as cudaStream_t. */
+typedef struct CUstream_st* rl_stream_t;
+
+typedef enum rl_status {
+  RL_OK = 0,
+  RL_ERR_INVALID_ARG = 1,         /* null pointer, negative size, bad enum value, ld < V ... */
+  RL_ERR_UNSUPPORTED = 2,         /* a shape the kernels do not handle (e.g. V too large) */
+  RL_ERR_ALIGNMENT = 3,           /* a base pointer that must be 16-byte aligned is not */
+  RL_ERR_WORKSPACE_TOO_SMALL = 4, /* ws_bytes below rl_workspace_size(...) */
+  RL_ERR_CUDA = 5,                /* a CUDA runtime call failed; see rl_last_error_message() */
+  RL_ERR_DEVICE_CHECK = 6,        /* rl_query_status: a device-side check failed */
+  RL_ERR_TIMEOUT = 7              /* rl_query_status: a bounded device wait ran out */
+} rl_status;
+
+typedef enum rl_dtype { RL_BF16 = 0, RL_F32 = 1 } rl_dtype;
+
+/* How per-token terms are weighted into the batch loss (the coefficient c_i of
+ * trajectory i, so that loss = sum_t c_{i(t)} M_t l_t). */
+typedef enum rl_loss_agg {
+  /* c_i = 1 / (N * L_i), N = number of valid trajectories with L_i > 0: the
+   * per-trajectory token mean of Sec. 2.3.2, then the mean over trajectories. */
+  RL_AGG_SEQ_MEAN_TOKEN_MEAN = 0,
+  RL_AGG_TOKEN_MEAN = 1, /* c_i = 1 / sum_valid L_i */
+  RL_AGG_TOKEN_SUM = 2   /* c_i = 1 */
+} rl_loss_agg;
+
+/* Bits of the device status word. */
+enum {
+  RL_DEV_BAD_TOKEN = 1,   /* a token id outside [0, V); that row gets no loss and a zero gradient */
+  RL_DEV_BAD_TRAJ = 2,    /* token_traj outside [0, n_traj); same treatment */
+  RL_DEV_BAD_OFFSETS = 4, /* group / trajectory offsets not non-decreasing within range */
+  RL_DEV_TIMEOUT = 8      /* a bounded wait for an asynchronous copy ran out */
+};
+
+typedef struct rl_loss_params {
+  float clip_eps_low;  /* ratio clipped to [1 - clip_eps_low, 1 + clip_eps_high] */
+  float clip_eps_high;
+  float kl_coef;       /* beta; used when kl_estimator == 3 and ref_logp != NULL */
+  int32_t kl_estimator;/* 0 = no KL term, 3 = k3: exp(r - logp) - (r - logp) - 1 */
+  float entropy_coef;  /* alpha >= 0: loss -= alpha * H_t (entropy bonus) */
+  float tis_cap;       /* c-bar; <= 0 or rollout_logp == NULL disables the TIS weight */
+  float adv_eps;       /* epsilon added to sigma in the advantage denominator */
+  int32_t loss_agg;    /* rl_loss_agg */
+} rl_loss_params;
+
+/* Library version, major * 10000 + minor * 100 + patch. */
+int32_t rl_version(void);
+
+/* Text of the last error returned on this host thread ("" if none). The
+ * pointer stays valid until the next call into the library on this thread. */
+const char* rl_last_error_message(void);
+
+/* Workspace bytes needed by calls on at most `max_rows` logits rows of
+ * vocabulary V (D = hidden size of the fused head, 0 if unused). The
+ * workspace holds the device status word and per-row loss contributions. */
+size_t rl_workspace_size(int64_t max_rows, int64_t V, int64_t D);
+
+/* Zero the workspace's status word. Call once after allocating a workspace,
+ * and again to clear a reported device error. */
+rl_status rl_workspace_init(void* ws, size_t ws_bytes, rl_stream_t stream);
+
+/* Synchronise `stream`, then read the device status word into
+ * *device_status_out (0 = no error; else RL_DEV_* bits). Returns RL_OK,
+ * RL_ERR_DEVICE_CHECK or RL_ERR_TIMEOUT. The word is not cleared. */
+rl_status rl_query_status(const void* ws, rl_stream_t stream, int32_t* device_status_out);
+
+/*
+ * Group-relative advantages and loss coefficients (Sec. 2.3.2 GRPO advantage
+ * and objective; Sec. 3.2.3 rollout groups; Sec. 3.3 task-harness groups;
+ * Sec. 3.4 discarded rollouts are left out of advantage estimation and
+ * optimisation).
+ *
+ *   n_traj            number of trajectories n (>= 0)
+ *   n_groups          number of groups (>= 0)
+ *   group_offsets     int32 [n_groups + 1]: group g owns trajectories
+ *                     [group_offsets[g], group_offsets[g+1]); non-decreasing, in [0, n_traj]
+ *   rewards           float [n_traj]: R_i
+ *   traj_valid        uint8 [n_traj] or NULL (all valid): 0 = discarded rollout
+ *   n_tokens          T, length of the packed token stream (>= 0)
+ *   traj_offsets      int64 [n_traj + 1]: trajectory i owns tokens
+ *                     [traj_offsets[i], traj_offsets[i+1]) of the packed stream
+ *   mask              uint8 [T]: M_t (nonzero = trainable, policy-generated token)
+ *   params            host pointer; adv_eps and loss_agg are used
+ *   adv_out           float [n_traj]: A_i (0 for invalid trajectories, for
+ *                     trajectories in no group, and for groups whose valid rewards
+ *                     are all equal)
+ *   coef_out          float [n_traj]: c_i per loss_agg (0 if invalid or L_i = 0)
+ *   n_tok_out         int32 [n_traj]: L_i = sum of M_t over the trajectory (exact)
+ *   token_traj_out    int32 [T] or NULL: owner trajectory of each token
+ *   ws, ws_bytes      workspace (rl_workspace_size(0, 0, 0) bytes suffice)
+ *
+ * mu and sigma are taken over the valid members of each group in double
+ * precision; outputs are rounded to float.
+ */
+rl_status rl_group_advantages(int32_t n_traj, int32_t n_groups, const int32_t* group_offsets,
+                              const float* rewards, const uint8_t* traj_valid, int64_t n_tokens,
+                              const int64_t* traj_offsets, const uint8_t* mask,
+                              const rl_loss_params* params, float* adv_out, float* coef_out,
+                              int32_t* n_tok_out, int32_t* token_traj_out, void* ws,
+                              size_t ws_bytes, rl_stream_t stream);
+
+/*
+ * Forward-only log-probabilities of the sampled tokens (the pi_old / pi_ref
+ * recompute of Sec. 3.2.4): for every row r,
+ *   lse_r = log sum_v exp(z_rv), logp_r = z_{r,a_r} - lse_r, H_r = -sum_v p_rv log p_rv.
+ *
+ *   logits       [rows x ld] of `dtype`; base 16-byte aligned
+ *   rows, V, ld  rows >= 0, 1 <= V <= ld
+ *   token_ids    int32 [rows]: a_r (out of range -> logp_r = NaN and RL_DEV_BAD_TOKEN)
+ *   logp_out     float [rows]
+ *   entropy_out  float [rows] or NULL (entropy work is skipped when NULL)
+ *   lse_out      float [rows] or NULL
+ * One streaming pass over the logits (online softmax, fp32 accumulation).
+ */
+rl_status rl_token_logprobs(const void* logits, rl_dtype dtype, int64_t rows, int64_t V, int64_t ld,
+                            const int32_t* token_ids, float* logp_out, float* entropy_out,
+                            float* lse_out, void* ws, size_t ws_bytes, rl_stream_t stream);
+
+/*
+ * Masked clipped policy loss over one microbatch of logits rows and its
+ * gradient d loss / d logits (Sec. 2.3.1 PPO masked objective; Sec. 2.3.2 GRPO
+ * objective with the KL penalty; Sec. 3.2.4 TIS weight).
+ *
+ * For each row t with M_t != 0 and c_{i(t)} != 0 (i(t) = token_traj[t]):
+ *   logp = z_a - lse; rho = exp(logp - old_logp);
+ *   surr = min(rho A, clip(rho, 1 - eps_low, 1 + eps_high) A);
+ *   w = min(exp(old_logp - rollout_logp), tis_cap) if enabled, else 1 (no gradient);
+ *   KL = exp(r - logp) - (r - logp) - 1 with r = ref_logp (k3), if enabled;
+ *   l_t = -w surr + beta KL - alpha H;
+ *   loss += c_i l_t;
+ *   grad_v = c_i [g (delta_{v,a} - p_v) + alpha p_v (log p_v + H)],
+ *   g = -w A rho act + beta (1 - exp(r - logp)), act = 0 iff
+ *   (A > 0 and rho > 1 + eps_high) or (A < 0 and rho < 1 - eps_low).
+ * Every other row gets an exactly-zero gradient row and contributes nothing.
+ *
+ *   logits        [rows x ld] of `dtype`, base 16-byte aligned
+ *   rows, V, ld   rows >= 0, 1 <= V <= ld
+ *   token_ids     int32 [rows]
+ *   mask          uint8 [rows]: M_t
+ *   token_traj    int32 [rows]: trajectory of each row (index into adv / coef)
+ *   n_traj        length of adv and coef
+ *   adv, coef     float [n_traj]: A_i and c_i for the WHOLE batch (from
+ *                 rl_group_advantages), so a trajectory split across
+ *                 microbatches keeps its normaliser
+ *   old_logp      float [rows]: log pi_old(a_t | s_t)
+ *   ref_logp      float [rows] or NULL: log pi_ref(a_t | s_t) for the KL term
+ *   rollout_logp  float [rows] or NULL: log pi_rollout(a_t | s_t) for TIS
+ *   params        host pointer
+ *   grad_out      [rows x ld] of `dtype`, base 16-byte aligned; may equal logits
+ *                 (in place); elements v >= V of each row are not written
+ *   loss_accum    double [1] on the device: the microbatch loss is ADDED to it
+ *                 (deterministic: fixed-order reduction)
+ *   token_stats   float [rows x 5] or NULL: (logp, rho, clipped flag, H, KL) for
+ *                 active rows, zeros for the others
+ *   ws, ws_bytes  workspace of at least rl_workspace_size(rows, V, 0) bytes
+ */
+rl_status rl_policy_loss_fwd_bwd(const void* logits, rl_dtype dtype, int64_t rows, int64_t V,
+                                 int64_t ld, const int32_t* token_ids, const uint8_t* mask,
+                                 const int32_t* token_traj, int32_t n_traj, const float* adv,
+                                 const float* coef, const float* old_logp, const float* ref_logp,
+                                 const float* rollout_logp, const rl_loss_params* params,
+                                 void* grad_out, double* loss_accum, float* token_stats, void* ws,
+                                 size_t ws_bytes, rl_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* RL_LOSS_H */

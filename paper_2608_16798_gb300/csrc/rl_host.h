@@ -1,0 +1,27 @@
+// Host-side internals shared by the library's translation units.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <string>
+
+#include <cuda_runtime.h>
+
+#include "rl_loss.h"
+
+namespace rl {
+
+// Workspace layout (offsets in bytes from the caller's workspace pointer):
+//   [0, 256)                 header: int32 device status word at offset 0
+//   [256, 256 + 8 * rows)    double per-row loss contributions c_i * l_t
+constexpr size_t kWsHeader = 256;
+
+inline size_t ws_row_loss_offset() { return kWsHeader; }
+
+rl_status set_error(rl_status st, const std::string& msg);
+rl_status cuda_error(cudaError_t e, const char* what);
+void clear_error();
+
+inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+}  // namespace rl

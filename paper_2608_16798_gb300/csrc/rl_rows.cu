@@ -1,0 +1,687 @@
+// Streaming log-softmax kernels over logits rows:
+//
+//   rl_token_logprobs       logp / entropy / lse of the sampled token per row
+//                           (pi(a_t | s_t) of Sec. 2.3; the pi_old recompute of
+//                           Sec. 3.2.4)
+//   rl_policy_loss_fwd_bwd  the masked clipped objective (Sec. 2.3.1, 2.3.2),
+//                           k3-KL, entropy bonus and TIS weight (Sec. 3.2.4), and
+//                           d loss / d logits
+//
+// Design (GB300, sm_103a). Each logits row is owned by one thread-block
+// cluster of C CTAs; CTA k of the cluster holds the vocabulary slice
+// [k * slice, (k + 1) * slice) of the row in shared memory. The slice arrives
+// by bulk asynchronous copies (cp.async.bulk, the 1-D TMA) completing on an
+// mbarrier, double-buffered so the copy of the cluster's next row overlaps the
+// work on the current one. Pass 1 reads the slice once from shared memory and
+// forms an online-softmax partial (max m, sum exp(z - m), sum exp(z - m)(z - m));
+// the C partials are exchanged through distributed shared memory and merged
+// identically in every CTA. Pass 2 re-reads the slice from shared memory and
+// writes the gradient with 16-byte stores. Each unmasked row is therefore read
+// from HBM exactly once and its gradient written once; masked rows (and rows of
+// trajectories with c_i = 0) are not read at all, only zero-filled.
+//
+// The kernels are persistent: the grid holds as many clusters as fit on the
+// GPU at once, and cluster j processes rows j, j + n_clusters, ... . Per-row
+// loss contributions go to the workspace and are summed in a fixed order by a
+// one-CTA kernel, so the loss is bit-reproducible.
+#include <algorithm>
+#include <cstdint>
+#include <map>
+#include <mutex>
+#include <tuple>
+
+#include "rl_device.cuh"
+#include "rl_host.h"
+
+namespace rl {
+
+struct RowArgs {
+  const void* logits;
+  void* grad;
+  int64_t rows, V, ld;
+  const int32_t* token_ids;
+  const uint8_t* mask;
+  const int32_t* token_traj;
+  int32_t n_traj;
+  const float* adv;
+  const float* coef;
+  const float* old_logp;
+  const float* ref_logp;
+  const float* rollout_logp;
+  float clip_lo, clip_hi;  // 1 - eps_low, 1 + eps_high
+  float beta;              // 0 when the KL term is off
+  float alpha;             // entropy bonus
+  float tis_cap;           // <= 0 when TIS is off
+  double* row_loss;
+  float* token_stats;
+  float* logp_out;
+  float* entropy_out;
+  float* lse_out;
+  int32_t* status;
+  int64_t slice;      // elements per CTA slice, a multiple of the 16-byte vector
+  int64_t buf_elems;  // element stride between the two shared-memory buffers
+  int32_t tma;        // rows 16-byte aligned: bulk copies and 16-byte stores
+};
+
+#ifndef RL_STORE_CS
+#define RL_STORE_CS 0
+#endif
+
+// 16-byte global store; with RL_STORE_CS the line is marked evict-first (streaming)
+__device__ __forceinline__ void st_global_16(void* p, uint4 w) {
+#if RL_STORE_CS
+  asm volatile("st.global.cs.v4.b32 [%0], {%1, %2, %3, %4};" :: "l"(p), "r"(w.x), "r"(w.y), "r"(w.z), "r"(w.w)
+               : "memory");
+#else
+  *reinterpret_cast<uint4*>(p) = w;
+#endif
+}
+
+template <typename T>
+struct Vec;
+template <>
+struct Vec<uint16_t> {  // bf16
+  static constexpr int N = 8;
+  static __device__ __forceinline__ void load(const uint16_t* buf, int64_t j, float (&v)[8]) {
+    const uint4 w = reinterpret_cast<const uint4*>(buf)[j];
+    v[0] = bf16_lo(w.x); v[1] = bf16_hi(w.x); v[2] = bf16_lo(w.y); v[3] = bf16_hi(w.y);
+    v[4] = bf16_lo(w.z); v[5] = bf16_hi(w.z); v[6] = bf16_lo(w.w); v[7] = bf16_hi(w.w);
+  }
+  static __device__ __forceinline__ void store(uint16_t* dst, const float (&g)[8]) {
+    uint4 w;
+    w.x = pack_bf16x2(g[0], g[1]); w.y = pack_bf16x2(g[2], g[3]);
+    w.z = pack_bf16x2(g[4], g[5]); w.w = pack_bf16x2(g[6], g[7]);
+    st_global_16(dst, w);
+  }
+  static __device__ __forceinline__ void store_scalar(uint16_t* dst, float g) { *dst = f32_to_bf16(g); }
+  static __device__ __forceinline__ float to_f(uint16_t x) { return bf16_to_f32(x); }
+};
+template <>
+struct Vec<float> {
+  static constexpr int N = 4;
+  static __device__ __forceinline__ void load(const float* buf, int64_t j, float (&v)[4]) {
+    const float4 w = reinterpret_cast<const float4*>(buf)[j];
+    v[0] = w.x; v[1] = w.y; v[2] = w.z; v[3] = w.w;
+  }
+  static __device__ __forceinline__ void store(float* dst, const float (&g)[4]) {
+    st_global_16(dst, make_uint4(__float_as_uint(g[0]), __float_as_uint(g[1]), __float_as_uint(g[2]),
+                                 __float_as_uint(g[3])));
+  }
+  static __device__ __forceinline__ void store_scalar(float* dst, float g) { *dst = g; }
+  static __device__ __forceinline__ float to_f(float x) { return x; }
+};
+
+#define RL_NEG_INF (-__int_as_float(0x7f800000))
+constexpr uint32_t kBulkChunk = 32768;
+
+// fold one value into a per-thread online-softmax partial whose max is already >= z
+template <bool ENT>
+__device__ __forceinline__ void accumulate(SoftmaxPartial& ps, float z, float neg_m_l2e) {
+  if (ENT) {
+    const float t = fmaxf(z, -1e30f) - ps.m;  // -inf logits contribute 0, not NaN
+    const float e = ex2(t * kLog2e);
+    ps.s += e;
+    ps.u = fmaf(e, t, ps.u);
+  } else {
+    ps.s += ex2(fmaf(z, kLog2e, neg_m_l2e));
+  }
+}
+
+template <bool ENT>
+__device__ __forceinline__ void raise_max(SoftmaxPartial& ps, float vm) {
+  if (vm > ps.m) {
+    const float d = ps.m - vm;
+    const float sc = ex2(d * kLog2e);
+    if (ENT) ps.u = (ps.s == 0.f) ? 0.f : sc * fmaf(d, ps.s, ps.u);
+    ps.s *= sc;
+    ps.m = vm;
+  }
+}
+
+// Tuning knobs (compile-time): shared-memory stages per CTA, consumer warps per
+// CTA, and the slice size that picks the cluster width.
+#ifndef RL_STAGES
+#define RL_STAGES 2
+#endif
+#ifndef RL_CONSUMER_WARPS
+#define RL_CONSUMER_WARPS 8
+#endif
+#ifndef RL_SLICE_KB
+#define RL_SLICE_KB 48
+#endif
+
+constexpr int kMaxCluster = 16;
+constexpr int kZeroBytes = 8192;  // zero-filled shared region, source of the masked rows' bulk stores
+
+// Per-row inputs, staged in shared memory by the producer warp.
+struct RowMeta {
+  int64_t r;  // row index, -1 = end of the stream
+  int32_t a;  // sampled token id
+  float A, c, old, ref, roll;
+};
+
+// Warp-specialised, cluster-per-row kernel.
+//
+//   warp NW (producer): walks this cluster's rows cid, cid + ncl, ...; decides which
+//     are trained on; zero-fills the others with bulk stores from a zeroed shared
+//     region; for a trained row stages its metadata and bulk-copies this CTA's slice
+//     into the next free stage (full / empty mbarrier pair per stage).
+//   warps 0..NW-1 (consumers): per row, pass 1 over the slice gives one online-softmax
+//     partial per warp; every warp pushes its partial to all C CTAs of the cluster
+//     with st.async (remote store + complete_tx on the receiver's mailbox mbarrier);
+//     each warp then merges all C * NW partials in a fixed order (bit-identical in
+//     every warp of every CTA), computes the row's scalars, runs pass 2 (gradient
+//     from the on-chip slice) and releases the stage.
+// Nothing per row synchronises a whole CTA or the whole cluster.
+template <typename T, int NW, bool ENT, bool BWD>
+__global__ void __launch_bounds__((NW + 1) * 32, 2) rows_kernel(const RowArgs p) {
+  constexpr int EPV = Vec<T>::N;
+  constexpr int NB = RL_STAGES;
+  constexpr int NC = NW * 32;  // consumer threads
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  __shared__ __align__(8) uint64_t full_bar[NB], empty_bar[NB], xbar[2];
+  __shared__ RowMeta meta[NB];
+  __shared__ __align__(16) float4 mbox[2][kMaxCluster * NW];
+  __shared__ __align__(128) uint4 zeros[kZeroBytes / 16];
+
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const uint32_t rank = cluster_ctarank(), C = cluster_nctarank();
+  const int64_t cid = blockIdx.x / C, ncl = gridDim.x / C;
+  const int64_t rows = p.rows, V = p.V, ld = p.ld;
+  const int64_t s0 = static_cast<int64_t>(rank) * p.slice;
+  const int64_t n_end = (s0 + p.slice < V) ? s0 + p.slice : V;
+  const int64_t n = n_end > s0 ? n_end - s0 : 0;  // elements of my slice
+  const int64_t nv = n / EPV;                      // full 16-byte vectors
+  const int64_t first_scalar = p.tma ? nv * EPV : 0;
+  const uint32_t tma_bytes = p.tma ? static_cast<uint32_t>(nv * 16) : 0u;
+  const T* logits = static_cast<const T*>(p.logits);
+  T* grad = static_cast<T*>(p.grad);
+  T* const buf_base = reinterpret_cast<T*>(smem_raw);
+
+  if (tid == 0) {
+#pragma unroll
+    for (int k = 0; k < NB; ++k) {
+      mbar_init(&full_bar[k], 1);
+      mbar_init(&empty_bar[k], NW);
+    }
+    mbar_init(&xbar[0], 1);
+    mbar_init(&xbar[1], 1);
+    fence_mbar_init();
+  }
+  for (int k = tid; k < kZeroBytes / 16; k += blockDim.x) zeros[k] = make_uint4(0, 0, 0, 0);
+  fence_proxy_async_smem();
+  __syncthreads();
+  if (C > 1) cluster_sync_all();  // every peer's mailbox barrier exists before the first st.async
+
+  if (warp == NW) {
+    // =============================================================== producer warp
+    uint32_t it = 0;
+    bool failed = false, stored = false;
+    for (int64_t r = cid; r < rows && !failed; r += ncl) {
+      RowMeta m;
+      bool active = true;
+      m.r = r;
+      m.a = p.token_ids[r];
+      if (BWD) {
+        active = p.mask[r] != 0;
+        if (active) {
+          const int32_t i = p.token_traj[r];
+          if (i < 0 || i >= p.n_traj) {
+            if (rank == 0 && lane == 0) flag_status(p.status, RL_DEV_BAD_TRAJ);
+            active = false;
+          } else {
+            m.c = p.coef[i];
+            m.A = p.adv[i];
+            active = m.c != 0.f;
+            if (active && (m.a < 0 || m.a >= V)) {
+              if (rank == 0 && lane == 0) flag_status(p.status, RL_DEV_BAD_TOKEN);
+              active = false;
+            }
+          }
+        }
+        if (!active) {
+          // zero this CTA's slice of gradient row r
+          T* g = grad + r * ld + s0;
+          if (p.tma) {
+            if (lane == 0) {
+              const uint32_t bytes = tma_bytes;
+              for (uint32_t off = 0; off < bytes; off += kZeroBytes)
+                bulk_s2g(reinterpret_cast<char*>(g) + off, zeros, min(static_cast<uint32_t>(kZeroBytes), bytes - off));
+              bulk_commit();
+              stored = true;
+            }
+            for (int64_t e = nv * EPV + lane; e < n; e += 32) g[e] = T(0);
+          } else {
+            for (int64_t e = lane; e < n; e += 32) g[e] = T(0);
+          }
+          if (rank == 0 && lane == 0) {
+            p.row_loss[r] = 0.0;
+            if (p.token_stats)
+              for (int k = 0; k < 5; ++k) p.token_stats[r * 5 + k] = 0.f;
+          }
+          continue;
+        }
+        m.old = p.old_logp[r];
+        m.ref = p.ref_logp ? p.ref_logp[r] : 0.f;
+        m.roll = p.rollout_logp ? p.rollout_logp[r] : 0.f;
+      }
+      const int b = it % NB;
+      const uint32_t use = it / NB;
+      if (use > 0 && !mbar_wait_bounded(&empty_bar[b], (use - 1) & 1)) {
+        failed = true;
+        if (lane == 0) flag_status(p.status, RL_DEV_TIMEOUT);
+        break;
+      }
+      T* buf = buf_base + b * p.buf_elems;
+      const T* src = logits + r * ld + s0;
+      for (int64_t e = first_scalar + lane; e < n; e += 32) buf[e] = src[e];
+      __syncwarp();
+      if (lane == 0) {
+        meta[b] = m;
+        if (tma_bytes > 0) {
+          mbar_arrive_expect_tx(&full_bar[b], tma_bytes);
+          for (uint32_t off = 0; off < tma_bytes; off += kBulkChunk)
+            bulk_g2s(reinterpret_cast<char*>(buf) + off, reinterpret_cast<const char*>(src) + off,
+                     min(kBulkChunk, tma_bytes - off), &full_bar[b]);
+        } else {
+          mbar_arrive(&full_bar[b]);
+        }
+      }
+      ++it;
+    }
+    if (!failed) {
+      // end of stream
+      const int b = it % NB;
+      const uint32_t use = it / NB;
+      if (use > 0 && !mbar_wait_bounded(&empty_bar[b], (use - 1) & 1)) {
+        if (lane == 0) flag_status(p.status, RL_DEV_TIMEOUT);
+      } else if (lane == 0) {
+        meta[b].r = -1;
+        mbar_arrive(&full_bar[b]);
+      }
+    }
+    if (lane == 0 && stored) bulk_wait_read_all();
+  } else {
+    // =============================================================== consumer warps
+    for (uint32_t it = 0;; ++it) {
+      const int b = it % NB;
+      if (!mbar_wait_bounded(&full_bar[b], (it / NB) & 1)) {
+        if (tid == 0) flag_status(p.status, RL_DEV_TIMEOUT);
+        break;
+      }
+      const RowMeta m = meta[b];
+      if (m.r < 0) break;
+      const int64_t r = m.r;
+      const T* buf = buf_base + b * p.buf_elems;
+      const int32_t a = m.a;
+      const bool a_ok = a >= 0 && a < V;
+      const uint32_t owner = a_ok ? static_cast<uint32_t>(a / p.slice) : 0u;
+
+      // ---- pass 1: online softmax partial over the slice
+      SoftmaxPartial ps{RL_NEG_INF, 0.f, 0.f};
+      for (int64_t j = tid; j < nv; j += NC) {
+        float v[EPV];
+        Vec<T>::load(buf, j, v);
+        float vm = v[0];
+#pragma unroll
+        for (int k = 1; k < EPV; ++k) vm = fmaxf(vm, v[k]);
+        if (vm == RL_NEG_INF) continue;
+        raise_max<ENT>(ps, vm);
+        const float nm = -ps.m * kLog2e;
+#pragma unroll
+        for (int k = 0; k < EPV; ++k) accumulate<ENT>(ps, v[k], nm);
+      }
+      for (int64_t e = nv * EPV + tid; e < n; e += NC) {
+        const float z = Vec<T>::to_f(buf[e]);
+        if (z == RL_NEG_INF) continue;
+        raise_max<ENT>(ps, z);
+        accumulate<ENT>(ps, z, -ps.m * kLog2e);
+      }
+      ps = warp_merge(ps);
+      // lane 0's merge is the warp's partial: broadcast it so every copy sent is identical
+      ps.m = __shfl_sync(0xffffffffu, ps.m, 0);
+      ps.s = __shfl_sync(0xffffffffu, ps.s, 0);
+      ps.u = __shfl_sync(0xffffffffu, ps.u, 0);
+      // warp 0 of the CTA holding the sampled token carries z_a; every other partial carries 0
+      const float za_part = (warp == 0 && a_ok && rank == owner) ? Vec<T>::to_f(buf[a - s0]) : 0.f;
+
+      // ---- exchange: every warp's partial to every CTA of the cluster
+      const int par = it & 1;
+      if (warp == 0 && lane == 0) mbar_arrive_expect_tx(&xbar[par], C * NW * 16u);
+      if (lane < static_cast<int>(C)) {
+        const uint32_t dst = map_to_rank(smem_addr(&mbox[par][rank * NW + warp]), lane);
+        const uint32_t bar = map_to_rank(smem_addr(&xbar[par]), lane);
+        st_async_f4(dst, make_float4(ps.m, ps.s, ps.u, za_part), bar);
+      }
+      if (!mbar_wait_cluster_bounded(&xbar[par], (it >> 1) & 1)) {
+        if (lane == 0) flag_status(p.status, RL_DEV_TIMEOUT);
+        break;
+      }
+      // ---- merge all C * NW partials in a fixed order
+      const int total = static_cast<int>(C) * NW;
+      SoftmaxPartial qa{RL_NEG_INF, 0.f, 0.f}, qb{RL_NEG_INF, 0.f, 0.f};
+      float zsum = 0.f;
+      if (lane < total) {
+        const float4 w = mbox[par][lane];
+        qa = SoftmaxPartial{w.x, w.y, w.z};
+        zsum = w.w;
+      }
+      if (lane + 32 < total) {
+        const float4 w = mbox[par][lane + 32];
+        qb = SoftmaxPartial{w.x, w.y, w.z};
+        zsum += w.w;
+      }
+      for (int k = lane + 64; k < total; k += 32) {  // clusters of 16 with more than 4 consumer warps
+        const float4 w = mbox[par][k];
+        qb = merge(qb, SoftmaxPartial{w.x, w.y, w.z});
+        zsum += w.w;
+      }
+      SoftmaxPartial q = warp_merge(merge(qa, qb));
+      const float za = __shfl_sync(0xffffffffu, warp_sum(zsum), 0);
+      const float lnS = logf(__shfl_sync(0xffffffffu, q.s, 0));
+      const float lse = __shfl_sync(0xffffffffu, q.m, 0) + lnS;
+      const float H = lnS - __shfl_sync(0xffffffffu, q.u, 0) / __shfl_sync(0xffffffffu, q.s, 0);
+
+      if (!BWD) {
+        if (rank == 0 && warp == 0 && lane == 0) {
+          if (!a_ok) flag_status(p.status, RL_DEV_BAD_TOKEN);
+          p.logp_out[r] = a_ok ? za - lse : __int_as_float(0x7fc00000);
+          if (p.entropy_out) p.entropy_out[r] = H;
+          if (p.lse_out) p.lse_out[r] = lse;
+        }
+      } else {
+        // per-token scalars (every lane computes the same values)
+        const float A = m.A, c = m.c, old = m.old;
+        const float logp = za - lse;
+        const float rho = expf((za - old) - lse);   // large operands differenced first
+        const float crho = fminf(fmaxf(rho, p.clip_lo), p.clip_hi);
+        const float surr = fminf(rho * A, crho * A);
+        const bool cut = (A > 0.f && rho > p.clip_hi) || (A < 0.f && rho < p.clip_lo);
+        const float w = (p.tis_cap > 0.f && p.rollout_logp) ? fminf(expf(old - m.roll), p.tis_cap) : 1.f;
+        float kl = 0.f, dkl = 0.f;
+        if (p.beta != 0.f && p.ref_logp) {
+          const float d = (m.ref - za) + lse;  // r - logp
+          const float ed = expf(d);
+          kl = ed - d - 1.f;
+          dkl = 1.f - ed;
+        }
+        const float ell = -w * surr + p.beta * kl - p.alpha * H;
+        const float g = (cut ? 0.f : -w * A * rho) + p.beta * dkl;
+        const float cg = c * g, ca = c * p.alpha;
+        const float Kp = -cg;                    // gradient = Kp p_v (+ cg at v = a)
+        const float Ke = -cg + ca * (H - lse);   // entropy: p_v (ca z_v + Ke)
+        if (rank == 0 && warp == 0 && lane == 0) {
+          p.row_loss[r] = static_cast<double>(c) * static_cast<double>(ell);
+          if (p.token_stats) {
+            float* st = p.token_stats + r * 5;
+            st[0] = logp; st[1] = rho; st[2] = cut ? 1.f : 0.f; st[3] = H; st[4] = kl;
+          }
+        }
+        // ---- pass 2: gradient from the on-chip slice
+        const float nl = -lse * kLog2e;
+        T* g_row = grad + r * ld + s0;
+        for (int64_t j = tid; j < nv; j += NC) {
+          float v[EPV], o[EPV];
+          Vec<T>::load(buf, j, v);
+#pragma unroll
+          for (int k = 0; k < EPV; ++k) {
+            const float pk = ex2(fmaf(v[k], kLog2e, nl));
+            o[k] = ENT ? pk * fmaf(ca, fmaxf(v[k], -1e30f), Ke) : Kp * pk;
+          }
+          if (p.tma) {
+            Vec<T>::store(g_row + j * EPV, o);
+          } else {
+#pragma unroll
+            for (int k = 0; k < EPV; ++k) Vec<T>::store_scalar(g_row + j * EPV + k, o[k]);
+          }
+        }
+        for (int64_t e = nv * EPV + tid; e < n; e += NC) {
+          const float z = Vec<T>::to_f(buf[e]);
+          const float pk = ex2(fmaf(z, kLog2e, nl));
+          Vec<T>::store_scalar(g_row + e, ENT ? pk * fmaf(ca, fmaxf(z, -1e30f), Ke) : Kp * pk);
+        }
+        // the sampled token's element gets + c g; rewritten by the thread that stored it
+        if (rank == owner) {
+          const int64_t ia = a - s0;
+          const int64_t writer = ia < nv * EPV ? (ia / EPV) % NC : (ia - nv * EPV) % NC;
+          if (tid == writer) {
+            const float pk = ex2(fmaf(za, kLog2e, nl));
+            const float ga = (ENT ? pk * fmaf(ca, fmaxf(za, -1e30f), Ke) : Kp * pk) + cg;
+            Vec<T>::store_scalar(g_row + ia, ga);
+          }
+        }
+      }
+      // ---- release the stage
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty_bar[b]);
+    }
+  }
+  __syncthreads();
+  // no CTA leaves while a peer may still write into its mailbox
+  if (C > 1) cluster_sync_all();
+}
+
+// Fixed-order sum of the per-row contributions into the caller's accumulator.
+__global__ void __launch_bounds__(1024) reduce_loss_kernel(const double* __restrict__ row_loss, int64_t rows,
+                                                           double* loss_accum) {
+  __shared__ double part[32];
+  double acc = 0.0;
+  for (int64_t r = threadIdx.x; r < rows; r += 1024) acc += row_loss[r];
+  acc = warp_sum(acc);
+  if ((threadIdx.x & 31) == 0) part[threadIdx.x >> 5] = acc;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double t = 0.0;
+    for (int w = 0; w < 32; ++w) t += part[w];
+    *loss_accum += t;
+  }
+}
+
+// ------------------------------------------------------------------ host side
+
+constexpr int kConsumerWarps = RL_CONSUMER_WARPS;
+constexpr int kRowThreads = (RL_CONSUMER_WARPS + 1) * 32;
+constexpr int64_t kTargetSliceBytes = RL_SLICE_KB * 1024;
+constexpr int64_t kMaxSliceBytes = 100 * 1024;
+
+struct Plan {
+  int C;
+  int64_t slice, buf_elems;
+  size_t smem;
+};
+
+static bool make_plan(int64_t V, int es, Plan* out) {
+  const int64_t epv = 16 / es;
+  for (int C = 1; C <= 16; C *= 2) {
+    const int64_t per = (V + C - 1) / C;
+    const int64_t slice = (per + epv - 1) / epv * epv;
+    if (slice * es <= kTargetSliceBytes || (C == 16 && slice * es <= kMaxSliceBytes)) {
+      const int64_t stride_bytes = (slice * es + 127) / 128 * 128;
+      out->C = C;
+      out->slice = slice;
+      out->buf_elems = stride_bytes / es;
+      out->smem = static_cast<size_t>(RL_STAGES * stride_bytes);
+      return true;
+    }
+  }
+  return false;
+}
+
+template <typename T, bool ENT, bool BWD>
+static rl_status launch_rows(const RowArgs& args, const Plan& plan, cudaStream_t s) {
+  auto kern = rows_kernel<T, kConsumerWarps, ENT, BWD>;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_error(e, "cudaGetDevice");
+
+  static std::mutex mu;
+  static std::map<std::tuple<const void*, int, int, size_t>, int> cache;
+  static std::map<std::pair<const void*, int>, size_t> smem_attr;  // attribute value set per kernel and device
+  int max_clusters = 0;
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    // the function attribute bounds every later launch: keep it at the largest request so far
+    auto ka = std::make_pair(reinterpret_cast<const void*>(kern), dev);
+    auto ita = smem_attr.find(ka);
+    if (ita == smem_attr.end() || ita->second < plan.smem) {
+      e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(plan.smem));
+      if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(max dynamic smem)");
+      e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+      if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(non-portable cluster)");
+      smem_attr[ka] = plan.smem;
+    }
+    auto key = std::make_tuple(reinterpret_cast<const void*>(kern), dev, plan.C, plan.smem);
+    auto itc = cache.find(key);
+    if (itc != cache.end()) {
+      max_clusters = itc->second;
+    } else {
+      cudaLaunchConfig_t cfg = {};
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeClusterDimension;
+      attr[0].val.clusterDim.x = plan.C;
+      attr[0].val.clusterDim.y = 1;
+      attr[0].val.clusterDim.z = 1;
+      cfg.gridDim = dim3(plan.C * 1024, 1, 1);
+      cfg.blockDim = dim3(kRowThreads, 1, 1);
+      cfg.dynamicSmemBytes = plan.smem;
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      e = cudaOccupancyMaxActiveClusters(&max_clusters, kern, &cfg);
+      if (e != cudaSuccess) return cuda_error(e, "cudaOccupancyMaxActiveClusters");
+      if (max_clusters <= 0) return set_error(RL_ERR_UNSUPPORTED, "no cluster of this shape fits on the device");
+      cache[key] = max_clusters;
+    }
+  }
+  const int64_t n_clusters = std::max<int64_t>(1, std::min<int64_t>(max_clusters, args.rows));
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = plan.C;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.gridDim = dim3(static_cast<unsigned>(n_clusters * plan.C), 1, 1);
+  cfg.blockDim = dim3(kRowThreads, 1, 1);
+  cfg.dynamicSmemBytes = plan.smem;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, kern, args);
+  if (e != cudaSuccess) return cuda_error(e, "cudaLaunchKernelEx(rows_kernel)");
+  return RL_OK;
+}
+
+template <bool BWD>
+static rl_status dispatch_rows(rl_dtype dt, bool ent, const RowArgs& args, const Plan& plan, cudaStream_t s) {
+  if (dt == RL_BF16)
+    return ent ? launch_rows<uint16_t, true, BWD>(args, plan, s) : launch_rows<uint16_t, false, BWD>(args, plan, s);
+  return ent ? launch_rows<float, true, BWD>(args, plan, s) : launch_rows<float, false, BWD>(args, plan, s);
+}
+
+static rl_status check_rows_args(const char* fn, const void* logits, rl_dtype dt, int64_t rows, int64_t V,
+                                 int64_t ld, const void* ws, size_t ws_bytes, Plan* plan, int* es) {
+  if (dt != RL_BF16 && dt != RL_F32) return set_error(RL_ERR_INVALID_ARG, std::string(fn) + ": unknown dtype");
+  if (rows < 0 || V < 1 || ld < V)
+    return set_error(RL_ERR_INVALID_ARG, std::string(fn) + ": need rows >= 0, V >= 1, ld >= V");
+  if (!ws) return set_error(RL_ERR_INVALID_ARG, std::string(fn) + ": ws is NULL");
+  if (ws_bytes < rl_workspace_size(rows, V, 0))
+    return set_error(RL_ERR_WORKSPACE_TOO_SMALL, std::string(fn) + ": workspace smaller than rl_workspace_size(rows, V, 0)");
+  if (!aligned16(ws)) return set_error(RL_ERR_ALIGNMENT, std::string(fn) + ": ws not 16-byte aligned");
+  if (rows > 0 && !logits) return set_error(RL_ERR_INVALID_ARG, std::string(fn) + ": logits is NULL");
+  if (logits && !aligned16(logits)) return set_error(RL_ERR_ALIGNMENT, std::string(fn) + ": logits not 16-byte aligned");
+  if (V > INT32_MAX) return set_error(RL_ERR_UNSUPPORTED, std::string(fn) + ": V above 2^31 - 1");
+  *es = dt == RL_BF16 ? 2 : 4;
+  if (!make_plan(V, *es, plan))
+    return set_error(RL_ERR_UNSUPPORTED, std::string(fn) + ": vocabulary row larger than 16 x 100 KB");
+  return RL_OK;
+}
+
+}  // namespace rl
+
+extern "C" rl_status rl_token_logprobs(const void* logits, rl_dtype dtype, int64_t rows, int64_t V, int64_t ld,
+                                       const int32_t* token_ids, float* logp_out, float* entropy_out,
+                                       float* lse_out, void* ws, size_t ws_bytes, rl_stream_t stream) {
+  using namespace rl;
+  clear_error();
+  Plan plan;
+  int es = 0;
+  rl_status st = check_rows_args("rl_token_logprobs", logits, dtype, rows, V, ld, ws, ws_bytes, &plan, &es);
+  if (st != RL_OK) return st;
+  if (rows == 0) return RL_OK;
+  if (!token_ids || !logp_out) return set_error(RL_ERR_INVALID_ARG, "rl_token_logprobs: NULL array argument");
+  RowArgs a = {};
+  a.logits = logits;
+  a.rows = rows;
+  a.V = V;
+  a.ld = ld;
+  a.token_ids = token_ids;
+  a.logp_out = logp_out;
+  a.entropy_out = entropy_out;
+  a.lse_out = lse_out;
+  a.status = reinterpret_cast<int32_t*>(ws);
+  a.slice = plan.slice;
+  a.buf_elems = plan.buf_elems;
+  a.tma = ((ld * es) % 16) == 0;
+  return dispatch_rows<false>(dtype, entropy_out != nullptr, a, plan, reinterpret_cast<cudaStream_t>(stream));
+}
+
+extern "C" rl_status rl_policy_loss_fwd_bwd(const void* logits, rl_dtype dtype, int64_t rows, int64_t V,
+                                            int64_t ld, const int32_t* token_ids, const uint8_t* mask,
+                                            const int32_t* token_traj, int32_t n_traj, const float* adv,
+                                            const float* coef, const float* old_logp, const float* ref_logp,
+                                            const float* rollout_logp, const rl_loss_params* params,
+                                            void* grad_out, double* loss_accum, float* token_stats, void* ws,
+                                            size_t ws_bytes, rl_stream_t stream) {
+  using namespace rl;
+  clear_error();
+  Plan plan;
+  int es = 0;
+  rl_status st = check_rows_args("rl_policy_loss_fwd_bwd", logits, dtype, rows, V, ld, ws, ws_bytes, &plan, &es);
+  if (st != RL_OK) return st;
+  if (!params) return set_error(RL_ERR_INVALID_ARG, "rl_policy_loss_fwd_bwd: params is NULL");
+  if (!(params->clip_eps_low >= 0.f) || !(params->clip_eps_high >= 0.f))
+    return set_error(RL_ERR_INVALID_ARG, "rl_policy_loss_fwd_bwd: clip eps must be >= 0");
+  if (params->kl_estimator != 0 && params->kl_estimator != 3)
+    return set_error(RL_ERR_UNSUPPORTED, "rl_policy_loss_fwd_bwd: kl_estimator must be 0 or 3");
+  if (!loss_accum) return set_error(RL_ERR_INVALID_ARG, "rl_policy_loss_fwd_bwd: loss_accum is NULL");
+  if (n_traj < 0) return set_error(RL_ERR_INVALID_ARG, "rl_policy_loss_fwd_bwd: n_traj < 0");
+  if (rows == 0) return RL_OK;
+  if (!token_ids || !mask || !token_traj || !old_logp || !grad_out || (n_traj > 0 && (!adv || !coef)))
+    return set_error(RL_ERR_INVALID_ARG, "rl_policy_loss_fwd_bwd: NULL array argument");
+  if (!aligned16(grad_out)) return set_error(RL_ERR_ALIGNMENT, "rl_policy_loss_fwd_bwd: grad_out not 16-byte aligned");
+  const bool kl_on = params->kl_estimator == 3 && params->kl_coef != 0.f && ref_logp != nullptr;
+  RowArgs a = {};
+  a.logits = logits;
+  a.grad = grad_out;
+  a.rows = rows;
+  a.V = V;
+  a.ld = ld;
+  a.token_ids = token_ids;
+  a.mask = mask;
+  a.token_traj = token_traj;
+  a.n_traj = n_traj;
+  a.adv = adv;
+  a.coef = coef;
+  a.old_logp = old_logp;
+  a.ref_logp = kl_on ? ref_logp : nullptr;
+  a.rollout_logp = rollout_logp;
+  a.clip_lo = 1.f - params->clip_eps_low;
+  a.clip_hi = 1.f + params->clip_eps_high;
+  a.beta = kl_on ? params->kl_coef : 0.f;
+  a.alpha = params->entropy_coef;
+  a.tis_cap = rollout_logp ? params->tis_cap : 0.f;
+  double* row_loss = reinterpret_cast<double*>(static_cast<char*>(ws) + ws_row_loss_offset());
+  a.row_loss = row_loss;
+  a.token_stats = token_stats;
+  a.status = reinterpret_cast<int32_t*>(ws);
+  a.slice = plan.slice;
+  a.buf_elems = plan.buf_elems;
+  a.tma = ((ld * es) % 16) == 0;
+  const bool ent = params->entropy_coef != 0.f || token_stats != nullptr;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  st = dispatch_rows<true>(dtype, ent, a, plan, s);
+  if (st != RL_OK) return st;
+  reduce_loss_kernel<<<1, 1024, 0, s>>>(row_loss, rows, loss_accum);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_error(e, "reduce_loss_kernel launch");
+  return RL_OK;
+}

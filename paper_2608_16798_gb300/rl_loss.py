@@ -1,0 +1,250 @@
+"""Thin Python binding of the C ABI in ``include/rl_loss.h``.
+
+Argument marshalling only: each function checks the tensors it is handed
+(device, dtype, size, contiguity), passes their device pointers and the
+current CUDA stream to the library function of the same name, and raises
+``RLError`` on a non-OK status. Every step of the computation runs in the
+library's CUDA kernels; there is no fallback path. PyTorch only owns memory
+and streams.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "librl_loss.so")
+
+RL_OK = 0
+STATUS_NAMES = {0: "RL_OK", 1: "RL_ERR_INVALID_ARG", 2: "RL_ERR_UNSUPPORTED", 3: "RL_ERR_ALIGNMENT",
+                4: "RL_ERR_WORKSPACE_TOO_SMALL", 5: "RL_ERR_CUDA", 6: "RL_ERR_DEVICE_CHECK", 7: "RL_ERR_TIMEOUT"}
+RL_BF16, RL_F32 = 0, 1
+RL_DEV_BAD_TOKEN, RL_DEV_BAD_TRAJ, RL_DEV_BAD_OFFSETS, RL_DEV_TIMEOUT = 1, 2, 4, 8
+AGG_SEQ_MEAN_TOKEN_MEAN, AGG_TOKEN_MEAN, AGG_TOKEN_SUM = 0, 1, 2
+
+# C function name -> (restype, argtypes)
+_P = ctypes.c_void_p
+_I32, _I64, _SZ, _F = ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t, ctypes.c_float
+EXPORTS = {
+    "rl_version": (_I32, []),
+    "rl_last_error_message": (ctypes.c_char_p, []),
+    "rl_workspace_size": (_SZ, [_I64, _I64, _I64]),
+    "rl_workspace_init": (_I32, [_P, _SZ, _P]),
+    "rl_query_status": (_I32, [_P, _P, ctypes.POINTER(_I32)]),
+    "rl_group_advantages": (_I32, [_I32, _I32, _P, _P, _P, _I64, _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P]),
+    "rl_token_logprobs": (_I32, [_P, _I32, _I64, _I64, _I64, _P, _P, _P, _P, _P, _SZ, _P]),
+    "rl_policy_loss_fwd_bwd": (_I32, [_P, _I32, _I64, _I64, _I64, _P, _P, _P, _I32, _P, _P, _P, _P, _P, _P,
+                                      _P, _P, _P, _P, _SZ, _P]),
+}
+
+
+class rl_loss_params(ctypes.Structure):
+    _fields_ = [("clip_eps_low", _F), ("clip_eps_high", _F), ("kl_coef", _F), ("kl_estimator", _I32),
+                ("entropy_coef", _F), ("tis_cap", _F), ("adv_eps", _F), ("loss_agg", _I32)]
+
+
+def make_params(clip_eps_low=0.2, clip_eps_high=0.28, kl_coef=0.0, kl_estimator=0, entropy_coef=0.0,
+                tis_cap=0.0, adv_eps=1e-6, loss_agg=AGG_SEQ_MEAN_TOKEN_MEAN) -> rl_loss_params:
+    return rl_loss_params(clip_eps_low, clip_eps_high, kl_coef, kl_estimator, entropy_coef, tis_cap, adv_eps,
+                          loss_agg)
+
+
+class RLError(RuntimeError):
+    def __init__(self, fn, status, message):
+        super().__init__(f"{fn}: {STATUS_NAMES.get(status, status)}: {message}")
+        self.status = status
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """Load ``librl_loss.so`` (built by ``build.py``); raises if it is missing."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is missing: build it with paper_2608_16798_gb300.build.build()")
+        handle = ctypes.CDLL(LIB_PATH)
+        for name, (res, args) in EXPORTS.items():
+            f = getattr(handle, name)
+            f.restype = res
+            f.argtypes = args
+        _lib = handle
+    return _lib
+
+
+def _check(fn, st):
+    if st != RL_OK:
+        msg = lib().rl_last_error_message()
+        raise RLError(fn, st, msg.decode() if msg else "")
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _need(t, name, dtype, numel=None, device=None):
+    if t is None:
+        raise ValueError(f"{name} is required")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if numel is not None and t.numel() < numel:
+        raise ValueError(f"{name} has {t.numel()} elements, needs {numel}")
+    if device is not None and t.device != device:
+        raise ValueError(f"{name} is on {t.device}, expected {device}")
+    return t
+
+
+def _opt(t, name, dtype, numel=None, device=None):
+    return None if t is None else _need(t, name, dtype, numel, device)
+
+
+def _logits_dtype(t):
+    if t.dtype == torch.bfloat16:
+        return RL_BF16
+    if t.dtype == torch.float32:
+        return RL_F32
+    raise ValueError(f"logits must be bfloat16 or float32, got {t.dtype}")
+
+
+def _rows_view(logits):
+    if logits.dim() != 2 or logits.stride(1) != 1:
+        raise ValueError("logits must be a 2-D tensor with unit stride along the vocabulary")
+    return logits.shape[0], logits.shape[1], logits.stride(0)
+
+
+# ----------------------------------------------------------------------------- ABI functions
+
+def rl_version() -> int:
+    return int(lib().rl_version())
+
+
+def rl_last_error_message() -> str:
+    m = lib().rl_last_error_message()
+    return m.decode() if m else ""
+
+
+def rl_workspace_size(max_rows: int, V: int, D: int = 0) -> int:
+    return int(lib().rl_workspace_size(max_rows, V, D))
+
+
+def rl_workspace_init(ws: torch.Tensor, stream=None):
+    _need(ws, "ws", torch.uint8)
+    _check("rl_workspace_init", lib().rl_workspace_init(_ptr(ws), ws.numel(), _stream(stream)))
+
+
+def new_workspace(max_rows: int, V: int, D: int = 0, device=None, stream=None) -> torch.Tensor:
+    """Allocate (with torch) and initialise a workspace for calls of up to max_rows rows."""
+    ws = torch.empty(rl_workspace_size(max_rows, V, D), dtype=torch.uint8, device=device or "cuda")
+    rl_workspace_init(ws, stream)
+    return ws
+
+
+def rl_query_status(ws: torch.Tensor, stream=None):
+    """Synchronise the stream and return (status, device_status_word)."""
+    word = ctypes.c_int32(0)
+    st = lib().rl_query_status(_ptr(ws), _stream(stream), ctypes.byref(word))
+    if st not in (RL_OK, 6, 7):
+        _check("rl_query_status", st)
+    return st, int(word.value)
+
+
+def rl_group_advantages(group_offsets, rewards, traj_offsets, mask, params: rl_loss_params, ws,
+                        traj_valid=None, adv_out=None, coef_out=None, n_tok_out=None, token_traj_out=None,
+                        want_token_traj=True, stream=None):
+    """Advantages A_i, coefficients c_i, counts L_i (and token owners) for a packed batch."""
+    dev = rewards.device
+    n_traj = rewards.numel()
+    n_groups = group_offsets.numel() - 1
+    n_tokens = mask.numel()
+    _need(rewards, "rewards", torch.float32, device=dev)
+    _need(group_offsets, "group_offsets", torch.int32, device=dev)
+    _need(traj_offsets, "traj_offsets", torch.int64, n_traj + 1, device=dev)
+    _need(mask, "mask", torch.uint8, device=dev)
+    _opt(traj_valid, "traj_valid", torch.uint8, n_traj, device=dev)
+    adv_out = torch.empty(n_traj, dtype=torch.float32, device=dev) if adv_out is None else adv_out
+    coef_out = torch.empty(n_traj, dtype=torch.float32, device=dev) if coef_out is None else coef_out
+    n_tok_out = torch.empty(n_traj, dtype=torch.int32, device=dev) if n_tok_out is None else n_tok_out
+    if want_token_traj and token_traj_out is None:
+        token_traj_out = torch.empty(n_tokens, dtype=torch.int32, device=dev)
+    _need(adv_out, "adv_out", torch.float32, n_traj, device=dev)
+    _need(coef_out, "coef_out", torch.float32, n_traj, device=dev)
+    _need(n_tok_out, "n_tok_out", torch.int32, n_traj, device=dev)
+    _opt(token_traj_out, "token_traj_out", torch.int32, n_tokens, device=dev)
+    _need(ws, "ws", torch.uint8, device=dev)
+    st = lib().rl_group_advantages(n_traj, n_groups, _ptr(group_offsets), _ptr(rewards), _ptr(traj_valid),
+                                   n_tokens, _ptr(traj_offsets), _ptr(mask), ctypes.byref(params), _ptr(adv_out),
+                                   _ptr(coef_out), _ptr(n_tok_out), _ptr(token_traj_out), _ptr(ws), ws.numel(),
+                                   _stream(stream))
+    _check("rl_group_advantages", st)
+    return adv_out, coef_out, n_tok_out, token_traj_out
+
+
+def rl_token_logprobs(logits, token_ids, ws, logp_out=None, entropy_out=None, lse_out=None,
+                      want_entropy=False, want_lse=False, stream=None):
+    """logp of the sampled ids (and optionally entropy, lse) for every logits row."""
+    rows, V, ld = _rows_view(logits)
+    dt = _logits_dtype(logits)
+    dev = logits.device
+    _need(token_ids, "token_ids", torch.int32, rows, device=dev)
+    logp_out = torch.empty(rows, dtype=torch.float32, device=dev) if logp_out is None else logp_out
+    if want_entropy and entropy_out is None:
+        entropy_out = torch.empty(rows, dtype=torch.float32, device=dev)
+    if want_lse and lse_out is None:
+        lse_out = torch.empty(rows, dtype=torch.float32, device=dev)
+    _need(logp_out, "logp_out", torch.float32, rows, device=dev)
+    _opt(entropy_out, "entropy_out", torch.float32, rows, device=dev)
+    _opt(lse_out, "lse_out", torch.float32, rows, device=dev)
+    _need(ws, "ws", torch.uint8, device=dev)
+    st = lib().rl_token_logprobs(_ptr(logits), dt, rows, V, ld, _ptr(token_ids), _ptr(logp_out), _ptr(entropy_out),
+                                 _ptr(lse_out), _ptr(ws), ws.numel(), _stream(stream))
+    _check("rl_token_logprobs", st)
+    return logp_out, entropy_out, lse_out
+
+
+def rl_policy_loss_fwd_bwd(logits, token_ids, mask, token_traj, adv, coef, old_logp, params: rl_loss_params, ws,
+                           loss_accum, grad_out=None, ref_logp=None, rollout_logp=None, token_stats=None,
+                           stream=None):
+    """Adds the microbatch loss to ``loss_accum`` (float64 [1]) and writes d loss / d logits.
+
+    ``grad_out`` defaults to a new tensor shaped like ``logits``; pass ``logits`` itself
+    for an in-place gradient. Returns grad_out.
+    """
+    rows, V, ld = _rows_view(logits)
+    dt = _logits_dtype(logits)
+    dev = logits.device
+    n_traj = adv.numel()
+    _need(token_ids, "token_ids", torch.int32, rows, device=dev)
+    _need(mask, "mask", torch.uint8, rows, device=dev)
+    _need(token_traj, "token_traj", torch.int32, rows, device=dev)
+    _need(adv, "adv", torch.float32, device=dev)
+    _need(coef, "coef", torch.float32, n_traj, device=dev)
+    _need(old_logp, "old_logp", torch.float32, rows, device=dev)
+    _opt(ref_logp, "ref_logp", torch.float32, rows, device=dev)
+    _opt(rollout_logp, "rollout_logp", torch.float32, rows, device=dev)
+    _need(loss_accum, "loss_accum", torch.float64, 1, device=dev)
+    _opt(token_stats, "token_stats", torch.float32, rows * 5, device=dev)
+    if grad_out is None:
+        grad_out = torch.empty_strided(logits.shape, logits.stride(), dtype=logits.dtype, device=dev)
+    if grad_out.dtype != logits.dtype or grad_out.shape != logits.shape or grad_out.stride() != logits.stride():
+        raise ValueError("grad_out must match logits in dtype, shape and strides")
+    _need(ws, "ws", torch.uint8, device=dev)
+    st = lib().rl_policy_loss_fwd_bwd(_ptr(logits), dt, rows, V, ld, _ptr(token_ids), _ptr(mask), _ptr(token_traj),
+                                      n_traj, _ptr(adv), _ptr(coef), _ptr(old_logp), _ptr(ref_logp),
+                                      _ptr(rollout_logp), ctypes.byref(params), _ptr(grad_out), _ptr(loss_accum),
+                                      _ptr(token_stats), _ptr(ws), ws.numel(), _stream(stream))
+    _check("rl_policy_loss_fwd_bwd", st)
+    return grad_out

@@ -1,0 +1,174 @@
+"""Shared helpers for the GPU parity tests: seeded cases from the workload
+generators, the oracle's answers, the CUDA path's answers, and the tolerance
+checks.
+
+Inputs flow one way: the generators draw logits, ids, masks, rewards and noise;
+the oracle computes its own advantages, coefficients and log-probs (old_logp =
+oracle logp - noise); the CUDA path receives the same float32 / bf16 arrays.
+No value computed by the CUDA path is ever fed to the oracle.
+
+Tolerances (float32 kernels against the float64 oracle):
+  loss       |d| <= 1e-4 * max(|L|, sum_t |c l_t|)
+  gradient   |d| <= 2e-3 absolute (paper's weighting; not for token-sum, c = 1), and the tighter
+             |d| <= fmt * |g| + 2e-5 * |g| + 2e-5 * s_row, s_row = max(max_v |g_row|,
+             the row's coefficient size |c| (w |A| rho + beta |1 - e^(r-logp)| + alpha (1 + |H|)))
+             with fmt = 2^-8 for bf16 output (half an ulp of an 8-bit significand)
+             and 2^-23 for float32 output
+  logp       |d| <= 1e-5 + 2^-22 |logp|   (2^-22: float32 ulp at -1e4 rows)
+  ratio      |d| <= 2e-5 * rho
+  entropy    |d| <= 5e-5 + 2e-5 |H|
+  KL         |d| <= 1e-6 + 1e-4 |KL|
+  clipped flag, token owners, counts, masked / inactive rows: bit-exact
+"""
+
+from __future__ import annotations
+
+import dataclasses
+
+import numpy as np
+import torch
+
+import oracle.grpo_objective as O
+from paper_2608_16798_gb300 import workloads as W
+
+GRAD_ABS = 2e-3
+
+
+def loss_params(w: W.Workload, loss_agg=0, tis_cap=0.0):
+    return O.LossParams(clip_eps_low=W.CLIP_EPS_LOW, clip_eps_high=W.CLIP_EPS_HIGH, kl_coef=w.kl_coef,
+                        kl_estimator=3 if w.kl_coef else 0, entropy_coef=w.entropy_coef, tis_cap=tis_cap,
+                        adv_eps=1e-6, loss_agg=loss_agg)
+
+
+def cuda_params(R, P: O.LossParams):
+    return R.make_params(P.clip_eps_low, P.clip_eps_high, P.kl_coef, P.kl_estimator, P.entropy_coef, P.tis_cap,
+                         P.adv_eps, P.loss_agg)
+
+
+@dataclasses.dataclass
+class Case:
+    w: W.Workload
+    layout: W.Layout
+    row0: int
+    raw: np.ndarray          # uint16 (bf16 bits) or float32 [rows, V]
+    ids: np.ndarray          # int32 [rows]
+    old: np.ndarray          # float32 [rows]
+    ref: np.ndarray | None
+    roll: np.ndarray | None
+    P: O.LossParams
+    adv64: np.ndarray        # oracle advantages (float64, whole batch)
+    coef64: np.ndarray
+    L: np.ndarray
+    token_traj: np.ndarray   # oracle owners (whole batch)
+
+    @property
+    def rows(self):
+        return self.raw.shape[0]
+
+    @property
+    def sl(self):
+        return slice(self.row0, self.row0 + self.rows)
+
+    @property
+    def mask(self):
+        return self.layout.mask[self.sl]
+
+    @property
+    def tt(self):
+        return self.token_traj[self.sl]
+
+
+def make_case(name, seed=0, row0=0, rows=None, vocab=None, n_groups=None, loss_agg=0, tis=False,
+              invalid_frac=0.0, logit_std=None):
+    w = W.WORKLOADS[name]
+    over = {}
+    if vocab is not None:
+        over["vocab"] = vocab
+    if logit_std is not None:
+        over["logit_std"] = logit_std
+    if over:
+        w = dataclasses.replace(w, **over)
+    layout = W.make_layout(w, seed, n_groups)
+    if invalid_frac > 0:
+        rng = np.random.default_rng(seed + 77)
+        layout.traj_valid = (rng.random(layout.n_traj) >= invalid_frac).astype(np.uint8)
+    T = layout.n_tokens
+    rows = T - row0 if rows is None else min(rows, T - row0)
+    raw, vals = W.logits_rows_np(w, seed, row0, rows)
+    ids = W.sample_tokens_np(vals, seed, row0, w)
+    logp, _, _ = O.token_logprobs(raw, w.dtype, ids)
+    old = W.old_logp_from(logp, w, seed, row0)
+    ref = W.ref_logp_from(logp, w, seed, row0) if w.ref_noise_std else None
+    roll = W.rollout_logp_from(old, seed, row0=row0) if tis else None
+    P = loss_params(w, loss_agg, tis_cap=2.0 if tis else 0.0)
+    adv, coef, L, tt = O.advantages_and_coefficients(layout.rewards, layout.group_offsets, layout.traj_offsets,
+                                                     layout.mask, layout.traj_valid, P)
+    return Case(w, layout, row0, raw, ids, old, ref, roll, P, adv, coef, L, tt)
+
+
+def oracle_loss(case: Case, adv=None, coef=None, rows=None, want_grad=True):
+    adv = case.adv64 if adv is None else adv
+    coef = case.coef64 if coef is None else coef
+    return O.policy_loss_fwd_bwd(case.raw, case.w.dtype, case.ids, case.mask, case.tt, adv, coef, case.old, case.P,
+                                 case.ref, case.roll, want_grad=want_grad, rows=rows)
+
+
+def to_dev(x, dtype=None, device="cuda"):
+    t = torch.from_numpy(np.ascontiguousarray(x))
+    if dtype is not None:
+        t = t.to(dtype)
+    return t.to(device)
+
+
+def logits_to_dev(case: Case, ld=None, device="cuda"):
+    V = case.raw.shape[1]
+    ld = V if ld is None else ld
+    if case.w.dtype == "bf16":
+        host = torch.from_numpy(case.raw.view(np.int16).copy()).view(torch.bfloat16)
+    else:
+        host = torch.from_numpy(case.raw.copy())
+    if ld == V:
+        return host.to(device)
+    full = torch.full((case.rows, ld), float("nan"), dtype=host.dtype, device=device)
+    full[:, :V] = host.to(device)
+    return full[:, :V]
+
+
+def grad_to_np(g):
+    if g.dtype == torch.bfloat16:
+        return g.float().cpu().numpy().astype(np.float64)
+    return g.cpu().numpy().astype(np.float64)
+
+
+def check_grad(g_dev, g_ref, dtype, what="", row_scale=None, absolute=True):
+    """absolute=False for token-sum weighting (c = 1), where gradient elements are O(1) and
+    the 2e-3 absolute bound is below half a bf16 ulp; the relative bound still applies."""
+    d = np.abs(g_dev - g_ref)
+    if absolute:
+        assert d.max(initial=0.0) <= GRAD_ABS, f"{what}: max |dgrad| {d.max()} above {GRAD_ABS}"
+    fmt = 2.0 ** -8 if dtype == "bf16" else 2.0 ** -23
+    rs = np.abs(g_ref).max(axis=1, keepdims=True) if g_ref.size else np.zeros((g_ref.shape[0], 1))
+    row_scale = rs if row_scale is None else np.maximum(rs, row_scale)
+    tol = (fmt + 2e-5) * np.abs(g_ref) + 2e-5 * row_scale + 1e-30
+    bad = d > tol
+    if bad.any():
+        r, v = np.argwhere(bad)[0]
+        raise AssertionError(f"{what}: {bad.sum()} elements out of tolerance; first row {r} col {v}: "
+                             f"gpu {g_dev[r, v]!r} oracle {g_ref[r, v]!r} tol {tol[r, v]!r}")
+
+
+def check_loss(loss_dev, loss_ref, contrib_ref, what=""):
+    scale = max(abs(loss_ref), float(np.abs(contrib_ref).sum()))
+    assert abs(loss_dev - loss_ref) <= 1e-4 * scale + 1e-300, f"{what}: loss {loss_dev} vs {loss_ref} (scale {scale})"
+
+
+def check_stats(st_dev, st_ref, active, what=""):
+    st_dev = st_dev.astype(np.float64)
+    assert np.all(st_dev[~active] == 0.0), f"{what}: stats of inactive rows not zero"
+    a, b = st_dev[active], st_ref[active]
+    d = np.abs(a - b)
+    assert np.all(d[:, 0] <= 1e-5 + 2.0 ** -22 * np.abs(b[:, 0])), f"{what}: logp max diff {d[:, 0].max()}"
+    assert np.all(d[:, 1] <= 2e-5 * np.abs(b[:, 1])), f"{what}: ratio max rel diff {(d[:, 1] / b[:, 1]).max()}"
+    assert np.array_equal(a[:, 2], b[:, 2]), f"{what}: clipped flags differ"
+    assert np.all(d[:, 3] <= 5e-5 + 2e-5 * np.abs(b[:, 3])), f"{what}: entropy max diff {d[:, 3].max()}"
+    assert np.all(d[:, 4] <= 1e-6 + 1e-4 * np.abs(b[:, 4])), f"{what}: KL max diff {d[:, 4].max()}"

@@ -1,0 +1,142 @@
+"""Host-only checks of the C ABI: the library builds and loads, exports every
+function that include/rl_loss.h declares, and rejects bad arguments before
+launching anything (no GPU needed: every call here returns during argument
+validation, before the first CUDA runtime call)."""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2608_16798_gb300 import build as B
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADERS = [os.path.join(ROOT, "include", f) for f in os.listdir(os.path.join(ROOT, "include")) if f.endswith(".h")]
+
+
+@pytest.fixture(scope="module")
+def R():
+    B.build()
+    import paper_2608_16798_gb300.rl_loss as R
+
+    R.lib()
+    return R
+
+
+def declared_functions():
+    names = []
+    for h in HEADERS:
+        src = open(h).read()
+        src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+        src = re.sub(r"//[^\n]*", "", src)
+        names += re.findall(r"\b(rl_[a-z0-9_]+)\s*\(", src)
+    return sorted(set(names))
+
+
+def test_header_declares_the_four_path_functions():
+    names = declared_functions()
+    for f in ("rl_group_advantages", "rl_token_logprobs", "rl_policy_loss_fwd_bwd"):
+        assert f in names
+
+
+def test_every_declared_function_is_exported(R):
+    handle = ctypes.CDLL(R.LIB_PATH)
+    missing = [n for n in declared_functions() if not hasattr(handle, n)]
+    assert not missing, missing
+    # and the binding knows each of them
+    assert set(declared_functions()) <= set(R.EXPORTS)
+
+
+def test_version_and_workspace_size(R):
+    assert R.rl_version() >= 10000
+    assert R.rl_workspace_size(0, 0) == 256
+    assert R.rl_workspace_size(16384, 151936) == 256 + 16384 * 8
+    assert R.rl_workspace_size(3, 10) == 256 + 256
+
+
+FAKE = 0x10000  # never dereferenced: every call below fails validation first
+PARAMS = None
+
+
+def _params(R, **kw):
+    return ctypes.byref(R.make_params(**kw))
+
+
+def _loss(R, **over):
+    L = R.lib()
+    a = dict(logits=FAKE, dt=R.RL_BF16, rows=4, V=8, ld=8, ids=FAKE, mask=FAKE, tt=FAKE, n_traj=2, adv=FAKE,
+             coef=FAKE, old=FAKE, ref=None, roll=None, params=_params(R), grad=FAKE, loss=FAKE, stats=None,
+             ws=FAKE, ws_bytes=1 << 20, stream=None)
+    a.update(over)
+    return L.rl_policy_loss_fwd_bwd(a["logits"], a["dt"], a["rows"], a["V"], a["ld"], a["ids"], a["mask"], a["tt"],
+                                    a["n_traj"], a["adv"], a["coef"], a["old"], a["ref"], a["roll"], a["params"],
+                                    a["grad"], a["loss"], a["stats"], a["ws"], a["ws_bytes"], a["stream"])
+
+
+def test_policy_loss_argument_checks(R):
+    assert _loss(R, dt=7) == 1
+    assert _loss(R, rows=-1) == 1
+    assert _loss(R, V=0) == 1
+    assert _loss(R, ld=7) == 1
+    assert _loss(R, ws=None) == 1
+    assert _loss(R, ws_bytes=100) == 4
+    assert _loss(R, logits=FAKE + 2) == 3
+    assert _loss(R, grad=FAKE + 8) == 3
+    assert _loss(R, ws=FAKE + 4) == 3
+    assert _loss(R, params=None) == 1
+    assert _loss(R, params=_params(R, kl_estimator=2)) == 2
+    assert _loss(R, params=_params(R, clip_eps_low=-0.1)) == 1
+    assert _loss(R, loss=None) == 1
+    assert _loss(R, ids=None) == 1
+    assert _loss(R, n_traj=-1) == 1
+    assert _loss(R, V=10_000_000, ld=10_000_000) == 2  # row larger than 16 CTAs x 100 KB
+    assert "rl_policy_loss_fwd_bwd" in R.rl_last_error_message()
+    assert _loss(R, rows=0) == 0      # nothing to do: returns before any launch
+
+
+def test_token_logprobs_argument_checks(R):
+    L = R.lib()
+
+    def call(**over):
+        a = dict(logits=FAKE, dt=R.RL_F32, rows=4, V=8, ld=8, ids=FAKE, logp=FAKE, ent=None, lse=None, ws=FAKE,
+                 ws_bytes=1 << 20, stream=None)
+        a.update(over)
+        return L.rl_token_logprobs(a["logits"], a["dt"], a["rows"], a["V"], a["ld"], a["ids"], a["logp"], a["ent"],
+                                   a["lse"], a["ws"], a["ws_bytes"], a["stream"])
+
+    assert call(dt=3) == 1
+    assert call(ld=4) == 1
+    assert call(logp=None) == 1
+    assert call(logits=FAKE + 4) == 3
+    assert call(ws_bytes=8) == 4
+    assert call(rows=0) == 0
+
+
+def test_group_advantages_argument_checks(R):
+    L = R.lib()
+
+    def call(**over):
+        a = dict(n=4, g=1, go=FAKE, rw=FAKE, valid=None, T=16, to=FAKE, mask=FAKE, params=_params(R), adv=FAKE,
+                 coef=FAKE, ntok=FAKE, tt=None, ws=FAKE, ws_bytes=1024, stream=None)
+        a.update(over)
+        return L.rl_group_advantages(a["n"], a["g"], a["go"], a["rw"], a["valid"], a["T"], a["to"], a["mask"],
+                                     a["params"], a["adv"], a["coef"], a["ntok"], a["tt"], a["ws"], a["ws_bytes"],
+                                     a["stream"])
+
+    assert call(n=-1) == 1
+    assert call(params=None) == 1
+    assert call(params=_params(R, loss_agg=5)) == 1
+    assert call(params=_params(R, adv_eps=-1.0)) == 1
+    assert call(ws_bytes=16) == 4
+    assert call(rw=None) == 1
+    assert call(mask=None) == 1
+    assert call(n=0) == 0
+
+
+def test_status_and_init_argument_checks(R):
+    L = R.lib()
+    assert L.rl_workspace_init(None, 1024, None) == 1
+    assert L.rl_workspace_init(FAKE, 16, None) == 4
+    word = ctypes.c_int32(0)
+    assert L.rl_query_status(None, None, ctypes.byref(word)) == 1

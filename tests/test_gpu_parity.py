@@ -1,0 +1,251 @@
+"""CUDA path against the float64 oracle on seeded inputs (needs a GB300).
+
+Sizes here let the oracle finish in seconds while spanning many tiles, all
+cluster widths the launcher picks (1, 4, 8 and 16 CTAs per row), ragged
+vocabulary tails, unaligned leading dimensions and the degenerate cases.
+Full-size workloads are in test_gpu_fullsize.py.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+import oracle.grpo_objective as O
+from parity_cases import (GRAD_ABS, check_grad, check_loss, check_stats, cuda_params, grad_to_np, logits_to_dev,
+                          make_case, oracle_loss, to_dev)
+from paper_2608_16798_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def R():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_16798_gb300 import build
+
+    build.build()
+    import paper_2608_16798_gb300.rl_loss as R
+
+    R.lib()
+    return R
+
+
+def run_loss(R, case, adv32=None, coef32=None, ld=None, in_place=False, stats=True, ws=None):
+    dev = "cuda"
+    logits = logits_to_dev(case, ld)
+    adv32 = case.adv64.astype(np.float32) if adv32 is None else adv32
+    coef32 = case.coef64.astype(np.float32) if coef32 is None else coef32
+    ws = R.new_workspace(case.rows, case.raw.shape[1]) if ws is None else ws
+    loss = torch.zeros(1, dtype=torch.float64, device=dev)
+    st = torch.zeros(case.rows * 5, dtype=torch.float32, device=dev) if stats else None
+    g = R.rl_policy_loss_fwd_bwd(logits, to_dev(case.ids), to_dev(case.mask), to_dev(case.tt.astype(np.int32)),
+                                 to_dev(adv32), to_dev(coef32), to_dev(case.old), cuda_params(R, case.P), ws, loss,
+                                 grad_out=logits if in_place else None,
+                                 ref_logp=None if case.ref is None else to_dev(case.ref),
+                                 rollout_logp=None if case.roll is None else to_dev(case.roll), token_stats=st)
+    status, word = R.rl_query_status(ws)
+    return dict(loss=float(loss.item()), grad=grad_to_np(g), stats=None if st is None else st.view(-1, 5).cpu().numpy(),
+                status=status, word=word)
+
+
+def grad_scale(case, stats, adv, coef):
+    """Per-row size of the gradient's coefficients |c| (w |A| rho + beta |1 - e^(r - logp)| + alpha (1 + |H|)),
+    the scale of the float32 rounding in a row (used only as an error floor)."""
+    c = np.abs(coef[case.tt])
+    A = np.abs(adv[case.tt])
+    rho, H, logp = stats[:, 1], stats[:, 3], stats[:, 0]
+    w = np.ones_like(rho)
+    if case.roll is not None and case.P.tis_cap > 0:
+        w = np.minimum(np.exp(case.old.astype(np.float64) - case.roll), case.P.tis_cap)
+    kl = 0.0
+    if case.ref is not None and case.P.kl_coef:
+        kl = case.P.kl_coef * np.abs(1 - np.exp(np.clip(case.ref - logp, -50, 50)))
+    return (c * (w * A * rho + kl + case.P.entropy_coef * (1 + np.abs(H))))[:, None]
+
+
+def compare(case, out, what):
+    adv32 = case.adv64.astype(np.float32).astype(np.float64)
+    coef32 = case.coef64.astype(np.float32).astype(np.float64)
+    loss, grad, stats, contrib = oracle_loss(case, adv32, coef32)
+    check_loss(out["loss"], loss, contrib, what)
+    check_grad(out["grad"], grad, case.w.dtype, what, row_scale=grad_scale(case, stats, adv32, coef32),
+               absolute=case.P.loss_agg != O.AGG_TOKEN_SUM)
+    active = (case.mask != 0) & (coef32[case.tt] != 0)
+    assert np.all(out["grad"][~active] == 0.0), f"{what}: inactive rows not exactly zero"
+    if out["stats"] is not None:
+        check_stats(out["stats"], stats, active, what)
+    assert out["word"] == 0, f"{what}: device status {out['word']}"
+
+
+# ----------------------------------------------------------------------------- A1..A3
+
+@pytest.mark.parametrize("name,n_groups,invalid,agg", [
+    ("tiny", None, 0.0, 0), ("multiturn", None, 0.0, 0), ("longhorizon", None, 0.0, 0), ("edge", None, 0.0, 0),
+    ("multiturn", None, 0.2, 0), ("edge", 512, 0.1, 1), ("longhorizon", None, 0.1, 2)])
+def test_group_advantages_parity(R, name, n_groups, invalid, agg):
+    case_w = W.WORKLOADS[name]
+    lay = W.make_layout(case_w, 3, n_groups)
+    if invalid:
+        lay.traj_valid = (np.random.default_rng(5).random(lay.n_traj) >= invalid).astype(np.uint8)
+    P = O.LossParams(loss_agg=agg)
+    adv, coef, L, tt = O.advantages_and_coefficients(lay.rewards, lay.group_offsets, lay.traj_offsets, lay.mask,
+                                                     lay.traj_valid, P)
+    ws = R.new_workspace(0, 0)
+    a, c, n_tok, tt_d = R.rl_group_advantages(to_dev(lay.group_offsets), to_dev(lay.rewards), to_dev(lay.traj_offsets),
+                                              to_dev(lay.mask), cuda_params(R, P), ws, traj_valid=to_dev(lay.traj_valid))
+    st, word = R.rl_query_status(ws)
+    assert word == 0
+    assert np.array_equal(n_tok.cpu().numpy(), L), "trainable-token counts must be exact"
+    assert np.array_equal(tt_d.cpu().numpy(), tt), "token owners must be exact"
+    a, c = a.cpu().numpy().astype(np.float64), c.cpu().numpy().astype(np.float64)
+    # double-precision statistics rounded once to float32: within one float32 ulp
+    assert np.all(np.abs(a - adv) <= 2.0 ** -23 * np.abs(adv)), np.abs(a - adv).max()
+    assert np.all(np.abs(c - coef) <= 2.0 ** -23 * np.abs(coef)), np.abs(c - coef).max()
+    assert np.all(a[lay.traj_valid == 0] == 0) and np.all(c[lay.traj_valid == 0] == 0)
+
+
+def test_group_advantages_bad_offsets_flagged(R):
+    go = to_dev(np.array([0, 3, 2], np.int32))   # decreasing
+    rw = to_dev(np.zeros(3, np.float32))
+    to = to_dev(np.array([0, 1, 2, 3], np.int64))
+    mk = to_dev(np.ones(3, np.uint8))
+    ws = R.new_workspace(0, 0)
+    R.rl_group_advantages(go, rw, to, mk, R.make_params(), ws)
+    st, word = R.rl_query_status(ws)
+    assert st == 6 and word & R.RL_DEV_BAD_OFFSETS
+
+
+# ----------------------------------------------------------------------------- B1: token log-probs
+
+@pytest.mark.parametrize("name,row0,rows,vocab,ld_pad", [
+    ("tiny", 0, 512, None, 0), ("multiturn", 700, 48, None, 0), ("edge", 0, 1024, None, 0),
+    ("multiturn", 0, 16, 1001, 0), ("tiny", 0, 40, 4097, 3), ("edge", 0, 64, 999, 5),
+    ("multiturn", 0, 8, 400_000, 0), ("tiny", 0, 7, 1, 0), ("tiny", 0, 9, 3, 8)])
+def test_token_logprobs_parity(R, name, row0, rows, vocab, ld_pad):
+    case = make_case(name, seed=1, row0=row0, rows=rows, vocab=vocab)
+    V = case.raw.shape[1]
+    logits = logits_to_dev(case, V + ld_pad)
+    ws = R.new_workspace(case.rows, V)
+    logp, H, lse = R.rl_token_logprobs(logits, to_dev(case.ids), ws, want_entropy=True, want_lse=True)
+    st, word = R.rl_query_status(ws)
+    assert word == 0
+    lp_ref, H_ref, lse_ref = O.token_logprobs(case.raw, case.w.dtype, case.ids)
+    lp, Hd, ls = (x.cpu().numpy().astype(np.float64) for x in (logp, H, lse))
+    assert np.all(np.abs(lp - lp_ref) <= 1e-5 + 2.0 ** -22 * np.abs(lp_ref)), np.abs(lp - lp_ref).max()
+    assert np.all(np.abs(ls - lse_ref) <= 1e-5 + 2.0 ** -22 * np.abs(lse_ref)), np.abs(ls - lse_ref).max()
+    assert np.all(np.abs(Hd - H_ref) <= 5e-5 + 2e-5 * np.abs(H_ref)), np.abs(Hd - H_ref).max()
+    # without the entropy output the logp path is the same numbers
+    logp2, _, _ = R.rl_token_logprobs(logits, to_dev(case.ids), ws)
+    assert np.all(np.abs(logp2.cpu().numpy() - lp_ref) <= 1e-5 + 2.0 ** -22 * np.abs(lp_ref))
+
+
+def test_token_logprobs_bad_token_flagged(R):
+    case = make_case("tiny", rows=4)
+    ids = case.ids.copy()
+    ids[2] = case.raw.shape[1]
+    ws = R.new_workspace(4, case.raw.shape[1])
+    logp, _, _ = R.rl_token_logprobs(logits_to_dev(case), to_dev(ids), ws)
+    st, word = R.rl_query_status(ws)
+    assert word & R.RL_DEV_BAD_TOKEN
+    lp = logp.cpu().numpy()
+    assert np.isnan(lp[2]) and np.all(np.isfinite(lp[[0, 1, 3]]))
+
+
+# ----------------------------------------------------------------------------- B1..B4: policy loss
+
+@pytest.mark.parametrize("name,row0,rows,agg,tis", [
+    ("tiny", 0, None, 0, False), ("tiny", 0, None, 2, False), ("tiny", 0, None, 2, True),
+    ("multiturn", 1500, 96, 0, False), ("multiturn", 1500, 96, 2, False),
+    ("longhorizon", 5000, 64, 0, False), ("longhorizon", 5000, 64, 2, True),
+    ("edge", 0, 2048, 0, False), ("edge", 4096, 2048, 2, False), ("edge", 0, 2048, 1, True)])
+def test_policy_loss_parity(R, name, row0, rows, agg, tis):
+    case = make_case(name, seed=2, row0=row0, rows=rows, loss_agg=agg, tis=tis)
+    out = run_loss(R, case)
+    compare(case, out, f"{name}[{row0}:+{rows}] agg={agg} tis={tis}")
+
+
+@pytest.mark.parametrize("vocab,ld_pad,dtype_case", [
+    (1001, 0, "multiturn"), (4097, 3, "tiny"), (999, 1, "edge"), (400_000, 0, "multiturn"), (3, 5, "tiny"),
+    (1, 0, "tiny"), (151_936, 16, "multiturn")])
+def test_policy_loss_ragged_shapes(R, vocab, ld_pad, dtype_case):
+    case = make_case(dtype_case, seed=4, rows=24, vocab=vocab, loss_agg=2)
+    out = run_loss(R, case, ld=vocab + ld_pad)
+    compare(case, out, f"V={vocab} ld=V+{ld_pad}")
+
+
+def test_policy_loss_in_place_and_deterministic(R):
+    case = make_case("multiturn", seed=5, row0=300, rows=64, loss_agg=2)
+    a = run_loss(R, case)
+    b = run_loss(R, case, in_place=True)
+    c = run_loss(R, case)
+    assert a["loss"] == c["loss"], "loss must be bit-reproducible"
+    assert np.array_equal(a["grad"], c["grad"]) and np.array_equal(a["grad"], b["grad"])
+    compare(case, b, "in place")
+
+
+def test_policy_loss_microbatch_split(R):
+    case = make_case("longhorizon", seed=6, row0=2000, rows=80, loss_agg=0)
+    whole = run_loss(R, case)
+    parts = []
+    for lo, hi in ((0, 33), (33, 80)):
+        sub = make_case("longhorizon", seed=6, row0=2000 + lo, rows=hi - lo, loss_agg=0)
+        # the same rows: the generator is keyed by row, only the noise streams differ -> reuse the parent's
+        sub.raw, sub.ids, sub.old = case.raw[lo:hi], case.ids[lo:hi], case.old[lo:hi]
+        sub.ref = None if case.ref is None else case.ref[lo:hi]
+        parts.append(run_loss(R, sub))
+    assert abs(sum(p["loss"] for p in parts) - whole["loss"]) <= 1e-12 * max(1e-30, abs(whole["loss"])) + 1e-15
+    assert np.array_equal(np.concatenate([p["grad"] for p in parts]), whole["grad"])
+
+
+def test_policy_loss_all_masked_and_zero_rows(R):
+    case = make_case("tiny", seed=7, rows=64)
+    case.layout.mask[:] = 0
+    out = run_loss(R, case)
+    assert out["loss"] == 0.0 and np.all(out["grad"] == 0.0) and np.all(out["stats"] == 0.0)
+    ws = R.new_workspace(1, 8)
+    loss = torch.full((1,), 3.5, dtype=torch.float64, device="cuda")
+    empty = torch.zeros((0, 8), dtype=torch.bfloat16, device="cuda")
+    z32 = torch.zeros(0, dtype=torch.int32, device="cuda")
+    R.rl_policy_loss_fwd_bwd(empty, z32, torch.zeros(0, dtype=torch.uint8, device="cuda"), z32,
+                             torch.zeros(1, device="cuda"), torch.zeros(1, device="cuda"),
+                             torch.zeros(0, device="cuda"), R.make_params(), ws, loss)
+    assert loss.item() == 3.5
+
+
+def test_policy_loss_bad_ids_flagged_and_zeroed(R):
+    case = make_case("tiny", seed=8, rows=32, loss_agg=2)
+    bad_tok = case.ids.copy()
+    bad_tok[3] = -1
+    tt = case.tt.astype(np.int32).copy()
+    tt[5] = 10_000
+    logits = logits_to_dev(case)
+    ws = R.new_workspace(case.rows, case.raw.shape[1])
+    loss = torch.zeros(1, dtype=torch.float64, device="cuda")
+    g = R.rl_policy_loss_fwd_bwd(logits, to_dev(bad_tok), to_dev(case.mask), to_dev(tt),
+                                 to_dev(case.adv64.astype(np.float32)), to_dev(case.coef64.astype(np.float32)),
+                                 to_dev(case.old), cuda_params(R, case.P), ws, loss)
+    st, word = R.rl_query_status(ws)
+    assert word & R.RL_DEV_BAD_TOKEN and word & R.RL_DEV_BAD_TRAJ
+    gg = grad_to_np(g)
+    assert np.all(gg[[3, 5]] == 0.0) and np.any(gg[0] != 0.0)
+    R.rl_workspace_init(ws)
+    assert R.rl_query_status(ws)[1] == 0
+
+
+def test_end_to_end_advantages_then_loss(R):
+    """GPU advantages feed the GPU loss; the oracle runs A and B in float64 end to end."""
+    case = make_case("longhorizon", seed=9, row0=12000, rows=48, loss_agg=0)
+    lay = case.layout
+    ws = R.new_workspace(case.rows, case.raw.shape[1])
+    adv, coef, n_tok, tt = R.rl_group_advantages(to_dev(lay.group_offsets), to_dev(lay.rewards),
+                                                 to_dev(lay.traj_offsets), to_dev(lay.mask), cuda_params(R, case.P), ws)
+    logits = logits_to_dev(case)
+    loss = torch.zeros(1, dtype=torch.float64, device="cuda")
+    sl = case.sl
+    g = R.rl_policy_loss_fwd_bwd(logits, to_dev(case.ids), to_dev(case.mask), tt[sl.start:sl.stop].contiguous(),
+                                 adv, coef, to_dev(case.old), cuda_params(R, case.P), ws, loss,
+                                 ref_logp=to_dev(case.ref))
+    l_ref, g_ref, _, contrib = oracle_loss(case)
+    check_loss(loss.item(), l_ref, contrib, "end to end")
+    check_grad(grad_to_np(g), g_ref, "bf16", "end to end")
