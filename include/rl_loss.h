@@ -206,6 +206,38 @@ rl_status rl_policy_loss_fwd_bwd(const void* logits, rl_dtype dtype, int64_t row
                                  void* grad_out, double* loss_accum, float* token_stats, void* ws,
                                  size_t ws_bytes, rl_stream_t stream);
 
+/*
+ * Allocation-free form of rl_policy_loss_fwd_bwd (no counterpart in the paper:
+ * it exists for callers that cannot allocate device memory, e.g. code inside a
+ * memory pool that forbids cudaMalloc during a training step, or a plugin that
+ * only receives pointers from its host application).
+ *
+ * Same arguments and results as rl_policy_loss_fwd_bwd, without the workspace:
+ * the library uses its own fixed workspace, a 1 MiB + 256 B array in device
+ * global memory that every GPU loading the library holds until process exit.
+ * The call allocates nothing and calls no allocating routine.
+ *
+ *   rows           at most 131072; larger microbatches return RL_ERR_UNSUPPORTED
+ *                  before anything is launched
+ *   device_status  int32 [1] on the device, or NULL: receives the call's device
+ *                  status word (0 or RL_DEV_* bits) when the call completes on
+ *                  `stream`
+ *
+ * The first call on a device looks up the array's device address (once per
+ * device, with that device current); make that first call before any stream
+ * capture. Every call shares the one array, and each call clears the part that
+ * must start at zero (the status word); calls that overlap on the GPU (for
+ * example on two streams at once) race on it and must be serialised by the
+ * caller.
+ */
+rl_status rl_policy_loss_fwd_bwd_noalloc(const void* logits, rl_dtype dtype, int64_t rows, int64_t V,
+                                         int64_t ld, const int32_t* token_ids, const uint8_t* mask,
+                                         const int32_t* token_traj, int32_t n_traj, const float* adv,
+                                         const float* coef, const float* old_logp, const float* ref_logp,
+                                         const float* rollout_logp, const rl_loss_params* params,
+                                         void* grad_out, double* loss_accum, float* token_stats,
+                                         int32_t* device_status, rl_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -38,6 +38,8 @@ EXPORTS = {
     "rl_token_logprobs": (_I32, [_P, _I32, _I64, _I64, _I64, _P, _P, _P, _P, _P, _SZ, _P]),
     "rl_policy_loss_fwd_bwd": (_I32, [_P, _I32, _I64, _I64, _I64, _P, _P, _P, _I32, _P, _P, _P, _P, _P, _P,
                                       _P, _P, _P, _P, _SZ, _P]),
+    "rl_policy_loss_fwd_bwd_noalloc": (_I32, [_P, _I32, _I64, _I64, _I64, _P, _P, _P, _I32, _P, _P, _P, _P, _P,
+                                              _P, _P, _P, _P, _P, _P]),
 }
 
 
@@ -247,4 +249,39 @@ def rl_policy_loss_fwd_bwd(logits, token_ids, mask, token_traj, adv, coef, old_l
                                       _ptr(rollout_logp), ctypes.byref(params), _ptr(grad_out), _ptr(loss_accum),
                                       _ptr(token_stats), _ptr(ws), ws.numel(), _stream(stream))
     _check("rl_policy_loss_fwd_bwd", st)
+    return grad_out
+
+
+def rl_policy_loss_fwd_bwd_noalloc(logits, token_ids, mask, token_traj, adv, coef, old_logp,
+                                   params: rl_loss_params, loss_accum, grad_out, ref_logp=None, rollout_logp=None,
+                                   token_stats=None, device_status=None, stream=None):
+    """rl_policy_loss_fwd_bwd without a caller workspace, for callers that cannot allocate.
+
+    ``grad_out`` must be provided (this form allocates nothing, not even through torch).
+    ``device_status`` (int32 [1] on the device, optional) receives the call's status word.
+    """
+    rows, V, ld = _rows_view(logits)
+    dt = _logits_dtype(logits)
+    dev = logits.device
+    n_traj = adv.numel()
+    _need(token_ids, "token_ids", torch.int32, rows, device=dev)
+    _need(mask, "mask", torch.uint8, rows, device=dev)
+    _need(token_traj, "token_traj", torch.int32, rows, device=dev)
+    _need(adv, "adv", torch.float32, device=dev)
+    _need(coef, "coef", torch.float32, n_traj, device=dev)
+    _need(old_logp, "old_logp", torch.float32, rows, device=dev)
+    _opt(ref_logp, "ref_logp", torch.float32, rows, device=dev)
+    _opt(rollout_logp, "rollout_logp", torch.float32, rows, device=dev)
+    _need(loss_accum, "loss_accum", torch.float64, 1, device=dev)
+    _opt(token_stats, "token_stats", torch.float32, rows * 5, device=dev)
+    _opt(device_status, "device_status", torch.int32, 1, device=dev)
+    if grad_out is None or grad_out.dtype != logits.dtype or grad_out.shape != logits.shape or \
+            grad_out.stride() != logits.stride():
+        raise ValueError("grad_out must be given and match logits in dtype, shape and strides")
+    st = lib().rl_policy_loss_fwd_bwd_noalloc(_ptr(logits), dt, rows, V, ld, _ptr(token_ids), _ptr(mask),
+                                              _ptr(token_traj), n_traj, _ptr(adv), _ptr(coef), _ptr(old_logp),
+                                              _ptr(ref_logp), _ptr(rollout_logp), ctypes.byref(params),
+                                              _ptr(grad_out), _ptr(loss_accum), _ptr(token_stats),
+                                              _ptr(device_status), _stream(stream))
+    _check("rl_policy_loss_fwd_bwd_noalloc", st)
     return grad_out
