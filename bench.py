@@ -415,6 +415,46 @@ def run_reference(args):
     return 0
 
 
+def profile_case(rows):
+    """A small slice of the workload for profiler captures: the first `rows` packed tokens
+    (logits resident on the device), then three rl_policy_loss_fwd_bwd launches and three
+    rl_token_logprobs launches."""
+    import torch
+
+    from paper_2608_16798_gb300 import build as B
+
+    B.build()
+    import paper_2608_16798_gb300.rl_loss as R
+
+    dev = torch.device("cuda", 0)
+    w = WORKLOAD
+    lay = W.make_layout(w, 0)
+    rows = min(rows, lay.n_tokens)
+    logits = torch.empty((rows, w.vocab), dtype=torch.bfloat16, device=dev)
+    W.logits_rows_torch(w, 0, 0, rows, logits)
+    ids = W.sample_tokens_torch(logits, 0, 0, w)
+    d = lambda x: torch.from_numpy(np.ascontiguousarray(x)).to(dev)  # noqa: E731
+    params = R.make_params()
+    ws = R.new_workspace(rows, w.vocab, device=dev)
+    adv, coef, n_tok, tt = R.rl_group_advantages(d(lay.group_offsets), d(lay.rewards), d(lay.traj_offsets),
+                                                 d(lay.mask), params, ws)
+    logp, _, _ = R.rl_token_logprobs(logits, ids, ws)
+    old = d(W.old_logp_from(logp.cpu().numpy(), w, 0))
+    grad = torch.empty_like(logits)
+    loss = torch.zeros(1, dtype=torch.float64, device=dev)
+    mask = d(lay.mask[:rows])
+    for _ in range(3):
+        R.rl_policy_loss_fwd_bwd(logits, ids, mask, tt[:rows], adv, coef, old, params, ws, loss, grad_out=grad)
+    for _ in range(3):
+        R.rl_token_logprobs(logits, ids, ws, logp_out=logp)
+    st, word = R.rl_query_status(ws)
+    m = lay.mask[:rows].astype(np.int64)
+    print(json.dumps({"profile_case_rows": rows, "trained_rows": int(m.sum()), "status": word,
+                      "algorithmic_bytes_fwd_bwd": int(((m + 1) * w.vocab * 2).sum()),
+                      "algorithmic_bytes_fwd": rows * w.vocab * 2}))
+    return 0 if word == 0 else 1
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -424,7 +464,11 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--profile-case", type=int, default=0, metavar="ROWS",
+                    help="run a small slice of the workload for a profiler capture and exit")
     args = ap.parse_args()
+    if args.profile_case:
+        return profile_case(args.profile_case)
     if args.impl == "reference":
         return run_reference(args)
     args.warmup = max(3, args.warmup)

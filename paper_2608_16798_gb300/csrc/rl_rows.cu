@@ -87,6 +87,20 @@ struct Vec<uint16_t> {  // bf16
     v[0] = bf16_lo(w.x); v[1] = bf16_hi(w.x); v[2] = bf16_lo(w.y); v[3] = bf16_hi(w.y);
     v[4] = bf16_lo(w.z); v[5] = bf16_hi(w.z); v[6] = bf16_lo(w.w); v[7] = bf16_hi(w.w);
   }
+  static constexpr int NP = 4;  // float2 pairs per 16-byte vector
+  static constexpr uint32_t kPadWord = 0xFF7FFF7Fu;  // two most-negative finite bf16 values
+  static __device__ __forceinline__ void pairs(const uint4 w, float2 (&q)[4]) {
+    q[0] = make_float2(bf16_lo(w.x), bf16_hi(w.x)); q[1] = make_float2(bf16_lo(w.y), bf16_hi(w.y));
+    q[2] = make_float2(bf16_lo(w.z), bf16_hi(w.z)); q[3] = make_float2(bf16_lo(w.w), bf16_hi(w.w));
+  }
+  static __device__ __forceinline__ uint4 pack_pairs(const float2 (&o)[4]) {
+    return make_uint4(pack_bf16x2(o[0].x, o[0].y), pack_bf16x2(o[1].x, o[1].y), pack_bf16x2(o[2].x, o[2].y),
+                      pack_bf16x2(o[3].x, o[3].y));
+  }
+  static __device__ __forceinline__ void unpack(const uint4 w, float (&v)[8]) {
+    v[0] = bf16_lo(w.x); v[1] = bf16_hi(w.x); v[2] = bf16_lo(w.y); v[3] = bf16_hi(w.y);
+    v[4] = bf16_lo(w.z); v[5] = bf16_hi(w.z); v[6] = bf16_lo(w.w); v[7] = bf16_hi(w.w);
+  }
   static __device__ __forceinline__ void store(uint16_t* dst, const float (&g)[8]) {
     uint4 w;
     w.x = pack_bf16x2(g[0], g[1]); w.y = pack_bf16x2(g[2], g[3]);
@@ -102,6 +116,19 @@ struct Vec<float> {
   static __device__ __forceinline__ void load(const float* buf, int64_t j, float (&v)[4]) {
     const float4 w = reinterpret_cast<const float4*>(buf)[j];
     v[0] = w.x; v[1] = w.y; v[2] = w.z; v[3] = w.w;
+  }
+  static constexpr int NP = 2;
+  static constexpr uint32_t kPadWord = 0xFF7FFFFFu;  // most-negative finite float
+  static __device__ __forceinline__ void pairs(const uint4 w, float2 (&q)[2]) {
+    q[0] = make_float2(__uint_as_float(w.x), __uint_as_float(w.y));
+    q[1] = make_float2(__uint_as_float(w.z), __uint_as_float(w.w));
+  }
+  static __device__ __forceinline__ uint4 pack_pairs(const float2 (&o)[2]) {
+    return make_uint4(__float_as_uint(o[0].x), __float_as_uint(o[0].y), __float_as_uint(o[1].x),
+                      __float_as_uint(o[1].y));
+  }
+  static __device__ __forceinline__ void unpack(const uint4 w, float (&v)[4]) {
+    v[0] = __uint_as_float(w.x); v[1] = __uint_as_float(w.y); v[2] = __uint_as_float(w.z); v[3] = __uint_as_float(w.w);
   }
   static __device__ __forceinline__ void store(float* dst, const float (&g)[4]) {
     st_global_16(dst, make_uint4(__float_as_uint(g[0]), __float_as_uint(g[1]), __float_as_uint(g[2]),
@@ -144,14 +171,14 @@ __device__ __forceinline__ void raise_max(SoftmaxPartial& ps, float vm) {
 #define RL_STAGES 2
 #endif
 #ifndef RL_CONSUMER_WARPS
-#define RL_CONSUMER_WARPS 8
+#define RL_CONSUMER_WARPS 7
 #endif
 #ifndef RL_SLICE_KB
-#define RL_SLICE_KB 48
+#define RL_SLICE_KB 40
 #endif
 
 constexpr int kMaxCluster = 16;
-constexpr int kZeroBytes = 8192;  // zero-filled shared region, source of the masked rows' bulk stores
+constexpr int kZeroBytes = 2048;  // zero-filled shared region, source of the masked rows' bulk stores
 
 // Per-row inputs, staged in shared memory by the producer warp.
 struct RowMeta {
@@ -173,7 +200,129 @@ struct RowMeta {
 //     every warp of every CTA), computes the row's scalars, runs pass 2 (gradient
 //     from the on-chip slice) and releases the stage.
 // Nothing per row synchronises a whole CTA or the whole cluster.
-template <typename T, int NW, bool ENT, bool BWD>
+// Fold EPV values into an online-softmax partial. The reference ps.m is the first
+// finite vector maximum and moves only when a vector's exponentials sum above 1e30
+// (some value lies far above the reference): the common case needs no per-element
+// max. exp(z - m) <= e^88 < FLT_MAX for every z within 88 of m, so before that
+// test overflows nothing.
+template <bool ENT, int EPV>
+__device__ __forceinline__ void fold(SoftmaxPartial& ps, const float (&v)[EPV]) {
+  if (ps.m == RL_NEG_INF) {
+    float vm = v[0];
+#pragma unroll
+    for (int k = 1; k < EPV; ++k) vm = fmaxf(vm, v[k]);
+    if (vm == RL_NEG_INF) return;
+    ps.m = vm;
+  }
+  float e[EPV], t[EPV];
+  auto exps = [&]() {
+    const float nm = -ps.m * kLog2e;
+#pragma unroll
+    for (int k = 0; k < EPV; ++k) {
+      if (ENT) {
+        t[k] = fmaxf(v[k], -1e30f) - ps.m;  // -inf logits contribute 0, not NaN
+        e[k] = ex2(t[k] * kLog2e);
+      } else {
+        e[k] = ex2(fmaf(v[k], kLog2e, nm));
+      }
+    }
+  };
+  auto tree = [&](const float (&x)[EPV]) {
+    float a[EPV];
+#pragma unroll
+    for (int k = 0; k < EPV; ++k) a[k] = x[k];
+#pragma unroll
+    for (int w = EPV / 2; w > 0; w /= 2)
+#pragma unroll
+      for (int k = 0; k < w; ++k) a[k] += a[k + w];
+    return a[0];
+  };
+  exps();
+  float se = tree(e);
+  if (!(se <= 1e30f)) {  // rare: move the reference up to this vector's maximum
+    float vm = v[0];
+#pragma unroll
+    for (int k = 1; k < EPV; ++k) vm = fmaxf(vm, v[k]);
+    raise_max<ENT>(ps, vm);
+    exps();
+    se = tree(e);
+  }
+  ps.s += se;
+  if (ENT) {
+    float et[EPV];
+#pragma unroll
+    for (int k = 0; k < EPV; ++k) et[k] = e[k] * t[k];
+    ps.u += tree(et);
+  }
+}
+
+// Fold NV register-held 16-byte vectors into a partial, branch-free in the common
+// case. Vectors past the end of the data hold T's most-negative finite value, whose
+// exponential is exactly 0. The reference is the partial's own maximum or, for a
+// fresh partial, the first vector's maximum; when the exponentials sum above 1e30
+// (a value far above the reference) everything is redone against the exact
+// maximum. Values at or below -1e38 count as -inf.
+template <typename T, bool ENT, int NV, typename Reload>
+__device__ __forceinline__ void fold_block(SoftmaxPartial& ps, const uint4 (&x)[NV], Reload reload) {
+  constexpr int NP = Vec<T>::NP;
+  auto vmax = [&](const uint4 w) {
+    float2 q[NP];
+    Vec<T>::pairs(w, q);
+    float m = fmaxf(q[0].x, q[0].y);
+#pragma unroll
+    for (int i = 1; i < NP; ++i) m = fmaxf(m, fmaxf(q[i].x, q[i].y));
+    return m;
+  };
+  // exact maximum, recomputed from shared memory (the rare paths only)
+  auto all_max = [&]() {
+    float m = vmax(reload(0));
+    for (int k = 1; k < NV; ++k) m = fmaxf(m, vmax(reload(k)));
+    return m;
+  };
+  if (!(ps.m > -1e38f)) {
+    float m0 = vmax(x[0]);
+    if (!(m0 > -1e38f)) m0 = all_max();
+    if (!(m0 > -1e38f)) return;
+    ps.m = m0;
+  }
+  auto exps = [&](const uint4 w, float2& s0, float2& s1, float2& u0) {
+    const float nm = -ps.m * kLog2e;
+    const float2 l2 = make_float2(kLog2e, kLog2e), nm2 = make_float2(nm, nm), mm = make_float2(-ps.m, -ps.m);
+    float2 q[NP];
+    Vec<T>::pairs(w, q);
+#pragma unroll
+    for (int i = 0; i < NP; ++i) {
+      if (ENT) {
+        const float2 t = __fadd2_rn(make_float2(fmaxf(q[i].x, -1e30f), fmaxf(q[i].y, -1e30f)), mm);
+        const float2 xx = __fmul2_rn(t, l2);
+        const float2 e = make_float2(ex2(xx.x), ex2(xx.y));
+        if (i & 1) s1 = __fadd2_rn(s1, e); else s0 = __fadd2_rn(s0, e);
+        u0 = __ffma2_rn(e, t, u0);
+      } else {
+        const float2 xx = __ffma2_rn(q[i], l2, nm2);
+        const float2 e = make_float2(ex2(xx.x), ex2(xx.y));
+        if (i & 1) s1 = __fadd2_rn(s1, e); else s0 = __fadd2_rn(s0, e);
+      }
+    }
+  };
+  const float2 z2 = make_float2(0.f, 0.f);
+  float2 s0 = z2, s1 = z2, u0 = z2;
+#pragma unroll
+  for (int k = 0; k < NV; ++k) exps(x[k], s0, s1, u0);
+  float2 sacc = __fadd2_rn(s0, s1);
+  float se = sacc.x + sacc.y;
+  if (!(se <= 1e30f)) {  // rare: move the reference up to the exact maximum and redo from shared memory
+    raise_max<ENT>(ps, all_max());
+    s0 = z2; s1 = z2; u0 = z2;
+    for (int k = 0; k < NV; ++k) exps(reload(k), s0, s1, u0);
+    sacc = __fadd2_rn(s0, s1);
+    se = sacc.x + sacc.y;
+  }
+  ps.s += se;
+  if (ENT) ps.u += u0.x + u0.y;
+}
+
+template <typename T, int NW, bool ENT, bool BWD, int HOLDV>
 __global__ void __launch_bounds__((NW + 1) * 32, 2) rows_kernel(const RowArgs p) {
   constexpr int EPV = Vec<T>::N;
   constexpr int NB = RL_STAGES;
@@ -190,9 +339,9 @@ __global__ void __launch_bounds__((NW + 1) * 32, 2) rows_kernel(const RowArgs p)
   const int64_t rows = p.rows, V = p.V, ld = p.ld;
   const int64_t s0 = static_cast<int64_t>(rank) * p.slice;
   const int64_t n_end = (s0 + p.slice < V) ? s0 + p.slice : V;
-  const int64_t n = n_end > s0 ? n_end - s0 : 0;  // elements of my slice
-  const int64_t nv = n / EPV;                      // full 16-byte vectors
-  const int64_t first_scalar = p.tma ? nv * EPV : 0;
+  const int n = n_end > s0 ? static_cast<int>(n_end - s0) : 0;  // elements of my slice
+  const int nv = n / EPV;                                        // full 16-byte vectors
+  const int first_scalar = p.tma ? nv * EPV : 0;
   const uint32_t tma_bytes = p.tma ? static_cast<uint32_t>(nv * 16) : 0u;
   const T* logits = static_cast<const T*>(p.logits);
   T* grad = static_cast<T*>(p.grad);
@@ -250,9 +399,9 @@ __global__ void __launch_bounds__((NW + 1) * 32, 2) rows_kernel(const RowArgs p)
               bulk_commit();
               stored = true;
             }
-            for (int64_t e = nv * EPV + lane; e < n; e += 32) g[e] = T(0);
+            for (int e = nv * EPV + lane; e < n; e += 32) g[e] = T(0);
           } else {
-            for (int64_t e = lane; e < n; e += 32) g[e] = T(0);
+            for (int e = lane; e < n; e += 32) g[e] = T(0);
           }
           if (rank == 0 && lane == 0) {
             p.row_loss[r] = 0.0;
@@ -274,7 +423,7 @@ __global__ void __launch_bounds__((NW + 1) * 32, 2) rows_kernel(const RowArgs p)
       }
       T* buf = buf_base + b * p.buf_elems;
       const T* src = logits + r * ld + s0;
-      for (int64_t e = first_scalar + lane; e < n; e += 32) buf[e] = src[e];
+      for (int e = first_scalar + lane; e < n; e += 32) buf[e] = src[e];
       __syncwarp();
       if (lane == 0) {
         meta[b] = m;
@@ -317,25 +466,36 @@ __global__ void __launch_bounds__((NW + 1) * 32, 2) rows_kernel(const RowArgs p)
       const bool a_ok = a >= 0 && a < V;
       const uint32_t owner = a_ok ? static_cast<uint32_t>(a / p.slice) : 0u;
 
-      // ---- pass 1: online softmax partial over the slice
+      // ---- pass 1: online softmax partial over the slice. With HOLDV > 0 the slice moves
+      // into registers here (vector j = tid + k * NC in hold[k]) and the stage is released
+      // right after, so the next copy lands while the exchange and pass 2 run.
       SoftmaxPartial ps{RL_NEG_INF, 0.f, 0.f};
-      for (int64_t j = tid; j < nv; j += NC) {
-        float v[EPV];
-        Vec<T>::load(buf, j, v);
-        float vm = v[0];
+      uint4 hold[HOLDV > 0 ? HOLDV : 1];
+      float tail_z = 0.f;
+      if (HOLDV > 0) {
+        const uint32_t pad = Vec<T>::kPadWord;
+        auto reload = [&](int k) {
+          const int j = tid + k * NC;
+          return j < nv ? reinterpret_cast<const uint4*>(buf)[j] : make_uint4(pad, pad, pad, pad);
+        };
 #pragma unroll
-        for (int k = 1; k < EPV; ++k) vm = fmaxf(vm, v[k]);
-        if (vm == RL_NEG_INF) continue;
-        raise_max<ENT>(ps, vm);
-        const float nm = -ps.m * kLog2e;
-#pragma unroll
-        for (int k = 0; k < EPV; ++k) accumulate<ENT>(ps, v[k], nm);
+        for (int k = 0; k < (HOLDV > 0 ? HOLDV : 1); ++k) hold[k] = reload(k);
+        fold_block<T, ENT>(ps, hold, reload);
+      } else {
+        for (int j = tid; j < nv; j += NC) {
+          float v[EPV];
+          Vec<T>::load(buf, j, v);
+          fold<ENT>(ps, v);
+        }
       }
-      for (int64_t e = nv * EPV + tid; e < n; e += NC) {
-        const float z = Vec<T>::to_f(buf[e]);
-        if (z == RL_NEG_INF) continue;
-        raise_max<ENT>(ps, z);
-        accumulate<ENT>(ps, z, -ps.m * kLog2e);
+      // ragged tail (fewer than EPV elements): one per thread at most
+      if (nv * EPV + tid < n) {
+        const float z = Vec<T>::to_f(buf[nv * EPV + tid]);
+        tail_z = z;
+        if (z != RL_NEG_INF) {
+          raise_max<ENT>(ps, z);
+          accumulate<ENT>(ps, z, -ps.m * kLog2e);
+        }
       }
       ps = warp_merge(ps);
       // lane 0's merge is the warp's partial: broadcast it so every copy sent is identical
@@ -344,6 +504,10 @@ __global__ void __launch_bounds__((NW + 1) * 32, 2) rows_kernel(const RowArgs p)
       ps.u = __shfl_sync(0xffffffffu, ps.u, 0);
       // warp 0 of the CTA holding the sampled token carries z_a; every other partial carries 0
       const float za_part = (warp == 0 && a_ok && rank == owner) ? Vec<T>::to_f(buf[a - s0]) : 0.f;
+      if (HOLDV > 0) {  // every read of the stage is done
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty_bar[b]);
+      }
 
       // ---- exchange: every warp's partial to every CTA of the cluster
       const int par = it & 1;
@@ -420,9 +584,8 @@ __global__ void __launch_bounds__((NW + 1) * 32, 2) rows_kernel(const RowArgs p)
         // ---- pass 2: gradient from the on-chip slice
         const float nl = -lse * kLog2e;
         T* g_row = grad + r * ld + s0;
-        for (int64_t j = tid; j < nv; j += NC) {
-          float v[EPV], o[EPV];
-          Vec<T>::load(buf, j, v);
+        auto grad_vec = [&](const float (&v)[EPV], int j) {
+          float o[EPV];
 #pragma unroll
           for (int k = 0; k < EPV; ++k) {
             const float pk = ex2(fmaf(v[k], kLog2e, nl));
@@ -434,16 +597,55 @@ __global__ void __launch_bounds__((NW + 1) * 32, 2) rows_kernel(const RowArgs p)
 #pragma unroll
             for (int k = 0; k < EPV; ++k) Vec<T>::store_scalar(g_row + j * EPV + k, o[k]);
           }
+        };
+        if (HOLDV > 0 && p.tma) {
+          constexpr int NP = Vec<T>::NP;
+          const float2 l2 = make_float2(kLog2e, kLog2e), nl2 = make_float2(nl, nl);
+          const float2 kp2 = make_float2(Kp, Kp), ca2 = make_float2(ca, ca), ke2 = make_float2(Ke, Ke);
+#pragma unroll
+          for (int k = 0; k < (HOLDV > 0 ? HOLDV : 1); ++k) {
+            const int j = tid + k * NC;
+            float2 q[NP], o[NP];
+            Vec<T>::pairs(hold[k], q);
+#pragma unroll
+            for (int i = 0; i < NP; ++i) {
+              const float2 xx = __ffma2_rn(q[i], l2, nl2);
+              const float2 pk = make_float2(ex2(xx.x), ex2(xx.y));
+              if (ENT) {
+                const float2 zc = make_float2(fmaxf(q[i].x, -1e30f), fmaxf(q[i].y, -1e30f));
+                o[i] = __fmul2_rn(pk, __ffma2_rn(ca2, zc, ke2));
+              } else {
+                o[i] = __fmul2_rn(kp2, pk);
+              }
+            }
+            if (j < nv) st_global_16(g_row + j * EPV, Vec<T>::pack_pairs(o));
+          }
+        } else if (HOLDV > 0) {
+#pragma unroll
+          for (int k = 0; k < (HOLDV > 0 ? HOLDV : 1); ++k) {
+            const int j = tid + k * NC;
+            if (j < nv) {
+              float v[EPV];
+              Vec<T>::unpack(hold[k], v);
+              grad_vec(v, j);
+            }
+          }
+        } else {
+          for (int j = tid; j < nv; j += NC) {
+            float v[EPV];
+            Vec<T>::load(buf, j, v);
+            grad_vec(v, j);
+          }
         }
-        for (int64_t e = nv * EPV + tid; e < n; e += NC) {
-          const float z = Vec<T>::to_f(buf[e]);
+        if (nv * EPV + tid < n) {
+          const float z = tail_z;
           const float pk = ex2(fmaf(z, kLog2e, nl));
-          Vec<T>::store_scalar(g_row + e, ENT ? pk * fmaf(ca, fmaxf(z, -1e30f), Ke) : Kp * pk);
+          Vec<T>::store_scalar(g_row + nv * EPV + tid, ENT ? pk * fmaf(ca, fmaxf(z, -1e30f), Ke) : Kp * pk);
         }
         // the sampled token's element gets + c g; rewritten by the thread that stored it
         if (rank == owner) {
-          const int64_t ia = a - s0;
-          const int64_t writer = ia < nv * EPV ? (ia / EPV) % NC : (ia - nv * EPV) % NC;
+          const int ia = static_cast<int>(a - s0);
+          const int writer = ia < nv * EPV ? (ia / EPV) % NC : (ia - nv * EPV);
           if (tid == writer) {
             const float pk = ex2(fmaf(za, kLog2e, nl));
             const float ga = (ENT ? pk * fmaf(ca, fmaxf(za, -1e30f), Ke) : Kp * pk) + cg;
@@ -451,14 +653,181 @@ __global__ void __launch_bounds__((NW + 1) * 32, 2) rows_kernel(const RowArgs p)
           }
         }
       }
-      // ---- release the stage
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&empty_bar[b]);
+      // ---- release the stage (already released after pass 1 when the slice is held in registers)
+      if (HOLDV == 0) {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty_bar[b]);
+      }
     }
   }
   __syncthreads();
   // no CTA leaves while a peer may still write into its mailbox
   if (C > 1) cluster_sync_all();
+}
+
+// ------------------------------------------------------------------ forward-only stream
+//
+// rl_token_logprobs reads each row exactly once and keeps nothing on chip, so it
+// needs no cluster: one CTA owns a row at a time (persistent over rows). A
+// producer warp streams the CTA's rows as back-to-back chunks through a ring of
+// shared-memory stages (bulk copies, full / empty mbarriers); consumer warps fold
+// each chunk into per-thread online-softmax partials and, at the end of a row,
+// merge them (one named barrier among the consumers per row).
+#ifndef RL_FWD_STAGES
+#define RL_FWD_STAGES 6
+#endif
+#ifndef RL_FWD_CHUNK_KB
+#define RL_FWD_CHUNK_KB 16
+#endif
+
+struct StreamArgs {
+  const void* logits;
+  int64_t rows, V, ld;
+  const int32_t* token_ids;
+  float* logp_out;
+  float* entropy_out;
+  float* lse_out;
+  int32_t* status;
+  int64_t chunk;      // elements per chunk (a multiple of the 16-byte vector)
+  int64_t buf_elems;  // element stride between stages
+  int32_t tma;        // rows 16-byte aligned
+};
+
+struct ChunkInfo {
+  int64_t r;      // row, -1 = end of stream
+  int32_t first;  // first element of the chunk within the row
+  int32_t count;  // elements in the chunk
+};
+
+template <typename T, int NW, bool ENT>
+__global__ void __launch_bounds__((NW + 1) * 32, 2) stream_logprobs_kernel(const StreamArgs p) {
+  constexpr int EPV = Vec<T>::N;
+  constexpr int NS = RL_FWD_STAGES;
+  constexpr int NC = NW * 32;
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  __shared__ __align__(8) uint64_t full_bar[NS], empty_bar[NS];
+  __shared__ ChunkInfo info[NS];
+  __shared__ SoftmaxPartial red[2][NW];
+
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t rows = p.rows, V = p.V, ld = p.ld, CH = p.chunk;
+  const int64_t nchunk = (V + CH - 1) / CH;
+  const T* logits = static_cast<const T*>(p.logits);
+  T* const buf_base = reinterpret_cast<T*>(smem_raw);
+
+  if (tid == 0) {
+#pragma unroll
+    for (int k = 0; k < NS; ++k) {
+      mbar_init(&full_bar[k], 1);
+      mbar_init(&empty_bar[k], NW);
+    }
+    fence_mbar_init();
+  }
+  __syncthreads();
+
+  if (warp == NW) {
+    // =============================================================== producer warp
+    uint32_t q = 0;
+    bool failed = false;
+    for (int64_t r = blockIdx.x; r < rows && !failed; r += gridDim.x) {
+      for (int64_t k = 0; k < nchunk; ++k, ++q) {
+        const int st = q % NS;
+        const uint32_t use = q / NS;
+        if (use > 0 && !mbar_wait_bounded(&empty_bar[st], (use - 1) & 1)) {
+          failed = true;
+          if (lane == 0) flag_status(p.status, RL_DEV_TIMEOUT);
+          break;
+        }
+        const int64_t first = k * CH;
+        const int64_t cnt = (first + CH < V ? first + CH : V) - first;
+        const int cv = p.tma ? static_cast<int>(cnt / EPV) : 0;
+        T* buf = buf_base + st * p.buf_elems;
+        const T* src = logits + r * ld + first;
+        for (int e = cv * EPV + lane; e < static_cast<int>(cnt); e += 32) buf[e] = src[e];
+        __syncwarp();
+        if (lane == 0) {
+          info[st] = ChunkInfo{r, static_cast<int32_t>(first), static_cast<int32_t>(cnt)};
+          if (cv > 0) {
+            mbar_arrive_expect_tx(&full_bar[st], static_cast<uint32_t>(cv * 16));
+            bulk_g2s(buf, src, static_cast<uint32_t>(cv * 16), &full_bar[st]);
+          } else {
+            mbar_arrive(&full_bar[st]);
+          }
+        }
+      }
+    }
+    if (!failed) {
+      const int st = q % NS;
+      const uint32_t use = q / NS;
+      if (use > 0 && !mbar_wait_bounded(&empty_bar[st], (use - 1) & 1)) {
+        if (lane == 0) flag_status(p.status, RL_DEV_TIMEOUT);
+      } else if (lane == 0) {
+        info[st].r = -1;
+        mbar_arrive(&full_bar[st]);
+      }
+    }
+  } else {
+    // =============================================================== consumer warps
+    SoftmaxPartial ps{RL_NEG_INF, 0.f, 0.f};
+    uint32_t row_it = 0;
+    for (uint32_t q = 0;; ++q) {
+      const int st = q % NS;
+      if (!mbar_wait_bounded(&full_bar[st], (q / NS) & 1)) {
+        if (tid == 0) flag_status(p.status, RL_DEV_TIMEOUT);
+        break;
+      }
+      const ChunkInfo ci = info[st];
+      if (ci.r < 0) break;
+      const T* buf = buf_base + st * p.buf_elems;
+      const int cv = ci.count / EPV;
+      {
+        constexpr int KV = (RL_FWD_CHUNK_KB * 1024 / 16 + NC - 1) / NC;  // vectors per thread per chunk
+        uint4 x[KV];
+        const uint32_t pad = Vec<T>::kPadWord;
+        auto reload = [&](int k) {
+          const int j = tid + k * NC;
+          return j < cv ? reinterpret_cast<const uint4*>(buf)[j] : make_uint4(pad, pad, pad, pad);
+        };
+#pragma unroll
+        for (int k = 0; k < KV; ++k) x[k] = reload(k);
+        fold_block<T, ENT>(ps, x, reload);
+      }
+      if (cv * EPV + tid < ci.count) {
+        const float z = Vec<T>::to_f(buf[cv * EPV + tid]);
+        if (z != RL_NEG_INF) {
+          raise_max<ENT>(ps, z);
+          accumulate<ENT>(ps, z, -ps.m * kLog2e);
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty_bar[st]);
+      if (ci.first + ci.count == V) {
+        // ---- end of row ci.r: merge the consumers' partials
+        const int par = row_it & 1;
+        ps = warp_merge(ps);
+        if (lane == 0) red[par][warp] = ps;
+        asm volatile("bar.sync 1, %0;" :: "n"(NC) : "memory");
+        if (warp == 0) {
+          SoftmaxPartial qq = lane < NW ? red[par][lane] : SoftmaxPartial{RL_NEG_INF, 0.f, 0.f};
+          qq = warp_merge(qq);
+          if (lane == 0) {
+            const int64_t r = ci.r;
+            const float lnS = logf(qq.s);
+            const float lse = qq.m + lnS;
+            const int32_t a = p.token_ids[r];
+            const bool a_ok = a >= 0 && a < V;
+            if (!a_ok) flag_status(p.status, RL_DEV_BAD_TOKEN);
+            const float za = a_ok ? Vec<T>::to_f(logits[r * ld + a]) : 0.f;
+            p.logp_out[r] = a_ok ? za - lse : __int_as_float(0x7fc00000);
+            if (p.entropy_out) p.entropy_out[r] = lnS - qq.u / qq.s;
+            if (p.lse_out) p.lse_out[r] = lse;
+          }
+        }
+        ps = SoftmaxPartial{RL_NEG_INF, 0.f, 0.f};
+        ++row_it;
+      }
+    }
+  }
 }
 
 // Fixed-order sum of the per-row contributions into the caller's accumulator.
@@ -492,7 +861,7 @@ struct Plan {
 
 static bool make_plan(int64_t V, int es, Plan* out) {
   const int64_t epv = 16 / es;
-  for (int C = 1; C <= 16; C *= 2) {
+  for (int C = 1; C <= 16; ++C) {
     const int64_t per = (V + C - 1) / C;
     const int64_t slice = (per + epv - 1) / epv * epv;
     if (slice * es <= kTargetSliceBytes || (C == 16 && slice * es <= kMaxSliceBytes)) {
@@ -507,29 +876,38 @@ static bool make_plan(int64_t V, int es, Plan* out) {
   return false;
 }
 
-template <typename T, bool ENT, bool BWD>
+// Configure a kernel once per (kernel, device): dynamic shared memory up to the
+// largest request so far, and non-portable cluster sizes allowed.
+static rl_status configure(const void* kern, int dev, size_t smem) {
+  static std::mutex mu;
+  static std::map<std::pair<const void*, int>, size_t> smem_attr;
+  std::lock_guard<std::mutex> lock(mu);
+  auto ka = std::make_pair(kern, dev);
+  auto ita = smem_attr.find(ka);
+  if (ita == smem_attr.end() || ita->second < smem) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(max dynamic smem)");
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(non-portable cluster)");
+    smem_attr[ka] = smem;
+  }
+  return RL_OK;
+}
+
+template <typename T, bool ENT, int HOLDV>
 static rl_status launch_rows(const RowArgs& args, const Plan& plan, cudaStream_t s) {
-  auto kern = rows_kernel<T, kConsumerWarps, ENT, BWD>;
+  auto kern = rows_kernel<T, kConsumerWarps, ENT, true, HOLDV>;
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return cuda_error(e, "cudaGetDevice");
+  rl_status st = configure(reinterpret_cast<const void*>(kern), dev, plan.smem);
+  if (st != RL_OK) return st;
 
   static std::mutex mu;
   static std::map<std::tuple<const void*, int, int, size_t>, int> cache;
-  static std::map<std::pair<const void*, int>, size_t> smem_attr;  // attribute value set per kernel and device
   int max_clusters = 0;
   {
     std::lock_guard<std::mutex> lock(mu);
-    // the function attribute bounds every later launch: keep it at the largest request so far
-    auto ka = std::make_pair(reinterpret_cast<const void*>(kern), dev);
-    auto ita = smem_attr.find(ka);
-    if (ita == smem_attr.end() || ita->second < plan.smem) {
-      e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(plan.smem));
-      if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(max dynamic smem)");
-      e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-      if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(non-portable cluster)");
-      smem_attr[ka] = plan.smem;
-    }
     auto key = std::make_tuple(reinterpret_cast<const void*>(kern), dev, plan.C, plan.smem);
     auto itc = cache.find(key);
     if (itc != cache.end()) {
@@ -570,11 +948,53 @@ static rl_status launch_rows(const RowArgs& args, const Plan& plan, cudaStream_t
   return RL_OK;
 }
 
-template <bool BWD>
-static rl_status dispatch_rows(rl_dtype dt, bool ent, const RowArgs& args, const Plan& plan, cudaStream_t s) {
-  if (dt == RL_BF16)
-    return ent ? launch_rows<uint16_t, true, BWD>(args, plan, s) : launch_rows<uint16_t, false, BWD>(args, plan, s);
-  return ent ? launch_rows<float, true, BWD>(args, plan, s) : launch_rows<float, false, BWD>(args, plan, s);
+// Registers hold the slice when it fits kHoldVecs 16-byte vectors per consumer thread.
+constexpr int kHoldVecs = 11;
+
+template <typename T>
+static rl_status dispatch_loss(bool ent, const RowArgs& args, const Plan& plan, cudaStream_t s) {
+  const bool hold = plan.slice * static_cast<int64_t>(sizeof(T)) / 16 <= int64_t(kHoldVecs) * kConsumerWarps * 32;
+  if (hold)
+    return ent ? launch_rows<T, true, kHoldVecs>(args, plan, s) : launch_rows<T, false, kHoldVecs>(args, plan, s);
+  return ent ? launch_rows<T, true, 0>(args, plan, s) : launch_rows<T, false, 0>(args, plan, s);
+}
+
+constexpr int kFwdWarps = 8;
+
+template <typename T, bool ENT>
+static rl_status launch_stream(const StreamArgs& args, cudaStream_t s) {
+  auto kern = stream_logprobs_kernel<T, kFwdWarps, ENT>;
+  const size_t smem = static_cast<size_t>(RL_FWD_STAGES) * args.buf_elems * sizeof(T);
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_error(e, "cudaGetDevice");
+  rl_status st = configure(reinterpret_cast<const void*>(kern), dev, smem);
+  if (st != RL_OK) return st;
+  static std::mutex mu;
+  static std::map<std::pair<const void*, int>, int> grid_cache;
+  int grid = 0;
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    auto key = std::make_pair(reinterpret_cast<const void*>(kern), dev);
+    auto it = grid_cache.find(key);
+    if (it != grid_cache.end()) {
+      grid = it->second;
+    } else {
+      int per_sm = 0, sms = 0;
+      e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, (kFwdWarps + 1) * 32, smem);
+      if (e != cudaSuccess) return cuda_error(e, "cudaOccupancyMaxActiveBlocksPerMultiprocessor");
+      e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+      if (e != cudaSuccess) return cuda_error(e, "cudaDeviceGetAttribute");
+      if (per_sm <= 0) return set_error(RL_ERR_UNSUPPORTED, "stream kernel does not fit on an SM");
+      grid = per_sm * sms;
+      grid_cache[key] = grid;
+    }
+  }
+  const unsigned blocks = static_cast<unsigned>(std::min<int64_t>(grid, args.rows));
+  kern<<<blocks, (kFwdWarps + 1) * 32, smem, s>>>(args);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_error(e, "stream_logprobs_kernel launch");
+  return RL_OK;
 }
 
 static rl_status check_rows_args(const char* fn, const void* logits, rl_dtype dt, int64_t rows, int64_t V,
@@ -608,7 +1028,7 @@ extern "C" rl_status rl_token_logprobs(const void* logits, rl_dtype dtype, int64
   if (st != RL_OK) return st;
   if (rows == 0) return RL_OK;
   if (!token_ids || !logp_out) return set_error(RL_ERR_INVALID_ARG, "rl_token_logprobs: NULL array argument");
-  RowArgs a = {};
+  StreamArgs a = {};
   a.logits = logits;
   a.rows = rows;
   a.V = V;
@@ -618,10 +1038,13 @@ extern "C" rl_status rl_token_logprobs(const void* logits, rl_dtype dtype, int64
   a.entropy_out = entropy_out;
   a.lse_out = lse_out;
   a.status = reinterpret_cast<int32_t*>(ws);
-  a.slice = plan.slice;
-  a.buf_elems = plan.buf_elems;
+  a.chunk = static_cast<int64_t>(RL_FWD_CHUNK_KB) * 1024 / es;
+  a.buf_elems = a.chunk;  // chunk bytes are a multiple of 128
   a.tma = ((ld * es) % 16) == 0;
-  return dispatch_rows<false>(dtype, entropy_out != nullptr, a, plan, reinterpret_cast<cudaStream_t>(stream));
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (dtype == RL_BF16)
+    return entropy_out ? launch_stream<uint16_t, true>(a, s) : launch_stream<uint16_t, false>(a, s);
+  return entropy_out ? launch_stream<float, true>(a, s) : launch_stream<float, false>(a, s);
 }
 
 extern "C" rl_status rl_policy_loss_fwd_bwd(const void* logits, rl_dtype dtype, int64_t rows, int64_t V,
@@ -678,7 +1101,7 @@ extern "C" rl_status rl_policy_loss_fwd_bwd(const void* logits, rl_dtype dtype, 
   a.tma = ((ld * es) % 16) == 0;
   const bool ent = params->entropy_coef != 0.f || token_stats != nullptr;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  st = dispatch_rows<true>(dtype, ent, a, plan, s);
+  st = dtype == RL_BF16 ? dispatch_loss<uint16_t>(ent, a, plan, s) : dispatch_loss<float>(ent, a, plan, s);
   if (st != RL_OK) return st;
   reduce_loss_kernel<<<1, 1024, 0, s>>>(row_loss, rows, loss_accum);
   cudaError_t e = cudaGetLastError();
