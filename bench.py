@@ -380,6 +380,22 @@ def host_sample_np(rows):
 
 # ----------------------------------------------------------------------------- main
 
+def max_over_ranks(value, dist, device):
+    """Maximum of a per-rank float over all ranks (the step time every rank reports)."""
+    if dist is None or not dist.is_initialized() or dist.get_world_size() == 1:
+        return float(value)
+    import torch
+
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(tokens_per_rank, world, ms_total, steps):
+    """Whole-job tokens per second: every rank processes tokens_per_rank per step (replicas)."""
+    return tokens_per_rank * world / (ms_total / 1e3 / steps)
+
+
 def dist_env():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     return int(os.environ.get("RANK", "0")), ws, int(os.environ.get("LOCAL_RANK", "0"))
@@ -520,12 +536,9 @@ def main():
     st, word = R.rl_query_status(batch.ws)
     if word != 0:
         raise RuntimeError(f"device status word {word} after the timed region")
-    if world > 1:
-        tt = torch.tensor([ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
+    ms = max_over_ranks(ms, dist if world > 1 else None, dev)
     ms_step = ms / args.steps
-    value = batch.T * world / (ms / 1e3 / args.steps)
+    value = job_throughput(batch.T, world, ms, args.steps)
 
     peak, peak_kind = measured_peaks()
     per_launch_bytes = sum(batch.mb_bytes) / n_mb
