@@ -96,7 +96,9 @@ const char* rl_last_error_message(void);
 
 /* Workspace bytes needed by calls on at most `max_rows` logits rows of
  * vocabulary V (D = hidden size of the fused head, 0 if unused). The
- * workspace holds the device status word and per-row loss contributions. */
+ * workspace holds the device status word and per-row loss contributions; with
+ * D > 0 it also holds the fused head's per-chunk buffers (about
+ * min(max_rows, 8192) * V * 2 bytes plus 32 MiB). */
 size_t rl_workspace_size(int64_t max_rows, int64_t V, int64_t D);
 
 /* Zero the workspace's status word. Call once after allocating a workspace,
@@ -205,6 +207,37 @@ rl_status rl_policy_loss_fwd_bwd(const void* logits, rl_dtype dtype, int64_t row
                                  const float* rollout_logp, const rl_loss_params* params,
                                  void* grad_out, double* loss_accum, float* token_stats, void* ws,
                                  size_t ws_bytes, rl_stream_t stream);
+
+/*
+ * Fused LM head: the same objective as rl_policy_loss_fwd_bwd with the logits
+ * Z = hidden W^T computed tile by tile on the tensor cores and never written to
+ * memory; returns the loss and the gradients with respect to hidden and W
+ * (pi_theta(a_t | s_t) of Sec. 2.3 as the softmax of the LM head's output;
+ * objective of Sec. 2.3.2 with the TIS weight of Sec. 3.2.4).
+ *
+ *   hidden        bf16 [T x D], row-major, 16-byte aligned
+ *   weight        bf16 [V x D], row-major (row v = output embedding of token v)
+ *   T, D, V       T >= 0, D >= 64 and a multiple of 64, V >= 1
+ *   token_ids, mask, token_traj, n_traj, adv, coef, old_logp, ref_logp,
+ *   rollout_logp, params, loss_accum, token_stats
+ *                 as for rl_policy_loss_fwd_bwd, with one row per token
+ *   d_hidden      [T x D] of d_hidden_dtype (RL_BF16 or RL_F32): d loss / d hidden
+ *                 (overwritten; zero rows for tokens that are not trained on)
+ *   d_weight      float [V x D]: d loss / d W is ADDED to it
+ *   ws, ws_bytes  workspace of at least rl_workspace_size(T, V, D) bytes; it holds,
+ *                 among others, the gradient of the logits for one chunk of 8,192
+ *                 tokens (bf16), consumed by the dH and dW products of that chunk
+ * Tokens are processed in chunks of 8,192: per chunk, a tensor-core pass forms the
+ * softmax statistics, a second pass recomputes the logits and forms their gradient,
+ * and two GEMMs (cuBLASLt) produce dH and accumulate dW.
+ */
+rl_status rl_fused_head_loss_fwd_bwd(const void* hidden, const void* weight, int64_t T, int64_t D, int64_t V,
+                                     const int32_t* token_ids, const uint8_t* mask, const int32_t* token_traj,
+                                     int32_t n_traj, const float* adv, const float* coef, const float* old_logp,
+                                     const float* ref_logp, const float* rollout_logp,
+                                     const rl_loss_params* params, void* d_hidden, rl_dtype d_hidden_dtype,
+                                     float* d_weight, double* loss_accum, float* token_stats, void* ws,
+                                     size_t ws_bytes, rl_stream_t stream);
 
 /*
  * Allocation-free form of rl_policy_loss_fwd_bwd (no counterpart in the paper:

@@ -30,9 +30,8 @@ int32_t rl_version(void) { return 10000; }
 const char* rl_last_error_message(void) { return rl::g_last_error.c_str(); }
 
 size_t rl_workspace_size(int64_t max_rows, int64_t V, int64_t D) {
-  (void)V;
-  (void)D;
   if (max_rows < 0) max_rows = 0;
+  if (D > 0 && V > 0) return rl::head_workspace_bytes(max_rows, V, D);
   const size_t rows_bytes = (static_cast<size_t>(max_rows) * sizeof(double) + 255) & ~size_t(255);
   return rl::kWsHeader + rows_bytes;
 }

@@ -1,0 +1,628 @@
+// Fused LM head: the policy loss and its gradients with respect to the hidden states
+// and the output projection, with the logits Z = H W^T never written to memory.
+//
+// For each chunk of tokens:
+//   1. head_kernel<STATS>  tcgen05 GEMM tiles Z[128 x 256] = H W^T (TMA-fed shared-memory
+//      stages, fp32 accumulators in TMEM, two accumulators so the epilogue of one tile
+//      overlaps the MMAs of the next); the epilogue folds every tile into per-row
+//      online-softmax partials for its vocabulary block.
+//   2. head_merge_kernel   one thread per token: merges the partials into lse, entropy and
+//      logp, evaluates the objective's per-token terms (same readings as the logits path),
+//      writes the row's loss contribution and the coefficients of dZ.
+//   3. head_kernel<DZ>     recomputes the same Z tiles; the epilogue forms
+//      dZ = c [g (delta_a - p) + alpha p (log p + H)] and stores it (bf16) for this chunk.
+//   4. dH = dZ W and dW += dZ^T H, two plain GEMMs through cuBLASLt.
+// The objective (Sec. 2.3.2, Sec. 3.2.4) is the same as for rl_policy_loss_fwd_bwd; here
+// pi_theta's logits come from the hidden states times the vocabulary projection.
+#include <cublasLt.h>
+#include <cuda.h>
+
+#include <algorithm>
+#include <map>
+#include <mutex>
+#include <string>
+
+#include "rl_device.cuh"
+#include "rl_host.h"
+#include "rl_tc.cuh"
+
+namespace rl {
+namespace head {
+
+constexpr int BM = 128;            // tokens per tile (TMEM lanes)
+constexpr int BN = 256;            // vocabulary entries per tile (TMEM columns per accumulator)
+constexpr int BK = 64;             // hidden elements per stage (one 128-byte swizzle row)
+constexpr int NS = 4;              // shared-memory stages
+constexpr int VB_TILES = 16;       // N tiles per work item (a vocabulary block of 4,096)
+constexpr uint32_t A_BYTES = BM * BK * 2, B_BYTES = BN * BK * 2, STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int kThreads = 192;      // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
+constexpr size_t kSmem = NS * STAGE_BYTES + 1024;
+constexpr int64_t kChunk = 8192;   // tokens per chunk
+constexpr size_t kLtWorkspace = 32u << 20;
+
+enum Mode { STATS = 0, DZ = 1 };
+
+// Per-token coefficients of dZ (from head_merge_kernel).
+struct RowCoef {
+  float nlse2;  // -lse * log2(e)
+  float Kp;     // dZ_v = Kp p_v (+ cg at v = a), without the entropy term
+  float cg;
+  float ca;     // entropy: dZ_v = p_v (ca z_v + Ke) (+ cg at v = a)
+  float Ke;
+  int32_t a;
+  int32_t active;
+  float pad;
+};
+
+struct HeadArgs {
+  int64_t t0;  // first token of the chunk
+  int32_t Tc, D, V, n_mt, n_vb, n_nt;
+  int32_t ent;
+  const int32_t* token_ids;
+  float4* partials;        // [n_vb][Tc] (m, s, u, z_a)
+  const RowCoef* rc;       // [Tc]
+  uint16_t* dz;            // [Tc x ldz] bf16
+  int64_t ldz;
+  int32_t* status;
+};
+
+template <int MODE>
+__global__ void __launch_bounds__(kThreads, 1) head_kernel(const __grid_constant__ CUtensorMap tmH,
+                                                           const __grid_constant__ CUtensorMap tmW,
+                                                           const HeadArgs p) {
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t full[NS], empty[NS], accf[2], acce[2];
+  __shared__ uint32_t tbase;
+  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n_items = p.n_mt * p.n_vb;
+  const int nkb = p.D / BK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < NS; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&accf[a], 1);
+      mbar_init(&acce[a], 4);
+    }
+    fence_mbar_init();
+  }
+  if (warp == 1) tc::tmem_alloc(&tbase, 2 * BN);
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = tbase;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- TMA producer
+    if (lane == 0) {
+      uint32_t g = 0;
+      bool ok = true;
+      for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+        const int vb = item / p.n_mt, m0 = (item % p.n_mt) * BM;
+        const int nt1 = min((vb + 1) * VB_TILES, p.n_nt);
+        for (int nt = vb * VB_TILES; nt < nt1 && ok; ++nt) {
+          for (int kb = 0; kb < nkb; ++kb, ++g) {
+            const int s = g % NS;
+            const uint32_t use = g / NS;
+            if (use > 0 && !mbar_wait_bounded(&empty[s], (use - 1) & 1)) {
+              flag_status(p.status, RL_DEV_TIMEOUT);
+              ok = false;
+              break;
+            }
+            uint8_t* st = sm + s * STAGE_BYTES;
+            mbar_arrive_expect_tx(&full[s], STAGE_BYTES);
+            tc::tma_load_2d(st, &tmH, kb * BK, m0, &full[s]);
+            tc::tma_load_2d(st + A_BYTES, &tmW, kb * BK, nt * BN, &full[s]);
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc = tc::idesc_bf16_f32(BM, BN);
+      uint32_t g = 0, t = 0;
+      bool ok = true;
+      for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+        const int vb = item / p.n_mt;
+        const int nt1 = min((vb + 1) * VB_TILES, p.n_nt);
+        for (int nt = vb * VB_TILES; nt < nt1 && ok; ++nt, ++t) {
+          const int acc = t & 1;
+          if (t >= 2 && !mbar_wait_bounded(&acce[acc], ((t >> 1) - 1) & 1)) {
+            flag_status(p.status, RL_DEV_TIMEOUT);
+            ok = false;
+            break;
+          }
+          tc::fence_after_sync();
+          const uint32_t d = tmem + acc * BN;
+          for (int kb = 0; kb < nkb; ++kb, ++g) {
+            const int s = g % NS;
+            if (!mbar_wait_bounded(&full[s], (g / NS) & 1)) {
+              flag_status(p.status, RL_DEV_TIMEOUT);
+              ok = false;
+              break;
+            }
+            tc::fence_after_sync();
+            const uint32_t a = smem_addr(sm + s * STAGE_BYTES), b = a + A_BYTES;
+#pragma unroll
+            for (int k = 0; k < BK / 16; ++k)
+              tc::mma_bf16(d, tc::desc_kmajor_sw128(a + k * 32), tc::desc_kmajor_sw128(b + k * 32), idesc,
+                           (kb | k) != 0);
+            tc::mma_commit(&empty[s]);
+          }
+          if (ok) tc::mma_commit(&accf[acc]);
+        }
+      }
+    }
+  } else {
+    // ---------------------------------------------------------------- epilogue (4 warps)
+    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    const int rl = 32 * q + lane;
+    uint32_t t = 0;
+    bool ok = true;
+    for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+      const int vb = item / p.n_mt, m0 = (item % p.n_mt) * BM;
+      const int r = m0 + rl;  // token within the chunk
+      const bool row_ok = r < p.Tc;
+      const int nt1 = min((vb + 1) * VB_TILES, p.n_nt);
+      SoftmaxPartial ps{-__int_as_float(0x7f800000), 0.f, 0.f};
+      float za = 0.f;
+      int32_t a = -1;
+      RowCoef rc = {};
+      if (MODE == STATS) {
+        if (row_ok) a = p.token_ids[p.t0 + r];
+      } else {
+        if (row_ok) rc = p.rc[r];
+        a = rc.a;
+      }
+      for (int nt = vb * VB_TILES; nt < nt1; ++nt, ++t) {
+        const int acc = t & 1;
+        if (!mbar_wait_bounded(&accf[acc], (t >> 1) & 1)) {
+          if (lane == 0) flag_status(p.status, RL_DEV_TIMEOUT);
+          ok = false;
+          break;
+        }
+        tc::fence_after_sync();
+        const int n0 = nt * BN;
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+          float v[32];
+          tc::tmem_ld32(tmem + (static_cast<uint32_t>(32 * q) << 16) + acc * BN + c, v);
+          const int col0 = n0 + c;
+          const int nvalid = min(32, p.V - col0);
+          if (nvalid <= 0) continue;  // past the vocabulary (uniform across the warp)
+          if (MODE == STATS) {
+            float vm = -__int_as_float(0x7f800000);
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+              if (j >= nvalid) v[j] = -1e30f;  // contributes exp(...) = 0
+              vm = fmaxf(vm, v[j]);
+            }
+            if (vm > ps.m) {
+              const float dd = ps.m - vm;
+              const float sc = ex2(dd * kLog2e);
+              ps.u = (ps.s == 0.f) ? 0.f : sc * fmaf(dd, ps.s, ps.u);
+              ps.s *= sc;
+              ps.m = vm;
+            }
+            const float nm = -ps.m * kLog2e;
+            float s0 = 0.f, s1 = 0.f, u0 = 0.f;
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+              const float e = ex2(fmaf(v[j], kLog2e, nm));
+              if (j & 1) s1 += e; else s0 += e;
+              if (p.ent) u0 = fmaf(e, v[j] - ps.m, u0);
+            }
+            ps.s += s0 + s1;
+            ps.u += u0;
+            const int ja = a - col0;
+            if (ja >= 0 && ja < 32) {
+#pragma unroll
+              for (int j = 0; j < 32; ++j)
+                if (j == ja) za = v[j];
+            }
+          } else if (row_ok) {
+            uint16_t* out = p.dz + static_cast<int64_t>(r) * p.ldz + col0;
+            uint32_t w[16];
+            if (rc.active) {
+#pragma unroll
+              for (int j = 0; j < 32; j += 2) {
+                float o[2];
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                  const float z = v[j + h];
+                  const float pk = ex2(fmaf(z, kLog2e, rc.nlse2));
+                  float x = p.ent ? pk * fmaf(rc.ca, z, rc.Ke) : rc.Kp * pk;
+                  if (col0 + j + h == a) x += rc.cg;
+                  o[h] = x;
+                }
+                w[j / 2] = pack_bf16x2(o[0], o[1]);
+              }
+            } else {
+#pragma unroll
+              for (int j = 0; j < 16; ++j) w[j] = 0u;
+            }
+            if (nvalid == 32) {
+#pragma unroll
+              for (int j = 0; j < 4; ++j)
+                *reinterpret_cast<uint4*>(out + 8 * j) = make_uint4(w[4 * j], w[4 * j + 1], w[4 * j + 2], w[4 * j + 3]);
+            } else {
+#pragma unroll
+              for (int j = 0; j < 32; ++j)
+                if (j < nvalid) out[j] = static_cast<uint16_t>((w[j / 2] >> (16 * (j & 1))) & 0xFFFFu);
+            }
+          }
+        }
+        tc::fence_before_sync();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&acce[acc]);
+      }
+      if (MODE == STATS && ok && row_ok)
+        p.partials[static_cast<int64_t>(vb) * p.Tc + r] = make_float4(ps.m, ps.s, ps.u, za);
+    }
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == 1) {
+    tc::fence_after_sync();
+    tc::tmem_dealloc(tmem, 2 * BN);
+  }
+}
+
+struct MergeArgs {
+  int64_t t0;
+  int32_t Tc, V, n_vb, n_traj;
+  const float4* partials;
+  const int32_t* token_ids;
+  const uint8_t* mask;
+  const int32_t* token_traj;
+  const float* adv;
+  const float* coef;
+  const float* old_logp;
+  const float* ref_logp;
+  const float* rollout_logp;
+  float clip_lo, clip_hi, beta, alpha, tis_cap;
+  RowCoef* rc;
+  double* row_loss;
+  float* token_stats;
+  int32_t* status;
+};
+
+// One thread per token of the chunk: merge the vocabulary blocks' partials (fixed order)
+// and evaluate the per-token objective terms.
+__global__ void __launch_bounds__(256) head_merge_kernel(const MergeArgs p) {
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= p.Tc) return;
+  const int64_t t = p.t0 + r;
+  RowCoef rc = {};
+  rc.a = -1;
+  bool active = p.mask[t] != 0;
+  int32_t i = 0;
+  if (active) {
+    i = p.token_traj[t];
+    if (i < 0 || i >= p.n_traj) {
+      flag_status(p.status, RL_DEV_BAD_TRAJ);
+      active = false;
+    } else if (p.coef[i] == 0.f) {
+      active = false;
+    }
+  }
+  const int32_t a = p.token_ids[t];
+  if (active && (a < 0 || a >= p.V)) {
+    flag_status(p.status, RL_DEV_BAD_TOKEN);
+    active = false;
+  }
+  if (!active) {
+    p.rc[r] = rc;
+    p.row_loss[t] = 0.0;
+    if (p.token_stats)
+      for (int k = 0; k < 5; ++k) p.token_stats[t * 5 + k] = 0.f;
+    return;
+  }
+  SoftmaxPartial q{-__int_as_float(0x7f800000), 0.f, 0.f};
+  float za = 0.f;
+  for (int b = 0; b < p.n_vb; ++b) {
+    const float4 w = p.partials[static_cast<int64_t>(b) * p.Tc + r];
+    q = merge(q, SoftmaxPartial{w.x, w.y, w.z});
+    za += w.w;
+  }
+  const float lnS = logf(q.s);
+  const float lse = q.m + lnS;
+  const float H = lnS - q.u / q.s;
+  const float A = p.adv[i], c = p.coef[i], old = p.old_logp[t];
+  const float logp = za - lse;
+  const float rho = expf((za - old) - lse);
+  const float crho = fminf(fmaxf(rho, p.clip_lo), p.clip_hi);
+  const float surr = fminf(rho * A, crho * A);
+  const bool cut = (A > 0.f && rho > p.clip_hi) || (A < 0.f && rho < p.clip_lo);
+  const float w = (p.tis_cap > 0.f && p.rollout_logp) ? fminf(expf(old - p.rollout_logp[t]), p.tis_cap) : 1.f;
+  float kl = 0.f, dkl = 0.f;
+  if (p.beta != 0.f && p.ref_logp) {
+    const float d = (p.ref_logp[t] - za) + lse;
+    const float ed = expf(d);
+    kl = ed - d - 1.f;
+    dkl = 1.f - ed;
+  }
+  const float ell = -w * surr + p.beta * kl - p.alpha * H;
+  const float g = (cut ? 0.f : -w * A * rho) + p.beta * dkl;
+  const float cg = c * g, ca = c * p.alpha;
+  rc.nlse2 = -lse * kLog2e;
+  rc.Kp = -cg;
+  rc.cg = cg;
+  rc.ca = ca;
+  rc.Ke = -cg + ca * (H - lse);
+  rc.a = a;
+  rc.active = 1;
+  p.rc[r] = rc;
+  p.row_loss[t] = static_cast<double>(c) * static_cast<double>(ell);
+  if (p.token_stats) {
+    float* st = p.token_stats + t * 5;
+    st[0] = logp; st[1] = rho; st[2] = cut ? 1.f : 0.f; st[3] = H; st[4] = kl;
+  }
+}
+
+// ------------------------------------------------------------------ host side
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static rl_status encoder(EncodeTiledFn* out) {
+  static std::mutex mu;
+  static EncodeTiledFn fn = nullptr;
+  std::lock_guard<std::mutex> lock(mu);
+  if (!fn) {
+    cudaDriverEntryPointQueryResult q;
+    void* f = nullptr;
+    cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q);
+    if (e != cudaSuccess || !f || q != cudaDriverEntryPointSuccess)
+      return set_error(RL_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
+    fn = reinterpret_cast<EncodeTiledFn>(f);
+  }
+  *out = fn;
+  return RL_OK;
+}
+
+// bf16 matrix [rows x inner] (row stride inner), tiles of box_rows x 64 with the 128-byte swizzle.
+static rl_status make_map(CUtensorMap* m, const void* base, int64_t inner, int64_t rows, uint32_t box_rows) {
+  EncodeTiledFn enc;
+  rl_status st = encoder(&enc);
+  if (st != RL_OK) return st;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(inner) * 2};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t es[2] = {1, 1};
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return set_error(RL_ERR_CUDA, "cuTensorMapEncodeTiled failed");
+  return RL_OK;
+}
+
+struct Layout {
+  int64_t Tc, n_vb, ldz;
+  size_t off_partials, off_rc, off_dz, off_lt, total;
+};
+
+static Layout layout(int64_t max_rows, int64_t V) {
+  Layout L;
+  L.Tc = std::max<int64_t>(1, std::min<int64_t>(max_rows, kChunk));
+  const int64_t n_nt = (V + BN - 1) / BN;
+  L.n_vb = (n_nt + VB_TILES - 1) / VB_TILES;
+  L.ldz = (V + 7) / 8 * 8;
+  auto al = [](size_t x) { return (x + 255) & ~size_t(255); };
+  size_t off = kWsHeader + al(static_cast<size_t>(std::max<int64_t>(max_rows, 0)) * sizeof(double));
+  L.off_partials = off;
+  off += al(static_cast<size_t>(L.n_vb * L.Tc) * sizeof(float4));
+  L.off_rc = off;
+  off += al(static_cast<size_t>(L.Tc) * sizeof(RowCoef));
+  L.off_dz = off;
+  off += al(static_cast<size_t>(L.Tc * L.ldz) * 2);
+  L.off_lt = off;
+  off += kLtWorkspace;
+  L.total = off;
+  return L;
+}
+
+// C (col-major m x n) = op(A) op(B) + beta C with bf16 A, B and fp32 accumulation.
+static rl_status lt_matmul(cublasLtHandle_t lt, bool ta, bool tb, int64_t m, int64_t n, int64_t k, const void* A,
+                           int64_t lda, const void* B, int64_t ldb, void* C, int64_t ldc, cudaDataType_t ctype,
+                           float beta, void* ws, size_t ws_bytes, cudaStream_t s) {
+  cublasLtMatmulDesc_t op = nullptr;
+  cublasLtMatrixLayout_t la = nullptr, lb = nullptr, lc = nullptr;
+  cublasLtMatmulPreference_t pref = nullptr;
+  rl_status st = RL_OK;
+  const float alpha = 1.f;
+  cublasOperation_t opa = ta ? CUBLAS_OP_T : CUBLAS_OP_N, opb = tb ? CUBLAS_OP_T : CUBLAS_OP_N;
+  cublasLtMatmulHeuristicResult_t heur = {};
+  int found = 0;
+  auto fail = [&](const char* what) { st = set_error(RL_ERR_CUDA, std::string("cuBLASLt: ") + what); };
+  if (cublasLtMatmulDescCreate(&op, CUBLAS_COMPUTE_32F, CUDA_R_32F) != CUBLAS_STATUS_SUCCESS) { fail("desc"); goto done; }
+  cublasLtMatmulDescSetAttribute(op, CUBLASLT_MATMUL_DESC_TRANSA, &opa, sizeof(opa));
+  cublasLtMatmulDescSetAttribute(op, CUBLASLT_MATMUL_DESC_TRANSB, &opb, sizeof(opb));
+  if (cublasLtMatrixLayoutCreate(&la, CUDA_R_16BF, ta ? k : m, ta ? m : k, lda) != CUBLAS_STATUS_SUCCESS ||
+      cublasLtMatrixLayoutCreate(&lb, CUDA_R_16BF, tb ? n : k, tb ? k : n, ldb) != CUBLAS_STATUS_SUCCESS ||
+      cublasLtMatrixLayoutCreate(&lc, ctype, m, n, ldc) != CUBLAS_STATUS_SUCCESS) {
+    fail("layout");
+    goto done;
+  }
+  if (cublasLtMatmulPreferenceCreate(&pref) != CUBLAS_STATUS_SUCCESS) { fail("preference"); goto done; }
+  cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MAX_WORKSPACE_BYTES, &ws_bytes, sizeof(ws_bytes));
+  if (cublasLtMatmulAlgoGetHeuristic(lt, op, la, lb, lc, lc, pref, 1, &heur, &found) != CUBLAS_STATUS_SUCCESS ||
+      found == 0) {
+    fail("no algorithm");
+    goto done;
+  }
+  if (cublasLtMatmul(lt, op, &alpha, A, la, B, lb, &beta, C, lc, C, lc, &heur.algo, ws, ws_bytes, s) !=
+      CUBLAS_STATUS_SUCCESS)
+    fail("matmul");
+done:
+  if (pref) cublasLtMatmulPreferenceDestroy(pref);
+  if (lc) cublasLtMatrixLayoutDestroy(lc);
+  if (lb) cublasLtMatrixLayoutDestroy(lb);
+  if (la) cublasLtMatrixLayoutDestroy(la);
+  if (op) cublasLtMatmulDescDestroy(op);
+  return st;
+}
+
+static rl_status lt_handle(cublasLtHandle_t* out) {
+  static std::mutex mu;
+  static cublasLtHandle_t h = nullptr;
+  std::lock_guard<std::mutex> lock(mu);
+  if (!h && cublasLtCreate(&h) != CUBLAS_STATUS_SUCCESS) return set_error(RL_ERR_CUDA, "cublasLtCreate failed");
+  *out = h;
+  return RL_OK;
+}
+
+template <int MODE>
+static rl_status launch_head(const CUtensorMap& mh, const CUtensorMap& mw, const HeadArgs& a, cudaStream_t s) {
+  auto kern = head_kernel<MODE>;
+  int dev = 0, sms = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return cuda_error(e, "cudaDeviceGetAttribute");
+  static std::mutex mu;
+  static std::map<std::pair<int, int>, bool> configured;
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    auto key = std::make_pair(dev, MODE);
+    if (!configured[key]) {
+      e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kSmem));
+      if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(head_kernel)");
+      configured[key] = true;
+    }
+  }
+  const int items = a.n_mt * a.n_vb;
+  kern<<<std::min(items, sms), kThreads, kSmem, s>>>(mh, mw, a);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_error(e, "head_kernel launch");
+  return RL_OK;
+}
+
+}  // namespace head
+
+size_t head_workspace_bytes(int64_t max_rows, int64_t V, int64_t D) {
+  (void)D;
+  return head::layout(max_rows, V).total;
+}
+
+}  // namespace rl
+
+extern "C" rl_status rl_fused_head_loss_fwd_bwd(
+    const void* hidden, const void* weight, int64_t T, int64_t D, int64_t V, const int32_t* token_ids,
+    const uint8_t* mask, const int32_t* token_traj, int32_t n_traj, const float* adv, const float* coef,
+    const float* old_logp, const float* ref_logp, const float* rollout_logp, const rl_loss_params* params,
+    void* d_hidden, rl_dtype d_hidden_dtype, float* d_weight, double* loss_accum, float* token_stats, void* ws,
+    size_t ws_bytes, rl_stream_t stream) {
+  using namespace rl;
+  using namespace rl::head;
+  clear_error();
+  if (T < 0 || D < 64 || V < 1 || n_traj < 0)
+    return set_error(RL_ERR_INVALID_ARG, "rl_fused_head_loss_fwd_bwd: need T >= 0, D >= 64, V >= 1, n_traj >= 0");
+  if (D % 64 != 0) return set_error(RL_ERR_UNSUPPORTED, "rl_fused_head_loss_fwd_bwd: D must be a multiple of 64");
+  if (T > INT32_MAX || V > INT32_MAX || D > 65536)
+    return set_error(RL_ERR_UNSUPPORTED, "rl_fused_head_loss_fwd_bwd: T or V above 2^31 - 1, or D above 65536");
+  if (!params || !loss_accum || !ws) return set_error(RL_ERR_INVALID_ARG, "rl_fused_head_loss_fwd_bwd: NULL argument");
+  if (d_hidden_dtype != RL_BF16 && d_hidden_dtype != RL_F32)
+    return set_error(RL_ERR_INVALID_ARG, "rl_fused_head_loss_fwd_bwd: unknown d_hidden dtype");
+  if (params->kl_estimator != 0 && params->kl_estimator != 3)
+    return set_error(RL_ERR_UNSUPPORTED, "rl_fused_head_loss_fwd_bwd: kl_estimator must be 0 or 3");
+  if (ws_bytes < rl_workspace_size(T, V, D))
+    return set_error(RL_ERR_WORKSPACE_TOO_SMALL,
+                     "rl_fused_head_loss_fwd_bwd: workspace smaller than rl_workspace_size(T, V, D)");
+  if (T == 0) return RL_OK;
+  if (!hidden || !weight || !token_ids || !mask || !token_traj || !old_logp || !d_hidden || !d_weight ||
+      (n_traj > 0 && (!adv || !coef)))
+    return set_error(RL_ERR_INVALID_ARG, "rl_fused_head_loss_fwd_bwd: NULL array argument");
+  if (!aligned16(hidden) || !aligned16(weight) || !aligned16(d_hidden) || !aligned16(d_weight) || !aligned16(ws))
+    return set_error(RL_ERR_ALIGNMENT,
+                     "rl_fused_head_loss_fwd_bwd: hidden, weight, d_hidden, d_weight and ws must be 16-byte aligned");
+
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const Layout L = layout(T, V);
+  char* wsb = static_cast<char*>(ws);
+  int32_t* status = reinterpret_cast<int32_t*>(wsb);
+  double* row_loss = reinterpret_cast<double*>(wsb + ws_row_loss_offset());
+  float4* partials = reinterpret_cast<float4*>(wsb + L.off_partials);
+  RowCoef* rcs = reinterpret_cast<RowCoef*>(wsb + L.off_rc);
+  uint16_t* dz = reinterpret_cast<uint16_t*>(wsb + L.off_dz);
+  void* lt_ws = wsb + L.off_lt;
+  cublasLtHandle_t lt;
+  rl_status st = lt_handle(&lt);
+  if (st != RL_OK) return st;
+  const bool kl_on = params->kl_estimator == 3 && params->kl_coef != 0.f && ref_logp != nullptr;
+  const bool ent = params->entropy_coef != 0.f || token_stats != nullptr;
+
+  CUtensorMap mw;
+  st = make_map(&mw, weight, D, V, BN);
+  if (st != RL_OK) return st;
+  const int n_nt = static_cast<int>((V + BN - 1) / BN);
+  for (int64_t t0 = 0; t0 < T; t0 += L.Tc) {
+    const int Tc = static_cast<int>(std::min<int64_t>(L.Tc, T - t0));
+    const uint16_t* h0 = static_cast<const uint16_t*>(hidden) + t0 * D;
+    CUtensorMap mh;
+    st = make_map(&mh, h0, D, Tc, BM);
+    if (st != RL_OK) return st;
+    HeadArgs ha = {};
+    ha.t0 = t0;
+    ha.Tc = Tc;
+    ha.D = static_cast<int>(D);
+    ha.V = static_cast<int>(V);
+    ha.n_mt = (Tc + BM - 1) / BM;
+    ha.n_nt = n_nt;
+    ha.n_vb = static_cast<int>(L.n_vb);
+    ha.ent = ent ? 1 : 0;
+    ha.token_ids = token_ids;
+    ha.partials = partials;
+    ha.rc = rcs;
+    ha.dz = dz;
+    ha.ldz = L.ldz;
+    ha.status = status;
+    st = launch_head<STATS>(mh, mw, ha, s);
+    if (st != RL_OK) return st;
+
+    MergeArgs ma = {};
+    ma.t0 = t0;
+    ma.Tc = Tc;
+    ma.V = static_cast<int>(V);
+    ma.n_vb = ha.n_vb;
+    ma.n_traj = n_traj;
+    ma.partials = partials;
+    ma.token_ids = token_ids;
+    ma.mask = mask;
+    ma.token_traj = token_traj;
+    ma.adv = adv;
+    ma.coef = coef;
+    ma.old_logp = old_logp;
+    ma.ref_logp = kl_on ? ref_logp : nullptr;
+    ma.rollout_logp = rollout_logp;
+    ma.clip_lo = 1.f - params->clip_eps_low;
+    ma.clip_hi = 1.f + params->clip_eps_high;
+    ma.beta = kl_on ? params->kl_coef : 0.f;
+    ma.alpha = params->entropy_coef;
+    ma.tis_cap = rollout_logp ? params->tis_cap : 0.f;
+    ma.rc = rcs;
+    ma.row_loss = row_loss;
+    ma.token_stats = token_stats;
+    ma.status = status;
+    head_merge_kernel<<<(Tc + 255) / 256, 256, 0, s>>>(ma);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_error(e, "head_merge_kernel launch");
+
+    st = launch_head<DZ>(mh, mw, ha, s);
+    if (st != RL_OK) return st;
+
+    // dH[t0 : t0 + Tc] = dZ W    (column-major: dH^T [D x Tc] = W^T [D x V] dZ^T [V x Tc])
+    void* dh = static_cast<char*>(d_hidden) + t0 * D * (d_hidden_dtype == RL_BF16 ? 2 : 4);
+    st = lt_matmul(lt, false, false, D, Tc, V, weight, D, dz, L.ldz, dh, D,
+                   d_hidden_dtype == RL_BF16 ? CUDA_R_16BF : CUDA_R_32F, 0.f, lt_ws, kLtWorkspace, s);
+    if (st != RL_OK) return st;
+    // dW += dZ^T H  (column-major: dW^T [D x V] += H^T [D x Tc] (dZ^T)^T [Tc x V])
+    st = lt_matmul(lt, false, true, D, V, Tc, h0, D, dz, L.ldz, d_weight, D, CUDA_R_32F, 1.f, lt_ws, kLtWorkspace, s);
+    if (st != RL_OK) return st;
+  }
+  return launch_reduce_loss(row_loss, T, loss_accum, s);
+}

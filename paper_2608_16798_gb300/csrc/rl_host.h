@@ -22,6 +22,11 @@ rl_status set_error(rl_status st, const std::string& msg);
 rl_status cuda_error(cudaError_t e, const char* what);
 void clear_error();
 
+// Fixed-order sum of per-row loss contributions into *loss_accum (rl_rows.cu).
+rl_status launch_reduce_loss(const double* row_loss, int64_t rows, double* loss_accum, cudaStream_t s);
+// Workspace of the fused LM head for up to max_rows tokens (rl_head.cu).
+size_t head_workspace_bytes(int64_t max_rows, int64_t V, int64_t D);
+
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 }  // namespace rl

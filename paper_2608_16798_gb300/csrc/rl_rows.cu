@@ -848,6 +848,13 @@ __global__ void __launch_bounds__(1024) reduce_loss_kernel(const double* __restr
 
 // ------------------------------------------------------------------ host side
 
+rl_status launch_reduce_loss(const double* row_loss, int64_t rows, double* loss_accum, cudaStream_t s) {
+  reduce_loss_kernel<<<1, 1024, 0, s>>>(row_loss, rows, loss_accum);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_error(e, "reduce_loss_kernel launch");
+  return RL_OK;
+}
+
 constexpr int kConsumerWarps = RL_CONSUMER_WARPS;
 constexpr int kRowThreads = (RL_CONSUMER_WARPS + 1) * 32;
 constexpr int64_t kTargetSliceBytes = RL_SLICE_KB * 1024;
@@ -1103,8 +1110,5 @@ extern "C" rl_status rl_policy_loss_fwd_bwd(const void* logits, rl_dtype dtype, 
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   st = dtype == RL_BF16 ? dispatch_loss<uint16_t>(ent, a, plan, s) : dispatch_loss<float>(ent, a, plan, s);
   if (st != RL_OK) return st;
-  reduce_loss_kernel<<<1, 1024, 0, s>>>(row_loss, rows, loss_accum);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return cuda_error(e, "reduce_loss_kernel launch");
-  return RL_OK;
+  return launch_reduce_loss(row_loss, rows, loss_accum, s);
 }

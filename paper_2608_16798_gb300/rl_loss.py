@@ -40,6 +40,8 @@ EXPORTS = {
                                       _P, _P, _P, _P, _SZ, _P]),
     "rl_policy_loss_fwd_bwd_noalloc": (_I32, [_P, _I32, _I64, _I64, _I64, _P, _P, _P, _I32, _P, _P, _P, _P, _P,
                                               _P, _P, _P, _P, _P, _P]),
+    "rl_fused_head_loss_fwd_bwd": (_I32, [_P, _P, _I64, _I64, _I64, _P, _P, _P, _I32, _P, _P, _P, _P, _P, _P, _P,
+                                          _I32, _P, _P, _P, _P, _SZ, _P]),
 }
 
 
@@ -285,3 +287,42 @@ def rl_policy_loss_fwd_bwd_noalloc(logits, token_ids, mask, token_traj, adv, coe
                                               _ptr(device_status), _stream(stream))
     _check("rl_policy_loss_fwd_bwd_noalloc", st)
     return grad_out
+
+
+def rl_fused_head_loss_fwd_bwd(hidden, weight, token_ids, mask, token_traj, adv, coef, old_logp,
+                               params: rl_loss_params, ws, loss_accum, d_weight, d_hidden=None,
+                               d_hidden_dtype=torch.bfloat16, ref_logp=None, rollout_logp=None, token_stats=None,
+                               stream=None):
+    """Loss of the LM head hidden @ weight^T without materialising the logits; returns d_hidden
+    (overwritten) and adds d loss / d weight into ``d_weight`` (float32 [V, D])."""
+    if hidden.dim() != 2 or weight.dim() != 2 or hidden.shape[1] != weight.shape[1]:
+        raise ValueError("hidden [T, D] and weight [V, D] must share D")
+    T, D = hidden.shape
+    V = weight.shape[0]
+    dev = hidden.device
+    n_traj = adv.numel()
+    _need(hidden, "hidden", torch.bfloat16, device=dev)
+    _need(weight, "weight", torch.bfloat16, device=dev)
+    _need(token_ids, "token_ids", torch.int32, T, device=dev)
+    _need(mask, "mask", torch.uint8, T, device=dev)
+    _need(token_traj, "token_traj", torch.int32, T, device=dev)
+    _need(adv, "adv", torch.float32, device=dev)
+    _need(coef, "coef", torch.float32, n_traj, device=dev)
+    _need(old_logp, "old_logp", torch.float32, T, device=dev)
+    _opt(ref_logp, "ref_logp", torch.float32, T, device=dev)
+    _opt(rollout_logp, "rollout_logp", torch.float32, T, device=dev)
+    _need(loss_accum, "loss_accum", torch.float64, 1, device=dev)
+    _opt(token_stats, "token_stats", torch.float32, T * 5, device=dev)
+    _need(d_weight, "d_weight", torch.float32, V * D, device=dev)
+    if d_hidden is None:
+        d_hidden = torch.empty((T, D), dtype=d_hidden_dtype, device=dev)
+    _need(d_hidden, "d_hidden", d_hidden.dtype, T * D, device=dev)
+    dt = _logits_dtype(d_hidden)
+    _need(ws, "ws", torch.uint8, device=dev)
+    st = lib().rl_fused_head_loss_fwd_bwd(_ptr(hidden), _ptr(weight), T, D, V, _ptr(token_ids), _ptr(mask),
+                                          _ptr(token_traj), n_traj, _ptr(adv), _ptr(coef), _ptr(old_logp),
+                                          _ptr(ref_logp), _ptr(rollout_logp), ctypes.byref(params), _ptr(d_hidden),
+                                          dt, _ptr(d_weight), _ptr(loss_accum), _ptr(token_stats), _ptr(ws),
+                                          ws.numel(), _stream(stream))
+    _check("rl_fused_head_loss_fwd_bwd", st)
+    return d_hidden

@@ -1,0 +1,146 @@
+"""Fused LM head (logits = hidden @ W^T never materialised) against the float64 oracle.
+
+The library rounds the logits' gradient dZ to bf16 before the two products
+dH = dZ W and dW = dZ^T H, so their elements carry independent rounding errors of at
+most 2^-9 relative per term: the bound used is 6 * 2^-9 * sqrt(sum of squared terms)
+(computed exactly in float64) plus 1e-4 of the element and 1e-6 of the largest
+element for the float32 parts. Loss, clip flags and per-token statistics use the
+logits-path tolerances.
+"""
+
+import dataclasses
+
+import numpy as np
+import pytest
+import torch
+
+import oracle.grpo_objective as O
+from parity_cases import check_loss, check_stats, cuda_params, to_dev
+from paper_2608_16798_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def R():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_16798_gb300 import build
+
+    build.build()
+    import paper_2608_16798_gb300.rl_loss as R
+
+    R.lib()
+    return R
+
+
+def _bf16_dev(bits):
+    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).cuda()
+
+
+def make_head_case(T, D, V, seed=0, masked=0.3, agg=0, ent=False, tis=False, wstd=0.05):
+    w = dataclasses.replace(W.WORKLOADS["fusedhead"], weight_std=wstd)
+    h_bits, w_bits = W.hidden_and_weight_np(w, seed, T, V, D)
+    Z = O.decode_logits(h_bits, "bf16") @ O.decode_logits(w_bits, "bf16").T
+    rng = np.random.default_rng(seed + 1)
+    gumbel = -np.log(-np.log(rng.random(Z.shape)))
+    ids = np.argmax(Z + gumbel, axis=1).astype(np.int32)
+    lse, logp, H, _, _ = O.row_statistics(Z, ids)
+    n_traj = max(4, (T // 50) // 4 * 4)
+    cuts = np.sort(rng.choice(np.arange(1, T), size=n_traj - 1, replace=False))
+    offs = np.concatenate([[0], cuts, [T]]).astype(np.int64)
+    mask = (rng.random(T) >= masked).astype(np.uint8)
+    rewards = (rng.random(n_traj) < 0.4).astype(np.float32)
+    go = np.arange(0, n_traj + 1, 4, dtype=np.int32)
+    P = O.LossParams(entropy_coef=1e-2 if ent else 0.0, kl_coef=2e-2 if ent else 0.0, kl_estimator=3 if ent else 0,
+                     tis_cap=2.0 if tis else 0.0, loss_agg=agg)
+    adv, coef, L, tt = O.advantages_and_coefficients(rewards, go, offs, mask, None, P)
+    delta = rng.uniform(-0.5, 0.5, size=T)
+    for b in (np.log(0.8), np.log(1.28)):
+        delta = np.where(np.abs(delta - b) < 1e-3, delta + 3e-3, delta)
+    old = (logp - delta).astype(np.float32)
+    ref = (logp + rng.normal(0, 0.2, size=T)).astype(np.float32) if ent else None
+    roll = (old + rng.normal(0, 0.3, size=T)).astype(np.float32) if tis else None
+    return dict(h=h_bits, w=w_bits, ids=ids, mask=mask, tt=tt, adv32=adv.astype(np.float32),
+                coef32=coef.astype(np.float32), old=old, ref=ref, roll=roll, P=P, T=T, D=D, V=V)
+
+
+def run_head(R, c, dh_dtype=torch.float32):
+    T, D, V = c["T"], c["D"], c["V"]
+    ws = R.new_workspace(T, V, D)
+    loss = torch.zeros(1, dtype=torch.float64, device="cuda")
+    dW = torch.zeros((V, D), dtype=torch.float32, device="cuda")
+    st = torch.zeros(T * 5, dtype=torch.float32, device="cuda")
+    dH = R.rl_fused_head_loss_fwd_bwd(_bf16_dev(c["h"]), _bf16_dev(c["w"]), to_dev(c["ids"]), to_dev(c["mask"]),
+                                      to_dev(c["tt"].astype(np.int32)), to_dev(c["adv32"]), to_dev(c["coef32"]),
+                                      to_dev(c["old"]), cuda_params(R, c["P"]), ws, loss, dW,
+                                      d_hidden_dtype=dh_dtype,
+                                      ref_logp=None if c["ref"] is None else to_dev(c["ref"]),
+                                      rollout_logp=None if c["roll"] is None else to_dev(c["roll"]), token_stats=st)
+    status, word = R.rl_query_status(ws)
+    return dict(loss=loss.item(), dH=dH.float().cpu().numpy().astype(np.float64),
+                dW=dW.cpu().numpy().astype(np.float64), stats=st.view(-1, 5).cpu().numpy(), word=word)
+
+
+def check_product(got, ref, S, what):
+    tol = 6 * 2.0 ** -9 * S + 1e-4 * np.abs(ref) + 1e-6 * np.abs(ref).max() + 1e-30
+    bad = np.abs(got - ref) > tol
+    if bad.any():
+        i, j = np.argwhere(bad)[0]
+        raise AssertionError(f"{what}: {bad.sum()} elements out of tolerance, e.g. [{i},{j}] "
+                             f"gpu {got[i, j]} oracle {ref[i, j]} tol {tol[i, j]}")
+
+
+def compare_head(c, out, dh_bf16=False):
+    P = c["P"]
+    adv, coef = c["adv32"].astype(np.float64), c["coef32"].astype(np.float64)
+    loss, dH, dW, stats = O.fused_head_loss_fwd_bwd(c["h"], c["w"], c["ids"], c["mask"], c["tt"], adv, coef, c["old"],
+                                                    P, c["ref"], c["roll"])
+    Hm, Wm = O.decode_logits(c["h"], "bf16"), O.decode_logits(c["w"], "bf16")
+    Z = Hm @ Wm.T
+    _, dZ, _, contrib = O.policy_loss_fwd_bwd(Z, "f64", c["ids"], c["mask"], c["tt"], adv, coef, c["old"], P, c["ref"],
+                                              c["roll"])
+    check_loss(out["loss"], loss, contrib, "fused head loss")
+    active = (c["mask"] != 0) & (coef[c["tt"]] != 0)
+    check_stats(out["stats"], stats, active, "fused head stats")
+    S_h = np.sqrt((dZ ** 2) @ (Wm ** 2))
+    S_w = np.sqrt((dZ.T ** 2) @ (Hm ** 2))
+    if dh_bf16:
+        S_h = S_h + 2.0 ** 8 * np.abs(dH) / 6  # plus half an ulp of the bf16 output
+    check_product(out["dH"], dH, S_h, "d_hidden")
+    check_product(out["dW"], dW, S_w, "d_weight")
+    assert np.all(out["dH"][~active] == 0.0), "tokens that are not trained on must get zero d_hidden rows"
+    assert out["word"] == 0
+
+
+@pytest.mark.parametrize("T,D,V,agg,ent,tis", [
+    (300, 256, 1000, 2, False, False),     # ragged M tile and vocabulary tile
+    (256, 128, 8292, 0, False, False),     # three vocabulary blocks
+    (200, 192, 700, 2, True, False),       # entropy + k3 KL
+    (130, 64, 513, 1, False, True),        # TIS, token-mean, smallest D
+])
+def test_fused_head_parity(R, T, D, V, agg, ent, tis):
+    c = make_head_case(T, D, V, seed=T + V, agg=agg, ent=ent, tis=tis)
+    out = run_head(R, c)
+    compare_head(c, out)
+
+
+def test_fused_head_two_chunks_bf16_grad(R):
+    """More than 8,192 tokens: two chunks, dW accumulated across them; bf16 d_hidden."""
+    c = make_head_case(8192 + 77, 128, 1100, seed=5, agg=2)
+    out = run_head(R, c, dh_dtype=torch.bfloat16)
+    compare_head(c, out, dh_bf16=True)
+
+
+def test_fused_head_matches_logits_path(R):
+    """The fused head's loss equals rl_policy_loss_fwd_bwd on the materialised fp32 logits."""
+    c = make_head_case(384, 256, 2048, seed=9, agg=0)
+    out = run_head(R, c)
+    Z = torch.from_numpy(O.decode_logits(c["h"], "bf16")) @ torch.from_numpy(O.decode_logits(c["w"], "bf16")).T
+    z32 = Z.float().cuda()
+    ws = R.new_workspace(c["T"], c["V"])
+    loss = torch.zeros(1, dtype=torch.float64, device="cuda")
+    R.rl_policy_loss_fwd_bwd(z32, to_dev(c["ids"]), to_dev(c["mask"]), to_dev(c["tt"].astype(np.int32)),
+                             to_dev(c["adv32"]), to_dev(c["coef32"]), to_dev(c["old"]), cuda_params(R, c["P"]), ws,
+                             loss)
+    assert abs(loss.item() - out["loss"]) <= 1e-4 * max(abs(loss.item()), 1e-12)
