@@ -431,6 +431,111 @@ def run_reference(args):
     return 0
 
 
+HEAD = W.WORKLOADS["fusedhead"]
+HEAD_T = 32768
+
+
+class HeadBatch:
+    """Fused-LM-head workload on the device: hidden bf16 [T x 4096] ~ N(0, 1), W bf16 [151,936 x 4096]
+    ~ N(0, 0.02^2); masks and trajectories of the first T packed tokens of a multi-turn batch, advantages
+    and coefficients from that whole batch; sampled ids drawn from softmax(hidden W^T) by Gumbel-max
+    (the logits for this draw come from a torch matmul in the set-up, not from the library).
+    old_logp sits near the sampled token's log-probability: z_a minus the log-sum-exp of V logits
+    distributed N(0, |h_t|^2 0.02^2), ln V + |h_t|^2 0.02^2 / 2, minus the workload's log-ratio noise."""
+
+    def __init__(self, torch, R, dev, T=HEAD_T, seed=0):
+        t = torch
+        w = HEAD
+        self.T, self.D, self.V = T, w.hidden, w.vocab
+        self.hidden = t.empty((T, self.D), dtype=t.bfloat16, device=dev)
+        self.weight = t.empty((self.V, self.D), dtype=t.bfloat16, device=dev)
+        W.hidden_and_weight_torch(w, seed, T, self.hidden, self.weight)
+        ids = t.empty(T, dtype=t.int32, device=dev)
+        za = t.empty(T, dtype=t.float32, device=dev)
+        g = t.Generator(device=dev)
+        for r0 in range(0, T, 1024):
+            r1 = min(T, r0 + 1024)
+            z = t.matmul(self.hidden[r0:r1], self.weight.t()).float()
+            g.manual_seed(seed * 7_000_003 + r0)
+            u = t.rand(z.shape, generator=g, device=dev).clamp_(min=1e-30).log_().neg_().log_().neg_()
+            a = t.argmax(z + u, dim=1)
+            ids[r0:r1] = a.to(t.int32)
+            za[r0:r1] = z.gather(1, a[:, None])[:, 0]
+            del z, u
+        lay = W.make_layout(w, seed)
+        d = lambda x: t.from_numpy(np.ascontiguousarray(x)).to(dev)  # noqa: E731
+        self.params = R.make_params(W.CLIP_EPS_LOW, W.CLIP_EPS_HIGH, 0.0, 0, 0.0, 0.0, 1e-6, 0)
+        ws_adv = R.new_workspace(0, 0, device=dev)
+        self.adv, self.coef, _, tt = R.rl_group_advantages(d(lay.group_offsets), d(lay.rewards),
+                                                           d(lay.traj_offsets), d(lay.mask), self.params, ws_adv)
+        self.token_traj = tt[:T].contiguous()
+        self.mask = d(lay.mask[:T])
+        self.ids = ids
+        h2 = self.hidden.float().pow(2).sum(dim=1) * (w.weight_std ** 2)
+        logp_hat = (za - (math.log(self.V) + h2 / 2)).cpu().numpy()
+        self.old = d(W.old_logp_from(logp_hat, w, seed))
+        self.ws = R.new_workspace(T, self.V, self.D, device=dev)
+        self.loss = t.zeros(1, dtype=t.float64, device=dev)
+        self.dW = t.zeros((self.V, self.D), dtype=t.float32, device=dev)
+        self.dH = t.empty((T, self.D), dtype=t.bfloat16, device=dev)
+        self.trained = int(lay.mask[:T].sum())
+
+    def call(self, R):
+        R.rl_fused_head_loss_fwd_bwd(self.hidden, self.weight, self.ids, self.mask, self.token_traj, self.adv,
+                                     self.coef, self.old, self.params, self.ws, self.loss, self.dW, d_hidden=self.dH)
+
+
+def time_head(torch, R, dev, warmup=2, reps=5):
+    hb = HeadBatch(torch, R, dev)
+    for _ in range(warmup):
+        hb.call(R)
+    torch.cuda.synchronize(dev)
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(reps):
+        hb.call(R)
+    b.record()
+    b.synchronize()
+    st, word = R.rl_query_status(hb.ws)
+    if word != 0:
+        raise RuntimeError(f"device status word {word} after the fused-head timing")
+    ms = a.elapsed_time(b) / reps
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    burst, sustained, kind = 1900.0, 1700.0, "fallback"
+    if os.path.exists(p):
+        with open(p) as f:
+            pk = json.load(f)
+        burst, sustained, kind = float(pk["bf16_tflops"]), float(pk["bf16_tflops_sustained"]), "measured"
+    flops = 6.0 * hb.T * hb.D * hb.V
+    tf = flops / (ms * 1e-3) / 1e12
+    chunks = (hb.T + 8191) // 8192
+    return {"workload": f"fusedhead: hidden bf16 [{hb.T} x {hb.D}] N(0,1), W bf16 [{hb.V} x {hb.D}] N(0,0.02^2), "
+                        f"masks and coefficients of the first {hb.T} multiturn tokens ({hb.trained} trained)",
+            "ms_per_call": ms, "tokens_per_s": hb.T / (ms * 1e-3), "bound": "tensor", "achieved": tf,
+            "peak": burst, "unit": "TFLOP/s", "frac": tf / burst, "frac_of_sustained": tf / sustained,
+            "peak_source": kind, "algorithmic_flops_per_call": flops, "executed_flops_per_call": 8.0 * hb.T * hb.D * hb.V,
+            "reps": reps, "chunks_per_call": chunks,
+            "note": "algorithmic 6 T D V (Z, dH, dW); executed 8 T D V (Z is computed twice); dH and dW through cuBLASLt"}
+
+
+def profile_head(T):
+    """A small fused-head case for profiler captures: three calls on the first T tokens."""
+    import torch
+
+    from paper_2608_16798_gb300 import build as B
+
+    B.build()
+    import paper_2608_16798_gb300.rl_loss as R
+
+    dev = torch.device("cuda", 0)
+    hb = HeadBatch(torch, R, dev, T=T)
+    for _ in range(3):
+        hb.call(R)
+    st, word = R.rl_query_status(hb.ws)
+    print(json.dumps({"profile_head_tokens": T, "status": word, "flops_per_call": 6.0 * T * hb.D * hb.V}))
+    return 0 if word == 0 else 1
+
+
 def profile_case(rows):
     """A small slice of the workload for profiler captures: the first `rows` packed tokens
     (logits resident on the device), then three rl_policy_loss_fwd_bwd launches and three
@@ -482,9 +587,14 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--profile-case", type=int, default=0, metavar="ROWS",
                     help="run a small slice of the workload for a profiler capture and exit")
+    ap.add_argument("--profile-head", type=int, default=0, metavar="TOKENS",
+                    help="run a small fused-head case for a profiler capture and exit")
+    ap.add_argument("--no-head", action="store_true", help="skip the fused-head measurement")
     args = ap.parse_args()
     if args.profile_case:
         return profile_case(args.profile_case)
+    if args.profile_head:
+        return profile_head(args.profile_head)
     if args.impl == "reference":
         return run_reference(args)
     args.warmup = max(3, args.warmup)
@@ -559,11 +669,15 @@ def main():
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = time_oracle(host_sample(torch, batch, 2048))
 
+    head = None
+    if not args.no_head:
+        head = time_head(torch, R, dev)
+
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": "f32", "data": "synthetic", "config": workload_config(batch.T, n_mb),
-                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks,
+                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks, "fused_head": head,
                 "gpu_launches": batch.launches_per_step() * args.steps,
                 "loss_per_step": float(batch.loss.item()) / (args.warmup + args.steps)}
         print(json.dumps(line))

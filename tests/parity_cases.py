@@ -19,6 +19,8 @@ Tolerances (float32 kernels against the float64 oracle):
   entropy    |d| <= 5e-5 + 2e-5 |H|
   KL         |d| <= 1e-6 + 1e-4 |KL|
   clipped flag, token owners, counts, masked / inactive rows: bit-exact
+  fused head: logits formed on the GPU add a per-token allowance zerr to logp, ratio,
+             entropy and KL (logit_error_bound)
 """
 
 from __future__ import annotations
@@ -162,13 +164,26 @@ def check_loss(loss_dev, loss_ref, contrib_ref, what=""):
     assert abs(loss_dev - loss_ref) <= 1e-4 * scale + 1e-300, f"{what}: loss {loss_dev} vs {loss_ref} (scale {scale})"
 
 
-def check_stats(st_dev, st_ref, active, what=""):
+def logit_error_bound(hidden_f64, weight_f64):
+    """Per-token bound on the error of logits the GPU forms itself (fused head): z = h . w
+    accumulated in fp32 over D products has partial sums bounded by |h| |w| (Cauchy-Schwarz)
+    and roundings of at most 2^-24 of them that add like a random walk over D terms, so
+    |dz| <= 2^-24 sqrt(D) |h_t| max_v |w_v|; logp = z_a - lse carries two such errors."""
+    D = hidden_f64.shape[1]
+    wmax = np.sqrt((weight_f64 ** 2).sum(axis=1)).max()
+    return 2 * 2.0 ** -24 * np.sqrt(D) * np.sqrt((hidden_f64 ** 2).sum(axis=1)) * wmax
+
+
+def check_stats(st_dev, st_ref, active, what="", zerr=None):
+    """zerr (per row, optional): error allowance of logits formed on the GPU (see logit_error_bound)."""
     st_dev = st_dev.astype(np.float64)
     assert np.all(st_dev[~active] == 0.0), f"{what}: stats of inactive rows not zero"
     a, b = st_dev[active], st_ref[active]
+    z = np.zeros(len(a)) if zerr is None else np.broadcast_to(zerr, active.shape)[active]
     d = np.abs(a - b)
-    assert np.all(d[:, 0] <= 1e-5 + 2.0 ** -22 * np.abs(b[:, 0])), f"{what}: logp max diff {d[:, 0].max()}"
-    assert np.all(d[:, 1] <= 2e-5 * np.abs(b[:, 1])), f"{what}: ratio max rel diff {(d[:, 1] / b[:, 1]).max()}"
+    assert np.all(d[:, 0] <= 1e-5 + 2.0 ** -22 * np.abs(b[:, 0]) + z), f"{what}: logp max diff {d[:, 0].max()}"
+    assert np.all(d[:, 1] <= (2e-5 + z) * np.abs(b[:, 1])), f"{what}: ratio max rel diff {(d[:, 1] / b[:, 1]).max()}"
     assert np.array_equal(a[:, 2], b[:, 2]), f"{what}: clipped flags differ"
-    assert np.all(d[:, 3] <= 5e-5 + 2e-5 * np.abs(b[:, 3])), f"{what}: entropy max diff {d[:, 3].max()}"
-    assert np.all(d[:, 4] <= 1e-6 + 1e-4 * np.abs(b[:, 4])), f"{what}: KL max diff {d[:, 4].max()}"
+    assert np.all(d[:, 3] <= 5e-5 + 2e-5 * np.abs(b[:, 3]) + 2 * z), f"{what}: entropy max diff {d[:, 3].max()}"
+    assert np.all(d[:, 4] <= 1e-6 + 1e-4 * np.abs(b[:, 4]) + 2 * z * (1 + np.abs(b[:, 4]))), \
+        f"{what}: KL max diff {d[:, 4].max()}"

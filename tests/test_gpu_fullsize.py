@@ -15,7 +15,8 @@ import torch
 
 import oracle.grpo_objective as O
 from oracle.pool import token_logprobs_parallel
-from parity_cases import check_grad, check_loss, check_stats, cuda_params, grad_to_np, loss_params, to_dev
+from parity_cases import (check_grad, check_loss, check_stats, cuda_params, grad_to_np, logit_error_bound, loss_params,
+                          to_dev)
 from paper_2608_16798_gb300 import workloads as W
 
 pytestmark = [pytest.mark.gpu, pytest.mark.slow]
@@ -119,3 +120,92 @@ def test_full_microbatch(R, name, mb):
     scale = (np.abs(c_row[sample]) * (np.abs(adv32.astype(np.float64)[tt_mb][sample]) * stats_ref[sample, 1]
                                       + P.kl_coef * 2 + P.entropy_coef * (1 + np.abs(H[sample]))))[:, None]
     check_grad(g_dev, g_ref, w.dtype, f"{name} mb {mb} sampled rows", row_scale=scale)
+
+
+def test_fused_head_full_size(R):
+    """The fused LM head at 32,768 x 4,096 x 151,936 (four chunks), as the benchmark calls it.
+
+    The oracle forms every token's logits row in float64 (host GEMM blocks) for lse and the
+    entropy; old_logp follows from them. Loss and statistics are checked for every token,
+    d_hidden on sampled tokens, d_weight on sampled vocabulary rows (their column of dZ over
+    all tokens), with the bf16-dZ bound of test_gpu_fused_head.py."""
+    w = W.WORKLOADS["fusedhead"]
+    T, D, V, seed = 32768, w.hidden, w.vocab, 0
+    hidden = torch.empty((T, D), dtype=torch.bfloat16, device="cuda")
+    weight = torch.empty((V, D), dtype=torch.bfloat16, device="cuda")
+    W.hidden_and_weight_torch(w, seed, T, hidden, weight)
+    Hm = O.decode_logits(_host_raw(hidden, "bf16"), "bf16")
+    Wm = O.decode_logits(_host_raw(weight, "bf16"), "bf16")
+    rng = np.random.default_rng(17)
+    # sampled ids: Gumbel-max over softmax(hidden W^T), drawn on the device (input synthesis)
+    ids_d = torch.empty(T, dtype=torch.int32, device="cuda")
+    g = torch.Generator(device="cuda")
+    for r0 in range(0, T, 1024):
+        g.manual_seed(1000 + r0)
+        z = torch.matmul(hidden[r0:r0 + 1024], weight.t()).float()
+        u = torch.rand(z.shape, generator=g, device="cuda").clamp_(min=1e-30).log_().neg_().log_().neg_()
+        ids_d[r0:r0 + 1024] = torch.argmax(z + u, dim=1).to(torch.int32)
+        del z, u
+    ids = ids_d.cpu().numpy()
+    lse, H, z_a = np.empty(T), np.empty(T), np.empty(T)
+    for r0 in range(0, T, 1024):
+        Z = Hm[r0:r0 + 1024] @ Wm.T
+        l, _, h, _, za = O.row_statistics(Z, ids[r0:r0 + 1024])
+        lse[r0:r0 + 1024], H[r0:r0 + 1024], z_a[r0:r0 + 1024] = l, h, za
+        del Z
+    logp = z_a - lse
+    lay = W.make_layout(w, seed)
+    P = loss_params(w)
+    adv, coef, L, tt = O.advantages_and_coefficients(lay.rewards, lay.group_offsets, lay.traj_offsets, lay.mask,
+                                                     lay.traj_valid, P)
+    adv32, coef32 = adv.astype(np.float32), coef.astype(np.float32)
+    mask, tt_t = lay.mask[:T], tt[:T]
+    old = W.old_logp_from(logp, w, seed)
+
+    ws = R.new_workspace(T, V, D)
+    loss = torch.zeros(1, dtype=torch.float64, device="cuda")
+    st = torch.zeros(T * 5, dtype=torch.float32, device="cuda")
+    dW = torch.zeros((V, D), dtype=torch.float32, device="cuda")
+    dH = R.rl_fused_head_loss_fwd_bwd(hidden, weight, to_dev(ids), to_dev(mask), to_dev(tt_t.astype(np.int32)),
+                                      to_dev(adv32), to_dev(coef32), to_dev(old), cuda_params(R, P), ws, loss, dW,
+                                      d_hidden_dtype=torch.float32, token_stats=st)
+    assert R.rl_query_status(ws)[1] == 0
+
+    A_t, c_t = adv32.astype(np.float64)[tt_t], coef32.astype(np.float64)[tt_t]
+    terms = O.token_terms(z_a, lse, H, old, A_t, P)
+    active = (mask != 0) & (c_t != 0)
+    contrib = np.where(active, c_t * terms["ell"], 0.0)
+    check_loss(loss.item(), math.fsum(contrib.tolist()), contrib, "fused head full-size loss")
+    stats_ref = np.stack([terms["logp"], terms["rho"], terms["cut"], H, terms["kl"]], axis=1)
+    stats_ref[~active] = 0.0
+    check_stats(st.view(-1, 5).cpu().numpy(), stats_ref, active, "fused head full-size stats",
+                zerr=logit_error_bound(Hm, Wm))
+
+    # dZ rows of sampled tokens and dZ columns of sampled vocabulary entries, in float64
+    g_t = np.where(active, c_t * terms["g"], 0.0)
+
+    def dz_rows(rows):
+        Z = Hm[rows] @ Wm.T
+        p = np.exp(Z - lse[rows, None])
+        dz = -g_t[rows, None] * p
+        dz[np.arange(len(rows)), ids[rows]] += g_t[rows]
+        return dz
+
+    act_idx = np.nonzero(active)[0]
+    rows = np.unique(np.concatenate([rng.choice(act_idx, 24, replace=False), np.nonzero(~active)[0][:4]]))
+    dz = dz_rows(rows)
+    ref_dH = dz @ Wm
+    S_h = np.sqrt((dz ** 2) @ (Wm ** 2))
+    got = dH.index_select(0, torch.from_numpy(rows).cuda()).cpu().numpy().astype(np.float64)
+    tol = 6 * 2.0 ** -9 * S_h + 1e-4 * np.abs(ref_dH) + 1e-6 * np.abs(ref_dH).max() + 1e-30
+    assert np.all(np.abs(got - ref_dH) <= tol), np.abs(got - ref_dH).max()
+
+    vs = np.unique(np.concatenate([ids[rng.choice(act_idx, 8, replace=False)], rng.integers(0, V, 24)]))
+    Zc = Hm @ Wm[vs].T                                     # [T x |vs|]
+    p = np.exp(Zc - lse[:, None])
+    dzc = -g_t[:, None] * p + g_t[:, None] * (ids[:, None] == vs[None, :])
+    ref_dW = dzc.T @ Hm                                    # [|vs| x D]
+    S_w = np.sqrt((dzc.T ** 2) @ (Hm ** 2))
+    got = dW.index_select(0, torch.from_numpy(vs).cuda()).cpu().numpy().astype(np.float64)
+    tol = 6 * 2.0 ** -9 * S_w + 1e-4 * np.abs(ref_dW) + 1e-6 * np.abs(ref_dW).max() + 1e-30
+    assert np.all(np.abs(got - ref_dW) <= tol), np.abs(got - ref_dW).max()

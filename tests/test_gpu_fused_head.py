@@ -15,7 +15,7 @@ import pytest
 import torch
 
 import oracle.grpo_objective as O
-from parity_cases import check_loss, check_stats, cuda_params, to_dev
+from parity_cases import check_loss, check_stats, cuda_params, logit_error_bound, to_dev
 from paper_2608_16798_gb300 import workloads as W
 
 pytestmark = pytest.mark.gpu
@@ -102,7 +102,8 @@ def compare_head(c, out, dh_bf16=False):
                                               c["roll"])
     check_loss(out["loss"], loss, contrib, "fused head loss")
     active = (c["mask"] != 0) & (coef[c["tt"]] != 0)
-    check_stats(out["stats"], stats, active, "fused head stats")
+    Hm, Wm = O.decode_logits(c["h"], "bf16"), O.decode_logits(c["w"], "bf16")
+    check_stats(out["stats"], stats, active, "fused head stats", zerr=logit_error_bound(Hm, Wm))
     S_h = np.sqrt((dZ ** 2) @ (Wm ** 2))
     S_w = np.sqrt((dZ.T ** 2) @ (Hm ** 2))
     if dh_bf16:
