@@ -30,6 +30,7 @@ Every function follows one passage of the paper (arXiv 2608.16798, "ClawGym II")
   pi_ref recompute of Sec. 3.2.4).
 * ``fused_head_loss_fwd_bwd``  -- the same objective with logits = hidden @ W^T
   and gradients with respect to hidden and W.
+* ``fused_head_logprobs``      -- forward-only log-probabilities of logits = hidden @ W^T.
 
 Readings of the paper where it is silent (all documented with the library):
 
@@ -363,3 +364,18 @@ def fused_head_loss_fwd_bwd(hidden_bf16, weight_bf16, token_ids, mask, token_tra
     d_hidden = dZ @ Wm
     d_weight = dZ.T @ Hm
     return loss, d_hidden, d_weight, stats
+
+
+def fused_head_logprobs(hidden_bf16, weight_bf16, token_ids, chunk: int = 256):
+    """Forward-only logp, entropy and lse of the sampled ids for logits Z = H W^T (float64):
+    the pi_old / pi_ref recompute of Sec. 3.2.4 on the LM head's output."""
+    Hm = decode_logits(hidden_bf16, "bf16")
+    Wm = decode_logits(weight_bf16, "bf16")
+    T = Hm.shape[0]
+    token_ids = np.asarray(token_ids, dtype=np.int64)
+    logp, H, lse = np.zeros(T), np.zeros(T), np.zeros(T)
+    for r0 in range(0, T, chunk):
+        Z = Hm[r0:r0 + chunk] @ Wm.T
+        l, lp, h, _, _ = row_statistics(Z, token_ids[r0:r0 + chunk])
+        lse[r0:r0 + chunk], logp[r0:r0 + chunk], H[r0:r0 + chunk] = l, lp, h
+    return logp, H, lse

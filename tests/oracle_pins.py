@@ -516,4 +516,23 @@ def pin_fused_head_zero_hidden(O):
     assert np.all(dW == 0.0)  # hidden = 0 -> dW = dZ^T H = 0
 
 
+def pin_fused_head_logprobs_vs_library(O):
+    """Forward-only fused-head log-probs against float64 torch.log_softmax(H W^T), and the
+    uniform case (zero hidden rows: logp = -ln V, H = ln V)."""
+    import torch
+
+    rng = np.random.default_rng(12)
+    h = _bf16(rng.normal(0, 1, size=(5, 64)))
+    w = _bf16(rng.normal(0, 0.3, size=(40, 64)))
+    h[3] = 0
+    a = rng.integers(0, 40, size=5)
+    logp, H, lse = O.fused_head_logprobs(h, w, a, chunk=2)
+    Z = torch.from_numpy(_unbf16(h)) @ torch.from_numpy(_unbf16(w)).T
+    ls = torch.log_softmax(Z, dim=1).numpy()
+    _close(logp, ls[np.arange(5), a], rtol=1e-12, atol=1e-12, what="fused logp vs torch")
+    _close(lse, torch.logsumexp(Z, dim=1).numpy(), rtol=1e-12, atol=1e-12, what="fused lse vs torch")
+    _close(H, -(np.exp(ls) * ls).sum(axis=1), rtol=1e-10, atol=1e-12, what="fused entropy")
+    _close([logp[3], H[3]], [-math.log(40), math.log(40)], what="zero hidden row")
+
+
 ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_")]
