@@ -479,27 +479,38 @@ class HeadBatch:
         self.dW = t.zeros((self.V, self.D), dtype=t.float32, device=dev)
         self.dH = t.empty((T, self.D), dtype=t.bfloat16, device=dev)
         self.trained = int(lay.mask[:T].sum())
+        self.logp = t.empty(T, dtype=t.float32, device=dev)
+        self.ent = t.empty(T, dtype=t.float32, device=dev)
 
     def call(self, R):
         R.rl_fused_head_loss_fwd_bwd(self.hidden, self.weight, self.ids, self.mask, self.token_traj, self.adv,
                                      self.coef, self.old, self.params, self.ws, self.loss, self.dW, d_hidden=self.dH)
 
+    def call_logprobs(self, R):
+        R.rl_fused_head_token_logprobs(self.hidden, self.weight, self.ids, self.ws, logp_out=self.logp,
+                                       entropy_out=self.ent)
 
-def time_head(torch, R, dev, warmup=2, reps=5):
-    hb = HeadBatch(torch, R, dev)
+
+def _time_calls(torch, fn, warmup, reps):
     for _ in range(warmup):
-        hb.call(R)
-    torch.cuda.synchronize(dev)
+        fn()
+    torch.cuda.synchronize()
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     a.record()
     for _ in range(reps):
-        hb.call(R)
+        fn()
     b.record()
     b.synchronize()
+    return a.elapsed_time(b) / reps
+
+
+def time_head(torch, R, dev, warmup=2, reps=5):
+    hb = HeadBatch(torch, R, dev)
+    ms = _time_calls(torch, lambda: hb.call(R), warmup, reps)
+    ms_fwd = _time_calls(torch, lambda: hb.call_logprobs(R), warmup, reps)
     st, word = R.rl_query_status(hb.ws)
     if word != 0:
         raise RuntimeError(f"device status word {word} after the fused-head timing")
-    ms = a.elapsed_time(b) / reps
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     burst, sustained, kind = 1900.0, 1700.0, "fallback"
     if os.path.exists(p):
@@ -509,17 +520,23 @@ def time_head(torch, R, dev, warmup=2, reps=5):
     flops = 6.0 * hb.T * hb.D * hb.V
     tf = flops / (ms * 1e-3) / 1e12
     chunks = (hb.T + 8191) // 8192
+    tf_fwd = 2.0 * hb.T * hb.D * hb.V / (ms_fwd * 1e-3) / 1e12
+    fwd = {"ms_per_call": ms_fwd, "tokens_per_s": hb.T / (ms_fwd * 1e-3), "achieved": tf_fwd, "frac": tf_fwd / burst,
+           "frac_of_sustained": tf_fwd / sustained, "algorithmic_flops_per_call": 2.0 * hb.T * hb.D * hb.V,
+           "note": "rl_fused_head_token_logprobs with entropy: one tensor-core pass (2 T D V) and the merge"}
     return {"workload": f"fusedhead: hidden bf16 [{hb.T} x {hb.D}] N(0,1), W bf16 [{hb.V} x {hb.D}] N(0,0.02^2), "
                         f"masks and coefficients of the first {hb.T} multiturn tokens ({hb.trained} trained)",
             "ms_per_call": ms, "tokens_per_s": hb.T / (ms * 1e-3), "bound": "tensor", "achieved": tf,
             "peak": burst, "unit": "TFLOP/s", "frac": tf / burst, "frac_of_sustained": tf / sustained,
             "peak_source": kind, "algorithmic_flops_per_call": flops, "executed_flops_per_call": 8.0 * hb.T * hb.D * hb.V,
             "reps": reps, "chunks_per_call": chunks,
-            "note": "algorithmic 6 T D V (Z, dH, dW); executed 8 T D V (Z is computed twice); dH and dW through cuBLASLt"}
+            "note": "algorithmic 6 T D V (Z, dH, dW); executed 8 T D V (Z is computed twice); dH and dW through cuBLASLt",
+            "logprobs": fwd}
 
 
 def profile_head(T):
-    """A small fused-head case for profiler captures: three calls on the first T tokens."""
+    """A small fused-head case for profiler captures: three loss calls, then three forward-only
+    log-prob calls, on the first T tokens."""
     import torch
 
     from paper_2608_16798_gb300 import build as B
@@ -531,6 +548,8 @@ def profile_head(T):
     hb = HeadBatch(torch, R, dev, T=T)
     for _ in range(3):
         hb.call(R)
+    for _ in range(3):
+        hb.call_logprobs(R)
     st, word = R.rl_query_status(hb.ws)
     print(json.dumps({"profile_head_tokens": T, "status": word, "flops_per_call": 6.0 * T * hb.D * hb.V}))
     return 0 if word == 0 else 1

@@ -240,6 +240,28 @@ rl_status rl_fused_head_loss_fwd_bwd(const void* hidden, const void* weight, int
                                      size_t ws_bytes, rl_stream_t stream);
 
 /*
+ * Forward-only log-probabilities through the fused LM head (the pi_old / pi_ref
+ * recompute of Sec. 3.2.4 when pi's logits are the LM head's output): for every
+ * token t, with z_t = hidden_t W^T formed tile by tile on the tensor cores and
+ * never written to memory,
+ *   lse_t = log sum_v exp(z_tv), logp_t = z_{t,a_t} - lse_t, H_t = -sum_v p_tv log p_tv.
+ *
+ *   hidden, weight, T, D, V   as for rl_fused_head_loss_fwd_bwd
+ *   token_ids    int32 [T]: a_t (out of range -> logp_t = NaN and RL_DEV_BAD_TOKEN)
+ *   logp_out     float [T]
+ *   entropy_out  float [T] or NULL (entropy work is skipped when NULL)
+ *   lse_out      float [T] or NULL
+ *   ws, ws_bytes workspace; rl_workspace_size(T, V, D) bytes always suffice (the
+ *                call uses the status word and 16 * ceil(V / 4096) * min(T, 8192)
+ *                bytes of per-block softmax partials after it)
+ * One tensor-core pass per chunk of 8,192 tokens, then a per-token merge of the
+ * vocabulary blocks' partials in fixed order (deterministic).
+ */
+rl_status rl_fused_head_token_logprobs(const void* hidden, const void* weight, int64_t T, int64_t D, int64_t V,
+                                       const int32_t* token_ids, float* logp_out, float* entropy_out,
+                                       float* lse_out, void* ws, size_t ws_bytes, rl_stream_t stream);
+
+/*
  * Allocation-free form of rl_policy_loss_fwd_bwd (no counterpart in the paper:
  * it exists for callers that cannot allocate device memory, e.g. code inside a
  * memory pool that forbids cudaMalloc during a training step, or a plugin that

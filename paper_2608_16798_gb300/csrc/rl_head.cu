@@ -364,6 +364,39 @@ __global__ void __launch_bounds__(256) head_merge_kernel(const MergeArgs p) {
   }
 }
 
+struct LogpMergeArgs {
+  int64_t t0;
+  int32_t Tc, V, n_vb;
+  const float4* partials;
+  const int32_t* token_ids;
+  float* logp_out;
+  float* entropy_out;
+  float* lse_out;
+  int32_t* status;
+};
+
+// Forward-only merge: one thread per token of the chunk writes logp, H and lse.
+__global__ void __launch_bounds__(256) head_logp_merge_kernel(const LogpMergeArgs p) {
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= p.Tc) return;
+  const int64_t t = p.t0 + r;
+  SoftmaxPartial q{-__int_as_float(0x7f800000), 0.f, 0.f};
+  float za = 0.f;
+  for (int b = 0; b < p.n_vb; ++b) {
+    const float4 w = p.partials[static_cast<int64_t>(b) * p.Tc + r];
+    q = merge(q, SoftmaxPartial{w.x, w.y, w.z});
+    za += w.w;  // nonzero in the one block that holds the sampled id
+  }
+  const float lnS = logf(q.s);
+  const float lse = q.m + lnS;
+  const int32_t a = p.token_ids[t];
+  const bool a_ok = a >= 0 && a < p.V;
+  if (!a_ok) flag_status(p.status, RL_DEV_BAD_TOKEN);
+  p.logp_out[t] = a_ok ? za - lse : __int_as_float(0x7fc00000);
+  if (p.entropy_out) p.entropy_out[t] = lnS - q.u / q.s;
+  if (p.lse_out) p.lse_out[t] = lse;
+}
+
 // ------------------------------------------------------------------ host side
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -407,13 +440,15 @@ struct Layout {
   size_t off_partials, off_rc, off_dz, off_lt, total;
 };
 
+static size_t al256(size_t x) { return (x + 255) & ~size_t(255); }
+
 static Layout layout(int64_t max_rows, int64_t V) {
   Layout L;
   L.Tc = std::max<int64_t>(1, std::min<int64_t>(max_rows, kChunk));
   const int64_t n_nt = (V + BN - 1) / BN;
   L.n_vb = (n_nt + VB_TILES - 1) / VB_TILES;
   L.ldz = (V + 7) / 8 * 8;
-  auto al = [](size_t x) { return (x + 255) & ~size_t(255); };
+  auto al = al256;
   size_t off = kWsHeader + al(static_cast<size_t>(std::max<int64_t>(max_rows, 0)) * sizeof(double));
   L.off_partials = off;
   off += al(static_cast<size_t>(L.n_vb * L.Tc) * sizeof(float4));
@@ -507,6 +542,13 @@ static rl_status launch_head(const CUtensorMap& mh, const CUtensorMap& mw, const
 size_t head_workspace_bytes(int64_t max_rows, int64_t V, int64_t D) {
   (void)D;
   return head::layout(max_rows, V).total;
+}
+
+// The forward-only call needs the status word and one chunk's partials, which sit at the
+// same offset as in the loss layout's header; rl_workspace_size(T, V, D) always suffices.
+static size_t head_logp_workspace_bytes(int64_t T, int64_t V) {
+  const head::Layout L = head::layout(T, V);
+  return kWsHeader + head::al256(static_cast<size_t>(L.n_vb * L.Tc) * sizeof(float4));
 }
 
 }  // namespace rl
@@ -625,4 +667,71 @@ extern "C" rl_status rl_fused_head_loss_fwd_bwd(
     if (st != RL_OK) return st;
   }
   return launch_reduce_loss(row_loss, T, loss_accum, s);
+}
+
+extern "C" rl_status rl_fused_head_token_logprobs(const void* hidden, const void* weight, int64_t T, int64_t D,
+                                                  int64_t V, const int32_t* token_ids, float* logp_out,
+                                                  float* entropy_out, float* lse_out, void* ws, size_t ws_bytes,
+                                                  rl_stream_t stream) {
+  using namespace rl;
+  using namespace rl::head;
+  clear_error();
+  if (T < 0 || D < 64 || V < 1)
+    return set_error(RL_ERR_INVALID_ARG, "rl_fused_head_token_logprobs: need T >= 0, D >= 64, V >= 1");
+  if (D % 64 != 0) return set_error(RL_ERR_UNSUPPORTED, "rl_fused_head_token_logprobs: D must be a multiple of 64");
+  if (T > INT32_MAX || V > INT32_MAX || D > 65536)
+    return set_error(RL_ERR_UNSUPPORTED, "rl_fused_head_token_logprobs: T or V above 2^31 - 1, or D above 65536");
+  if (!ws) return set_error(RL_ERR_INVALID_ARG, "rl_fused_head_token_logprobs: NULL workspace");
+  if (ws_bytes < head_logp_workspace_bytes(T, V))
+    return set_error(RL_ERR_WORKSPACE_TOO_SMALL, "rl_fused_head_token_logprobs: workspace too small");
+  if (T == 0) return RL_OK;
+  if (!hidden || !weight || !token_ids || !logp_out)
+    return set_error(RL_ERR_INVALID_ARG, "rl_fused_head_token_logprobs: NULL array argument");
+  if (!aligned16(hidden) || !aligned16(weight) || !aligned16(ws))
+    return set_error(RL_ERR_ALIGNMENT, "rl_fused_head_token_logprobs: hidden, weight and ws must be 16-byte aligned");
+
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const Layout L = layout(T, V);
+  char* wsb = static_cast<char*>(ws);
+  int32_t* status = reinterpret_cast<int32_t*>(wsb);
+  float4* partials = reinterpret_cast<float4*>(wsb + kWsHeader);
+  CUtensorMap mw;
+  rl_status st = make_map(&mw, weight, D, V, BN);
+  if (st != RL_OK) return st;
+  const int n_nt = static_cast<int>((V + BN - 1) / BN);
+  for (int64_t t0 = 0; t0 < T; t0 += L.Tc) {
+    const int Tc = static_cast<int>(std::min<int64_t>(L.Tc, T - t0));
+    CUtensorMap mh;
+    st = make_map(&mh, static_cast<const uint16_t*>(hidden) + t0 * D, D, Tc, BM);
+    if (st != RL_OK) return st;
+    HeadArgs ha = {};
+    ha.t0 = t0;
+    ha.Tc = Tc;
+    ha.D = static_cast<int>(D);
+    ha.V = static_cast<int>(V);
+    ha.n_mt = (Tc + BM - 1) / BM;
+    ha.n_nt = n_nt;
+    ha.n_vb = static_cast<int>(L.n_vb);
+    ha.ent = entropy_out ? 1 : 0;
+    ha.token_ids = token_ids;
+    ha.partials = partials;
+    ha.status = status;
+    st = launch_head<STATS>(mh, mw, ha, s);
+    if (st != RL_OK) return st;
+    LogpMergeArgs ma = {};
+    ma.t0 = t0;
+    ma.Tc = Tc;
+    ma.V = static_cast<int>(V);
+    ma.n_vb = ha.n_vb;
+    ma.partials = partials;
+    ma.token_ids = token_ids;
+    ma.logp_out = logp_out;
+    ma.entropy_out = entropy_out;
+    ma.lse_out = lse_out;
+    ma.status = status;
+    head_logp_merge_kernel<<<(Tc + 255) / 256, 256, 0, s>>>(ma);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_error(e, "head_logp_merge_kernel launch");
+  }
+  return RL_OK;
 }

@@ -40,6 +40,7 @@ EXPORTS = {
                                       _P, _P, _P, _P, _SZ, _P]),
     "rl_policy_loss_fwd_bwd_noalloc": (_I32, [_P, _I32, _I64, _I64, _I64, _P, _P, _P, _I32, _P, _P, _P, _P, _P,
                                               _P, _P, _P, _P, _P, _P]),
+    "rl_fused_head_token_logprobs": (_I32, [_P, _P, _I64, _I64, _I64, _P, _P, _P, _P, _P, _SZ, _P]),
     "rl_fused_head_loss_fwd_bwd": (_I32, [_P, _P, _I64, _I64, _I64, _P, _P, _P, _I32, _P, _P, _P, _P, _P, _P, _P,
                                           _I32, _P, _P, _P, _P, _SZ, _P]),
 }
@@ -326,3 +327,30 @@ def rl_fused_head_loss_fwd_bwd(hidden, weight, token_ids, mask, token_traj, adv,
                                           ws.numel(), _stream(stream))
     _check("rl_fused_head_loss_fwd_bwd", st)
     return d_hidden
+
+
+def rl_fused_head_token_logprobs(hidden, weight, token_ids, ws, logp_out=None, entropy_out=None, lse_out=None,
+                                 want_entropy=False, want_lse=False, stream=None):
+    """logp of the sampled ids (and optionally entropy, lse) under logits hidden @ weight^T,
+    without materialising the logits."""
+    if hidden.dim() != 2 or weight.dim() != 2 or hidden.shape[1] != weight.shape[1]:
+        raise ValueError("hidden [T, D] and weight [V, D] must share D")
+    T, D = hidden.shape
+    V = weight.shape[0]
+    dev = hidden.device
+    _need(hidden, "hidden", torch.bfloat16, device=dev)
+    _need(weight, "weight", torch.bfloat16, device=dev)
+    _need(token_ids, "token_ids", torch.int32, T, device=dev)
+    logp_out = torch.empty(T, dtype=torch.float32, device=dev) if logp_out is None else logp_out
+    if want_entropy and entropy_out is None:
+        entropy_out = torch.empty(T, dtype=torch.float32, device=dev)
+    if want_lse and lse_out is None:
+        lse_out = torch.empty(T, dtype=torch.float32, device=dev)
+    _need(logp_out, "logp_out", torch.float32, T, device=dev)
+    _opt(entropy_out, "entropy_out", torch.float32, T, device=dev)
+    _opt(lse_out, "lse_out", torch.float32, T, device=dev)
+    _need(ws, "ws", torch.uint8, device=dev)
+    st = lib().rl_fused_head_token_logprobs(_ptr(hidden), _ptr(weight), T, D, V, _ptr(token_ids), _ptr(logp_out),
+                                            _ptr(entropy_out), _ptr(lse_out), _ptr(ws), ws.numel(), _stream(stream))
+    _check("rl_fused_head_token_logprobs", st)
+    return logp_out, entropy_out, lse_out

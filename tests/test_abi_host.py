@@ -140,3 +140,31 @@ def test_status_and_init_argument_checks(R):
     assert L.rl_workspace_init(FAKE, 16, None) == 4
     word = ctypes.c_int32(0)
     assert L.rl_query_status(None, None, ctypes.byref(word)) == 1
+
+
+def test_fused_head_logprobs_argument_checks(R):
+    L = R.lib()
+
+    def call(**over):
+        a = dict(h=FAKE, w=FAKE, T=4, D=128, V=1000, ids=FAKE, logp=FAKE, ent=None, lse=None, ws=FAKE,
+                 ws_bytes=1 << 20, stream=None)
+        a.update(over)
+        return L.rl_fused_head_token_logprobs(a["h"], a["w"], a["T"], a["D"], a["V"], a["ids"], a["logp"], a["ent"],
+                                              a["lse"], a["ws"], a["ws_bytes"], a["stream"])
+
+    assert call(T=-1) == 1
+    assert call(D=32) == 1
+    assert call(D=96) == 2
+    assert call(V=0) == 1
+    assert call(ws=None) == 1
+    assert call(ws_bytes=300) == 4
+    assert call(logp=None) == 1
+    assert call(h=FAKE + 2) == 3
+    assert call(ws=FAKE + 8) == 3
+    assert call(T=0) == 0
+    # rl_workspace_size(T, V, D) always suffices; one chunk of partials is the minimum
+    # (logp=None makes a call that passed the workspace check stop at the next one)
+    big = dict(T=20000, V=151936, logp=None)
+    assert call(ws_bytes=R.rl_workspace_size(20000, 151936, 4096), **big) == 1
+    assert call(ws_bytes=256 + 16 * 38 * 8192, **big) == 1
+    assert call(ws_bytes=256 + 16 * 38 * 8192 - 1, **big) == 4

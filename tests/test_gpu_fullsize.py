@@ -163,6 +163,15 @@ def test_fused_head_full_size(R):
     old = W.old_logp_from(logp, w, seed)
 
     ws = R.new_workspace(T, V, D)
+    # forward-only log-probs (the old / reference policy recompute) on every token
+    zerr = logit_error_bound(Hm, Wm)
+    f_logp, f_H, f_lse = R.rl_fused_head_token_logprobs(hidden, weight, ids_d, ws, want_entropy=True, want_lse=True)
+    assert R.rl_query_status(ws)[1] == 0
+    f_logp, f_H, f_lse = (x.cpu().numpy().astype(np.float64) for x in (f_logp, f_H, f_lse))
+    assert np.all(np.abs(f_logp - logp) <= 1e-5 + 2.0 ** -22 * np.abs(logp) + zerr), np.abs(f_logp - logp).max()
+    assert np.all(np.abs(f_lse - lse) <= 1e-5 + 2.0 ** -22 * np.abs(lse) + zerr), np.abs(f_lse - lse).max()
+    assert np.all(np.abs(f_H - H) <= 5e-5 + 2e-5 * np.abs(H) + 2 * zerr), np.abs(f_H - H).max()
+
     loss = torch.zeros(1, dtype=torch.float64, device="cuda")
     st = torch.zeros(T * 5, dtype=torch.float32, device="cuda")
     dW = torch.zeros((V, D), dtype=torch.float32, device="cuda")

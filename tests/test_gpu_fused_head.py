@@ -145,3 +145,70 @@ def test_fused_head_matches_logits_path(R):
                              to_dev(c["adv32"]), to_dev(c["coef32"]), to_dev(c["old"]), cuda_params(R, c["P"]), ws,
                              loss)
     assert abs(loss.item() - out["loss"]) <= 1e-4 * max(abs(loss.item()), 1e-12)
+
+
+def check_logprobs(c, logp, H, lse, what):
+    """Forward-only outputs against the oracle, with the logit allowance zerr per token."""
+    ref_logp, ref_H, ref_lse = O.fused_head_logprobs(c["h"], c["w"], c["ids"])
+    zerr = logit_error_bound(O.decode_logits(c["h"], "bf16"), O.decode_logits(c["w"], "bf16"))
+    d = np.abs(logp - ref_logp)
+    assert np.all(d <= 1e-5 + 2.0 ** -22 * np.abs(ref_logp) + zerr), f"{what}: logp max diff {d.max()}"
+    d = np.abs(lse - ref_lse)
+    assert np.all(d <= 1e-5 + 2.0 ** -22 * np.abs(ref_lse) + zerr), f"{what}: lse max diff {d.max()}"
+    if H is not None:
+        d = np.abs(H - ref_H)
+        assert np.all(d <= 5e-5 + 2e-5 * np.abs(ref_H) + 2 * zerr), f"{what}: entropy max diff {d.max()}"
+
+
+def run_logprobs(R, c, want_entropy=True, ids=None):
+    T, V, D = c["T"], c["V"], c["D"]
+    ws = R.new_workspace(T, V, D)
+    logp, H, lse = R.rl_fused_head_token_logprobs(_bf16_dev(c["h"]), _bf16_dev(c["w"]),
+                                                  to_dev(c["ids"] if ids is None else ids), ws,
+                                                  want_entropy=want_entropy, want_lse=True)
+    word = R.rl_query_status(ws)[1]
+    f = lambda x: None if x is None else x.cpu().numpy().astype(np.float64)
+    return f(logp), f(H), f(lse), word
+
+
+@pytest.mark.parametrize("T,D,V", [
+    (300, 256, 1000),        # ragged M tile and vocabulary tile
+    (256, 128, 8292),        # three vocabulary blocks, ragged last block
+    (130, 64, 513),          # smallest D
+    (8192 + 77, 128, 1100),  # two chunks
+])
+def test_fused_head_logprobs_parity(R, T, D, V):
+    c = make_head_case(T, D, V, seed=3 * T + V)
+    logp, H, lse, word = run_logprobs(R, c)
+    assert word == 0
+    check_logprobs(c, logp, H, lse, f"fused logprobs {T}x{D}x{V}")
+
+
+def test_fused_head_logprobs_without_entropy_and_bad_ids(R):
+    """entropy_out NULL skips the entropy work and leaves logp and lse unchanged (bit for bit);
+    an id outside [0, V) gives NaN for its token only and sets RL_DEV_BAD_TOKEN."""
+    c = make_head_case(260, 128, 900, seed=4)
+    logp_e, _, lse_e, _ = run_logprobs(R, c, want_entropy=True)
+    logp, H, lse, word = run_logprobs(R, c, want_entropy=False)
+    assert H is None and word == 0
+    assert np.array_equal(logp, logp_e) and np.array_equal(lse, lse_e)
+    bad = c["ids"].copy()
+    bad[[5, 200]] = [-1, 900]
+    logp_b, _, lse_b, word = run_logprobs(R, c, ids=bad)
+    assert word == R.RL_DEV_BAD_TOKEN
+    assert np.isnan(logp_b[[5, 200]]).all()
+    keep = np.ones(260, bool)
+    keep[[5, 200]] = False
+    assert np.array_equal(logp_b[keep], logp[keep]) and np.array_equal(lse_b, lse)
+
+
+def test_fused_head_logprobs_match_loss_pass(R):
+    """The forward-only call and the loss call's first pass form the same statistics: logp and
+    entropy agree bit for bit with token_stats of rl_fused_head_loss_fwd_bwd on trained tokens."""
+    c = make_head_case(384, 192, 3000, seed=11, masked=0.3, ent=True)
+    out = run_head(R, c)
+    logp, H, _, word = run_logprobs(R, c)
+    active = (c["mask"] != 0) & (c["coef32"][c["tt"]] != 0)
+    st = out["stats"].astype(np.float64)
+    assert np.array_equal(st[active, 0], logp[active])
+    assert np.array_equal(st[active, 3], H[active])
