@@ -81,6 +81,7 @@ class LossParams:
     tis_cap: float = 0.0           # c-bar of the TIS weight; <= 0 disables it
     adv_eps: float = 1e-6          # epsilon of the advantage denominator
     loss_agg: int = AGG_SEQ_MEAN_TOKEN_MEAN
+    token_level_adv: bool = False  # adv holds one A_t per row (PPO, Sec. 2.3.1), not one per trajectory
 
 
 # ----------------------------------------------------------------------------
@@ -279,7 +280,8 @@ def policy_loss_fwd_bwd(logits, dtype, token_ids, mask, token_traj, adv, coef, o
     """Loss = sum_t c_{i(t)} M_t l_t over the rows of one microbatch and dLoss/dz.
 
     logits: [n_rows, V] bf16 bit patterns (uint16) or float32. token_traj maps each
-    row to its trajectory; adv and coef are per-trajectory. Returns
+    row to its trajectory; adv and coef are per-trajectory (with params.token_level_adv,
+    adv holds one A_t per row, as in the PPO objective of Sec. 2.3.1). Returns
     (loss, grad float64 [n_rows, V] or None, stats float64 [n_rows, 5], contrib)
     where contrib[t] = c M l_t and stats hold (logp, rho, clipped, H, KL) for active
     rows (M_t = 1 and c != 0) and zeros elsewhere.  If ``rows`` is given, only
@@ -297,7 +299,7 @@ def policy_loss_fwd_bwd(logits, dtype, token_ids, mask, token_traj, adv, coef, o
     stats = np.zeros((len(sel), 5), dtype=np.float64)
     contrib = np.zeros(len(sel), dtype=np.float64)
     c_row = coef[token_traj[sel]]
-    A_row = adv[token_traj[sel]]
+    A_row = adv[sel] if params.token_level_adv else adv[token_traj[sel]]
     active = (mask[sel] != 0) & (c_row != 0.0)
     idx_active = np.nonzero(active)[0]
     alpha = params.entropy_coef

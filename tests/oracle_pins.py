@@ -386,6 +386,33 @@ def pin_loss_ratio_one(O):
         _close(stats[act, 1], np.ones(act.sum()), rtol=1e-12, what="rho = 1")
 
 
+def pin_token_level_advantages(O):
+    """Per-token advantages (PPO, Sec. 2.3.1): rho = 1 and no other term gives
+    loss = -sum_t c M A_t and surrogate rows -c A_t (onehot_a - p); advantages broadcast
+    from the trajectories reproduce the per-trajectory call exactly."""
+    pr = _tiny_problem(13, n_traj=5, agg=1)
+    T = pr["z"].shape[0]
+    A_t = np.random.default_rng(14).normal(0, 1, size=T)
+    z = pr["z"]
+    zmax = z.max(axis=1)
+    lse = zmax + np.log(np.exp(z - zmax[:, None]).sum(axis=1))
+    logp = z[np.arange(T), pr["a"]] - lse
+    P = O.LossParams(loss_agg=1, token_level_adv=True)
+    loss, grad, _, _ = O.policy_loss_fwd_bwd(z, "f64", pr["a"], pr["mask"], pr["tt"], A_t, pr["coef"], logp, P)
+    c_t = pr["coef"][pr["tt"]] * (pr["mask"] != 0)
+    _close(loss, -(c_t * A_t).sum(), rtol=1e-12, atol=1e-14, what="token-level loss at rho = 1")
+    p = np.exp(z - lse[:, None])
+    onehot = np.zeros_like(p)
+    onehot[np.arange(T), pr["a"]] = 1.0
+    _close(grad, -(c_t * A_t)[:, None] * (onehot - p), rtol=1e-12, atol=1e-14, what="token-level rows")
+    P0 = O.LossParams(**pr["P"])
+    P1 = O.LossParams(**pr["P"], token_level_adv=True)
+    l0, g0, _, _ = _loss(O, pr, z, P0)
+    l1, g1, _, _ = O.policy_loss_fwd_bwd(z, "f64", pr["a"], pr["mask"], pr["tt"], pr["adv"][pr["tt"]], pr["coef"],
+                                         pr["old"], P1, pr["ref"], pr["roll"])
+    assert l0 == l1 and np.array_equal(g0, g1)
+
+
 def pin_loss_additive_and_permutation(O):
     """The loss of two microbatches adds up to the loss of the whole batch; permuting the
     rows permutes the gradient rows and keeps the loss."""

@@ -57,6 +57,8 @@ MUTANTS = {
     "head dW transposed": ("d_weight = dZ.T @ Hm", "d_weight = (dZ.T @ Hm).T"),
     "head dH uses W^T": ("d_hidden = dZ @ Wm", "d_hidden = dZ @ Wm.T"),
     "head logits transposed": ("Z = Hm @ Wm.T", "Z = (Hm @ Wm.T).T"),
+    "token-level adv ignored": ("A_row = adv[sel] if params.token_level_adv else adv[token_traj[sel]]",
+                                "A_row = adv[token_traj[sel]]"),
     "head logprobs chunk offset": ("Z = Hm[r0:r0 + chunk] @ Wm.T", "Z = Hm[r0 + 1:r0 + 1 + chunk] @ Wm.T"),
 }
 
