@@ -85,6 +85,9 @@ typedef struct rl_loss_params {
   float tis_cap;       /* c-bar; <= 0 or rollout_logp == NULL disables the TIS weight */
   float adv_eps;       /* epsilon added to sigma in the advantage denominator */
   int32_t loss_agg;    /* rl_loss_agg */
+  int32_t token_level_adv; /* 0: adv is float [n_traj], A_{i(t)} per trajectory (GRPO, Sec. 2.3.2);
+                              1: adv is float [rows], one A_t per row, e.g. from rl_masked_gae
+                              (PPO, Sec. 2.3.1); coef stays per trajectory */
 } rl_loss_params;
 
 /* Library version, major * 10000 + minor * 100 + patch. */
@@ -238,6 +241,60 @@ rl_status rl_fused_head_loss_fwd_bwd(const void* hidden, const void* weight, int
                                      const rl_loss_params* params, void* d_hidden, rl_dtype d_hidden_dtype,
                                      float* d_weight, double* loss_accum, float* token_stats, void* ws,
                                      size_t ws_bytes, rl_stream_t stream);
+
+/*
+ * Masked generalised advantage estimation for PPO (Sec. 2.3.1, masked GAE and TD
+ * residual; Sec. 2.3.4, PPO with each trajectory backed up on its own), per
+ * trajectory of the packed stream:
+ *   printed reading (skip_masked = 0):
+ *     A_t = sum_l (gamma lambda)^l delta_{t+l} M_{t+l},
+ *     delta_t = r_t + gamma V_{t+1} M_{t+1} - V_t   (V past the trajectory's end = 0);
+ *   skip reading (skip_masked = 1): the same recursion over the trajectory's
+ *     trainable tokens only (masked tokens are stepped over, their rewards ignored,
+ *     delta_t bootstraps from the next trainable token's value). With gamma =
+ *     lambda = 1 and the reward at the final trainable token it gives
+ *     A_t = R_i - V_t, the form Sec. 2.3.4 states; the printed reading does not
+ *     when the mask has gaps. Without masked tokens the two agree.
+ *   returns G_t = A_t + V_t (the targets of the value loss).
+ *
+ *   n_traj, traj_offsets  int64 [n_traj + 1]: trajectory i owns tokens
+ *                         [traj_offsets[i], traj_offsets[i+1]) (non-decreasing, in [0, n_tokens];
+ *                         else RL_DEV_BAD_OFFSETS and that trajectory is skipped)
+ *   mask                  uint8 [n_tokens]: M_t
+ *   values                float [n_tokens]: V(s_t) of the value model that scored the rollout
+ *   token_rewards         float [n_tokens] or NULL: r_t
+ *   traj_rewards          float [n_traj] or NULL: R_i, added to r_t at trajectory i's last
+ *                         token with M_t = 1 (none if it has no such token)
+ *   gamma, gae_lambda     in [0, 1]
+ *   adv_out               float [n_tokens]: A_t, 0 at masked tokens
+ *   returns_out           float [n_tokens] or NULL: G_t, 0 at masked tokens
+ *   ws, ws_bytes          workspace (rl_workspace_size(0, 0, 0) bytes suffice)
+ * Tokens outside every trajectory's span are not written. fp32 arithmetic: one CTA per
+ * trajectory runs a block-wide suffix scan of the recursion's affine maps.
+ */
+rl_status rl_masked_gae(int32_t n_traj, const int64_t* traj_offsets, int64_t n_tokens, const uint8_t* mask,
+                        const float* values, const float* token_rewards, const float* traj_rewards, float gamma,
+                        float gae_lambda, int32_t skip_masked, float* adv_out, float* returns_out, void* ws,
+                        size_t ws_bytes, rl_stream_t stream);
+
+/*
+ * Masked value loss of PPO (Sec. 2.3.1, masked mean-squared critic loss) over one
+ * microbatch of rows:
+ *   loss += sum_t c_{i(t)} M_t (V_t - G_t)^2,   d_values_t = 2 c_{i(t)} M_t (V_t - G_t).
+ * With coef from rl_group_advantages under RL_AGG_TOKEN_MEAN this is the token mean
+ * E_t of the paper. Rows with M_t = 0 or c = 0 get d_values_t = 0.
+ *
+ *   values, returns   float [rows]: V_t of the current value model, G_t (from rl_masked_gae)
+ *   mask, token_traj  uint8 [rows], int32 [rows] (token_traj outside [0, n_traj) on a row
+ *                     with M_t != 0 sets RL_DEV_BAD_TRAJ and the row contributes nothing)
+ *   coef              float [n_traj]
+ *   d_values          float [rows]
+ *   loss_accum        double [1] on the device, added to (fixed-order reduction)
+ *   ws, ws_bytes      workspace of at least rl_workspace_size(rows, 0, 0) bytes
+ */
+rl_status rl_value_loss_fwd_bwd(int64_t rows, const float* values, const float* returns, const uint8_t* mask,
+                                const int32_t* token_traj, int32_t n_traj, const float* coef, float* d_values,
+                                double* loss_accum, void* ws, size_t ws_bytes, rl_stream_t stream);
 
 /*
  * Forward-only log-probabilities through the fused LM head (the pi_old / pi_ref

@@ -285,6 +285,7 @@ struct MergeArgs {
   const float* ref_logp;
   const float* rollout_logp;
   float clip_lo, clip_hi, beta, alpha, tis_cap;
+  int32_t adv_per_row;  // adv holds one A_t per token (else one per trajectory)
   RowCoef* rc;
   double* row_loss;
   float* token_stats;
@@ -332,7 +333,7 @@ __global__ void __launch_bounds__(256) head_merge_kernel(const MergeArgs p) {
   const float lnS = logf(q.s);
   const float lse = q.m + lnS;
   const float H = lnS - q.u / q.s;
-  const float A = p.adv[i], c = p.coef[i], old = p.old_logp[t];
+  const float A = p.adv_per_row ? p.adv[t] : p.adv[i], c = p.coef[i], old = p.old_logp[t];
   const float logp = za - lse;
   const float rho = expf((za - old) - lse);
   const float crho = fminf(fmaxf(rho, p.clip_lo), p.clip_hi);
@@ -572,12 +573,14 @@ extern "C" rl_status rl_fused_head_loss_fwd_bwd(
     return set_error(RL_ERR_INVALID_ARG, "rl_fused_head_loss_fwd_bwd: unknown d_hidden dtype");
   if (params->kl_estimator != 0 && params->kl_estimator != 3)
     return set_error(RL_ERR_UNSUPPORTED, "rl_fused_head_loss_fwd_bwd: kl_estimator must be 0 or 3");
+  if (params->token_level_adv != 0 && params->token_level_adv != 1)
+    return set_error(RL_ERR_INVALID_ARG, "rl_fused_head_loss_fwd_bwd: token_level_adv must be 0 or 1");
   if (ws_bytes < rl_workspace_size(T, V, D))
     return set_error(RL_ERR_WORKSPACE_TOO_SMALL,
                      "rl_fused_head_loss_fwd_bwd: workspace smaller than rl_workspace_size(T, V, D)");
   if (T == 0) return RL_OK;
   if (!hidden || !weight || !token_ids || !mask || !token_traj || !old_logp || !d_hidden || !d_weight ||
-      (n_traj > 0 && (!adv || !coef)))
+      (n_traj > 0 && (!adv || !coef)) || (params->token_level_adv && !adv))
     return set_error(RL_ERR_INVALID_ARG, "rl_fused_head_loss_fwd_bwd: NULL array argument");
   if (!aligned16(hidden) || !aligned16(weight) || !aligned16(d_hidden) || !aligned16(d_weight) || !aligned16(ws))
     return set_error(RL_ERR_ALIGNMENT,
@@ -646,6 +649,7 @@ extern "C" rl_status rl_fused_head_loss_fwd_bwd(
     ma.beta = kl_on ? params->kl_coef : 0.f;
     ma.alpha = params->entropy_coef;
     ma.tis_cap = rollout_logp ? params->tis_cap : 0.f;
+    ma.adv_per_row = params->token_level_adv;
     ma.rc = rcs;
     ma.row_loss = row_loss;
     ma.token_stats = token_stats;

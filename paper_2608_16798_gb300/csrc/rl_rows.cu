@@ -52,6 +52,7 @@ struct RowArgs {
   float beta;              // 0 when the KL term is off
   float alpha;             // entropy bonus
   float tis_cap;           // <= 0 when TIS is off
+  int32_t adv_per_row;     // adv holds one A_t per row (else one per trajectory)
   double* row_loss;
   float* token_stats;
   float* logp_out;
@@ -380,7 +381,7 @@ __global__ void __launch_bounds__((NW + 1) * 32, 2) rows_kernel(const RowArgs p)
             active = false;
           } else {
             m.c = p.coef[i];
-            m.A = p.adv[i];
+            m.A = p.adv_per_row ? p.adv[r] : p.adv[i];
             active = m.c != 0.f;
             if (active && (m.a < 0 || m.a >= V)) {
               if (rank == 0 && lane == 0) flag_status(p.status, RL_DEV_BAD_TOKEN);
@@ -1075,8 +1076,11 @@ extern "C" rl_status rl_policy_loss_fwd_bwd(const void* logits, rl_dtype dtype, 
   if (!loss_accum) return set_error(RL_ERR_INVALID_ARG, "rl_policy_loss_fwd_bwd: loss_accum is NULL");
   if (n_traj < 0) return set_error(RL_ERR_INVALID_ARG, "rl_policy_loss_fwd_bwd: n_traj < 0");
   if (rows == 0) return RL_OK;
-  if (!token_ids || !mask || !token_traj || !old_logp || !grad_out || (n_traj > 0 && (!adv || !coef)))
+  if (!token_ids || !mask || !token_traj || !old_logp || !grad_out || (n_traj > 0 && (!adv || !coef)) ||
+      (params->token_level_adv && !adv))
     return set_error(RL_ERR_INVALID_ARG, "rl_policy_loss_fwd_bwd: NULL array argument");
+  if (params->token_level_adv != 0 && params->token_level_adv != 1)
+    return set_error(RL_ERR_INVALID_ARG, "rl_policy_loss_fwd_bwd: token_level_adv must be 0 or 1");
   if (!aligned16(grad_out)) return set_error(RL_ERR_ALIGNMENT, "rl_policy_loss_fwd_bwd: grad_out not 16-byte aligned");
   const bool kl_on = params->kl_estimator == 3 && params->kl_coef != 0.f && ref_logp != nullptr;
   RowArgs a = {};
@@ -1099,6 +1103,7 @@ extern "C" rl_status rl_policy_loss_fwd_bwd(const void* logits, rl_dtype dtype, 
   a.beta = kl_on ? params->kl_coef : 0.f;
   a.alpha = params->entropy_coef;
   a.tis_cap = rollout_logp ? params->tis_cap : 0.f;
+  a.adv_per_row = params->token_level_adv;
   double* row_loss = reinterpret_cast<double*>(static_cast<char*>(ws) + ws_row_loss_offset());
   a.row_loss = row_loss;
   a.token_stats = token_stats;

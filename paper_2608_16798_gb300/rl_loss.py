@@ -40,6 +40,8 @@ EXPORTS = {
                                       _P, _P, _P, _P, _SZ, _P]),
     "rl_policy_loss_fwd_bwd_noalloc": (_I32, [_P, _I32, _I64, _I64, _I64, _P, _P, _P, _I32, _P, _P, _P, _P, _P,
                                               _P, _P, _P, _P, _P, _P]),
+    "rl_masked_gae": (_I32, [_I32, _P, _I64, _P, _P, _P, _P, _F, _F, _I32, _P, _P, _P, _SZ, _P]),
+    "rl_value_loss_fwd_bwd": (_I32, [_I64, _P, _P, _P, _P, _I32, _P, _P, _P, _P, _SZ, _P]),
     "rl_fused_head_token_logprobs": (_I32, [_P, _P, _I64, _I64, _I64, _P, _P, _P, _P, _P, _SZ, _P]),
     "rl_fused_head_loss_fwd_bwd": (_I32, [_P, _P, _I64, _I64, _I64, _P, _P, _P, _I32, _P, _P, _P, _P, _P, _P, _P,
                                           _I32, _P, _P, _P, _P, _SZ, _P]),
@@ -48,13 +50,14 @@ EXPORTS = {
 
 class rl_loss_params(ctypes.Structure):
     _fields_ = [("clip_eps_low", _F), ("clip_eps_high", _F), ("kl_coef", _F), ("kl_estimator", _I32),
-                ("entropy_coef", _F), ("tis_cap", _F), ("adv_eps", _F), ("loss_agg", _I32)]
+                ("entropy_coef", _F), ("tis_cap", _F), ("adv_eps", _F), ("loss_agg", _I32),
+                ("token_level_adv", _I32)]
 
 
 def make_params(clip_eps_low=0.2, clip_eps_high=0.28, kl_coef=0.0, kl_estimator=0, entropy_coef=0.0,
-                tis_cap=0.0, adv_eps=1e-6, loss_agg=AGG_SEQ_MEAN_TOKEN_MEAN) -> rl_loss_params:
+                tis_cap=0.0, adv_eps=1e-6, loss_agg=AGG_SEQ_MEAN_TOKEN_MEAN, token_level_adv=0) -> rl_loss_params:
     return rl_loss_params(clip_eps_low, clip_eps_high, kl_coef, kl_estimator, entropy_coef, tis_cap, adv_eps,
-                          loss_agg)
+                          loss_agg, int(token_level_adv))
 
 
 class RLError(RuntimeError):
@@ -231,12 +234,12 @@ def rl_policy_loss_fwd_bwd(logits, token_ids, mask, token_traj, adv, coef, old_l
     rows, V, ld = _rows_view(logits)
     dt = _logits_dtype(logits)
     dev = logits.device
-    n_traj = adv.numel()
+    n_traj = coef.numel()
     _need(token_ids, "token_ids", torch.int32, rows, device=dev)
     _need(mask, "mask", torch.uint8, rows, device=dev)
     _need(token_traj, "token_traj", torch.int32, rows, device=dev)
-    _need(adv, "adv", torch.float32, device=dev)
     _need(coef, "coef", torch.float32, n_traj, device=dev)
+    _need(adv, "adv", torch.float32, rows if params.token_level_adv else n_traj, device=dev)
     _need(old_logp, "old_logp", torch.float32, rows, device=dev)
     _opt(ref_logp, "ref_logp", torch.float32, rows, device=dev)
     _opt(rollout_logp, "rollout_logp", torch.float32, rows, device=dev)
@@ -266,12 +269,12 @@ def rl_policy_loss_fwd_bwd_noalloc(logits, token_ids, mask, token_traj, adv, coe
     rows, V, ld = _rows_view(logits)
     dt = _logits_dtype(logits)
     dev = logits.device
-    n_traj = adv.numel()
+    n_traj = coef.numel()
     _need(token_ids, "token_ids", torch.int32, rows, device=dev)
     _need(mask, "mask", torch.uint8, rows, device=dev)
     _need(token_traj, "token_traj", torch.int32, rows, device=dev)
-    _need(adv, "adv", torch.float32, device=dev)
     _need(coef, "coef", torch.float32, n_traj, device=dev)
+    _need(adv, "adv", torch.float32, rows if params.token_level_adv else n_traj, device=dev)
     _need(old_logp, "old_logp", torch.float32, rows, device=dev)
     _opt(ref_logp, "ref_logp", torch.float32, rows, device=dev)
     _opt(rollout_logp, "rollout_logp", torch.float32, rows, device=dev)
@@ -301,14 +304,14 @@ def rl_fused_head_loss_fwd_bwd(hidden, weight, token_ids, mask, token_traj, adv,
     T, D = hidden.shape
     V = weight.shape[0]
     dev = hidden.device
-    n_traj = adv.numel()
+    n_traj = coef.numel()
     _need(hidden, "hidden", torch.bfloat16, device=dev)
     _need(weight, "weight", torch.bfloat16, device=dev)
     _need(token_ids, "token_ids", torch.int32, T, device=dev)
     _need(mask, "mask", torch.uint8, T, device=dev)
     _need(token_traj, "token_traj", torch.int32, T, device=dev)
-    _need(adv, "adv", torch.float32, device=dev)
     _need(coef, "coef", torch.float32, n_traj, device=dev)
+    _need(adv, "adv", torch.float32, T if params.token_level_adv else n_traj, device=dev)
     _need(old_logp, "old_logp", torch.float32, T, device=dev)
     _opt(ref_logp, "ref_logp", torch.float32, T, device=dev)
     _opt(rollout_logp, "rollout_logp", torch.float32, T, device=dev)
@@ -354,3 +357,49 @@ def rl_fused_head_token_logprobs(hidden, weight, token_ids, ws, logp_out=None, e
                                             _ptr(entropy_out), _ptr(lse_out), _ptr(ws), ws.numel(), _stream(stream))
     _check("rl_fused_head_token_logprobs", st)
     return logp_out, entropy_out, lse_out
+
+
+def rl_masked_gae(traj_offsets, mask, values, ws, gamma=1.0, gae_lambda=1.0, skip_masked=True, token_rewards=None,
+                  traj_rewards=None, adv_out=None, returns_out=None, want_returns=True, stream=None):
+    """Masked GAE per trajectory (Sec. 2.3.1): returns (adv, returns) float32 [T], zero at masked tokens.
+    traj_rewards [n] places R_i at trajectory i's last trainable token (Sec. 2.3.4)."""
+    n_traj = traj_offsets.numel() - 1
+    T = mask.numel()
+    dev = mask.device
+    _need(traj_offsets, "traj_offsets", torch.int64, n_traj + 1, device=dev)
+    _need(mask, "mask", torch.uint8, T, device=dev)
+    _need(values, "values", torch.float32, T, device=dev)
+    _opt(token_rewards, "token_rewards", torch.float32, T, device=dev)
+    _opt(traj_rewards, "traj_rewards", torch.float32, n_traj, device=dev)
+    adv_out = torch.empty(T, dtype=torch.float32, device=dev) if adv_out is None else adv_out
+    if want_returns and returns_out is None:
+        returns_out = torch.empty(T, dtype=torch.float32, device=dev)
+    _need(adv_out, "adv_out", torch.float32, T, device=dev)
+    _opt(returns_out, "returns_out", torch.float32, T, device=dev)
+    _need(ws, "ws", torch.uint8, device=dev)
+    st = lib().rl_masked_gae(n_traj, _ptr(traj_offsets), T, _ptr(mask), _ptr(values), _ptr(token_rewards),
+                             _ptr(traj_rewards), float(gamma), float(gae_lambda), 1 if skip_masked else 0,
+                             _ptr(adv_out), _ptr(returns_out), _ptr(ws), ws.numel(), _stream(stream))
+    _check("rl_masked_gae", st)
+    return adv_out, returns_out
+
+
+def rl_value_loss_fwd_bwd(values, returns, mask, token_traj, coef, ws, loss_accum, d_values=None, stream=None):
+    """Adds sum_t c M (V - G)^2 to ``loss_accum`` (float64 [1]); returns d loss / d values (float32)."""
+    rows = values.numel()
+    dev = values.device
+    n_traj = coef.numel()
+    _need(values, "values", torch.float32, rows, device=dev)
+    _need(returns, "returns", torch.float32, rows, device=dev)
+    _need(mask, "mask", torch.uint8, rows, device=dev)
+    _need(token_traj, "token_traj", torch.int32, rows, device=dev)
+    _need(coef, "coef", torch.float32, n_traj, device=dev)
+    _need(loss_accum, "loss_accum", torch.float64, 1, device=dev)
+    d_values = torch.empty(rows, dtype=torch.float32, device=dev) if d_values is None else d_values
+    _need(d_values, "d_values", torch.float32, rows, device=dev)
+    _need(ws, "ws", torch.uint8, device=dev)
+    st = lib().rl_value_loss_fwd_bwd(rows, _ptr(values), _ptr(returns), _ptr(mask), _ptr(token_traj), n_traj,
+                                     _ptr(coef), _ptr(d_values), _ptr(loss_accum), _ptr(ws), ws.numel(),
+                                     _stream(stream))
+    _check("rl_value_loss_fwd_bwd", st)
+    return d_values

@@ -22,6 +22,10 @@ vocabulary):
   fusedhead  hidden bf16 [32,768 x 4,096] ~ N(0, 1), W bf16 [151,936 x 4,096] ~ N(0, 0.02^2),
              masks and rewards of the first 32,768 tokens of a multiturn batch
 
+For the PPO path, value predictions V(s_t) are N(0.3, 0.25^2) per token and the
+rollout reward R_i of the layout is placed at each trajectory's last trainable token;
+sparse per-token rewards can be added.
+
 Quantities that depend on the current policy's log-probability (old_logp,
 ref_logp) are formed as ``logp + noise``; the caller supplies ``logp`` from
 whichever side it is preparing inputs for, and this module only adds the
@@ -316,6 +320,22 @@ def rollout_logp_from(old_logp: np.ndarray, seed: int, std: float = 0.05, row0: 
     """Rollout-engine log-probs for TIS tests: old_logp + N(0, std^2)."""
     rng = _rng(seed, 99, 6, row0)
     return (np.asarray(old_logp, dtype=np.float64) + rng.normal(0.0, std, size=len(old_logp))).astype(np.float32)
+
+
+def value_predictions(w: Workload, seed: int, n_tokens: int, mean: float = 0.3, std: float = 0.25) -> np.ndarray:
+    """V(s_t) of a value model for the PPO path: N(mean, std^2) per token as float32 (mean at
+    the workloads' reward rate 0.3)."""
+    rng = _rng(seed, _name_id(w.name), 7)
+    return rng.normal(mean, std, size=n_tokens).astype(np.float32)
+
+
+def token_reward_draws(w: Workload, seed: int, n_tokens: int, frac: float = 0.05, std: float = 0.1) -> np.ndarray:
+    """Sparse per-token rewards r_t (a fraction `frac` of tokens, N(0, std^2)) as float32, to
+    exercise the per-token reward input of the GAE next to the final-token reward."""
+    rng = _rng(seed, _name_id(w.name), 8)
+    r = rng.normal(0.0, std, size=n_tokens)
+    r[rng.random(n_tokens) >= frac] = 0.0
+    return r.astype(np.float32)
 
 
 # ----------------------------------------------------------------------------

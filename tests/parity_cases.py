@@ -26,6 +26,7 @@ Tolerances (float32 kernels against the float64 oracle):
 from __future__ import annotations
 
 import dataclasses
+import math
 
 import numpy as np
 import torch
@@ -44,7 +45,52 @@ def loss_params(w: W.Workload, loss_agg=0, tis_cap=0.0):
 
 def cuda_params(R, P: O.LossParams):
     return R.make_params(P.clip_eps_low, P.clip_eps_high, P.kl_coef, P.kl_estimator, P.entropy_coef, P.tis_cap,
-                         P.adv_eps, P.loss_agg)
+                         P.adv_eps, P.loss_agg, int(P.token_level_adv))
+
+
+def gae_error_scale(offs, mask, values, rewards, gamma, lam, skip):
+    """S_t = sum_l (gamma lambda)^l |b_{t+l}| with |b_u| = M_u (|r_u| + gamma |V_next(u)| + |V_u|):
+    the size of the terms an fp32 evaluation of the GAE recursion adds up (V_next is the next
+    token's value in the printed reading, the next trainable token's in the skip reading).
+    A scan of depth k rounds each partial sum at most k times, so |error_t| <= k 2^-24 S_t."""
+    M = np.asarray(mask) != 0
+    V = np.abs(np.asarray(values, dtype=np.float64))
+    r = np.abs(np.asarray(rewards, dtype=np.float64))
+    S = np.zeros(len(V))
+    gl = gamma * lam
+    for i in range(len(offs) - 1):
+        s, e = int(offs[i]), int(offs[i + 1])
+        acc, vn = 0.0, 0.0
+        for t in range(e - 1, s - 1, -1):
+            if skip:
+                if M[t]:
+                    acc = r[t] + gamma * vn + V[t] + gl * acc
+                    vn = V[t]
+            else:
+                nb = V[t + 1] if (t + 1 < e and M[t + 1]) else 0.0
+                acc = (r[t] + gamma * nb + V[t] if M[t] else 0.0) + gl * acc
+            S[t] = acc
+    return np.where(M, S, 0.0)
+
+
+def check_gae(adv_dev, ret_dev, adv_ref, ret_ref, values, S, mask, max_len, what=""):
+    """fp32 scan against the float64 oracle: |d adv| <= k 2^-24 S_t + 2^-24 |A_t| with the scan
+    depth k = 64 + 2 ceil(L_max / 1024); returns add the rounding of A + V. Masked tokens: exactly 0."""
+    u = 2.0 ** -24
+    k = 64 + 2 * math.ceil(max(max_len, 1) / 1024)
+    M = np.asarray(mask) != 0
+    assert np.all(adv_dev[~M] == 0.0) and np.all(ret_dev[~M] == 0.0), f"{what}: masked tokens not zero"
+    tol = k * u * S + u * np.abs(adv_ref) + 1e-30
+    d = np.abs(adv_dev - adv_ref)
+    if np.any(d > tol):
+        t = int(np.argmax(d - tol))
+        raise AssertionError(f"{what}: adv token {t} gpu {adv_dev[t]} oracle {adv_ref[t]} tol {tol[t]}")
+    tol_r = tol + u * (np.abs(adv_ref) + np.abs(np.asarray(values, dtype=np.float64)))
+    d = np.abs(ret_dev - ret_ref)
+    if np.any(d > tol_r):
+        t = int(np.argmax(d - tol_r))
+        raise AssertionError(f"{what}: return token {t} gpu {ret_dev[t]} oracle {ret_ref[t]} tol {tol_r[t]}")
+    return float((np.abs(adv_dev - adv_ref) / np.maximum(S, 1e-30))[M].max(initial=0.0))
 
 
 @dataclasses.dataclass

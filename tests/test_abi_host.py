@@ -168,3 +168,50 @@ def test_fused_head_logprobs_argument_checks(R):
     assert call(ws_bytes=R.rl_workspace_size(20000, 151936, 4096), **big) == 1
     assert call(ws_bytes=256 + 16 * 38 * 8192, **big) == 1
     assert call(ws_bytes=256 + 16 * 38 * 8192 - 1, **big) == 4
+
+
+def test_masked_gae_argument_checks(R):
+    L = R.lib()
+
+    def call(**over):
+        a = dict(n=4, offs=FAKE, T=100, mask=FAKE, V=FAKE, rt=None, rr=None, g=0.99, l=0.95, skip=1, adv=FAKE,
+                 ret=None, ws=FAKE, ws_bytes=1024, stream=None)
+        a.update(over)
+        return L.rl_masked_gae(a["n"], a["offs"], a["T"], a["mask"], a["V"], a["rt"], a["rr"], a["g"], a["l"],
+                               a["skip"], a["adv"], a["ret"], a["ws"], a["ws_bytes"], a["stream"])
+
+    assert call(n=-1) == 1
+    assert call(T=-5) == 1
+    assert call(g=1.5) == 1
+    assert call(l=-0.1) == 1
+    assert call(g=float("nan")) == 1
+    assert call(skip=2) == 1
+    assert call(ws=None) == 1
+    assert call(ws_bytes=16) == 4
+    assert call(offs=None) == 1
+    assert call(adv=None) == 1
+    assert call(n=0) == 0
+
+
+def test_value_loss_argument_checks(R):
+    L = R.lib()
+
+    def call(**over):
+        a = dict(rows=16, V=FAKE, G=FAKE, mask=FAKE, tt=FAKE, n=2, coef=FAKE, dV=FAKE, loss=FAKE, ws=FAKE,
+                 ws_bytes=1 << 16, stream=None)
+        a.update(over)
+        return L.rl_value_loss_fwd_bwd(a["rows"], a["V"], a["G"], a["mask"], a["tt"], a["n"], a["coef"], a["dV"],
+                                       a["loss"], a["ws"], a["ws_bytes"], a["stream"])
+
+    assert call(rows=-1) == 1
+    assert call(n=-1) == 1
+    assert call(loss=None) == 1
+    assert call(ws_bytes=256 + 8 * 16 - 1) == 4
+    assert call(dV=None) == 1
+    assert call(coef=None) == 1
+    assert call(rows=0) == 0
+
+
+def test_token_level_adv_flag_checks(R):
+    assert _loss(R, params=_params(R, token_level_adv=2)) == 1
+    assert _loss(R, params=_params(R, token_level_adv=1), adv=None, n_traj=0) == 1

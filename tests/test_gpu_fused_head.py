@@ -147,6 +147,15 @@ def test_fused_head_matches_logits_path(R):
     assert abs(loss.item() - out["loss"]) <= 1e-4 * max(abs(loss.item()), 1e-12)
 
 
+def test_fused_head_token_level_adv(R):
+    """Per-token advantages (PPO, Sec. 2.3.1) through the fused head, token-mean weights."""
+    c = make_head_case(300, 128, 1000, seed=21, agg=1)
+    c["adv32"] = np.random.default_rng(22).normal(0, 1, c["T"]).astype(np.float32)
+    c["P"] = dataclasses.replace(c["P"], token_level_adv=True)
+    out = run_head(R, c)
+    compare_head(c, out)
+
+
 def check_logprobs(c, logp, H, lse, what):
     """Forward-only outputs against the oracle, with the logit allowance zerr per token."""
     ref_logp, ref_H, ref_lse = O.fused_head_logprobs(c["h"], c["w"], c["ids"])
