@@ -181,6 +181,65 @@ class DeviceBatch:
         return 2 + 2 * len(self.mbs)
 
 
+def time_ppo(torch, R, batch, dev, warmup=3, reps=20):
+    """PPO step on the same batch (Sec. 2.3.1, Sec. 2.3.4): token-mean coefficients, masked GAE over
+    the whole batch (skip reading, gamma = lambda = 1, R_i at each trajectory's last trainable token,
+    value predictions N(0.3, 0.25^2)), then per microbatch the clipped policy loss with per-token
+    advantages and the masked value loss."""
+    t = torch
+    w = WORKLOAD
+    d = lambda x: t.from_numpy(np.ascontiguousarray(x)).to(dev)  # noqa: E731
+    values = d(W.value_predictions(w, 0, batch.T))
+    v_new = values + 0.05  # the value model being trained
+    traj_r = batch.rewards.float()
+    params = R.make_params(W.CLIP_EPS_LOW, W.CLIP_EPS_HIGH, 0.0, 0, 0.0, 0.0, 1e-6, 1, token_level_adv=1)
+    coef = t.empty_like(batch.coef)
+    adv_traj = t.empty_like(batch.adv)
+    adv = t.empty(batch.T, dtype=t.float32, device=dev)
+    ret = t.empty_like(adv)
+    dv = t.empty_like(adv)
+    loss = t.zeros(1, dtype=t.float64, device=dev)
+    vloss = t.zeros(1, dtype=t.float64, device=dev)
+
+    def gae():
+        R.rl_masked_gae(batch.traj_offsets, batch.mask, values, batch.ws, 1.0, 1.0, True, traj_rewards=traj_r,
+                        adv_out=adv, returns_out=ret)
+
+    def step():
+        R.rl_group_advantages(batch.group_offsets, batch.rewards, batch.traj_offsets, batch.mask, params, batch.ws,
+                              traj_valid=batch.valid, adv_out=adv_traj, coef_out=coef, n_tok_out=batch.n_tok,
+                              token_traj_out=batch.token_traj)
+        gae()
+        for lo, hi in batch.mbs:
+            R.rl_policy_loss_fwd_bwd(batch.logits[lo:hi], batch.ids[lo:hi], batch.mask[lo:hi],
+                                     batch.token_traj[lo:hi], adv[lo:hi], coef, batch.old[lo:hi], params, batch.ws,
+                                     loss, grad_out=batch.grad[lo:hi])
+            R.rl_value_loss_fwd_bwd(v_new[lo:hi], ret[lo:hi], batch.mask[lo:hi], batch.token_traj[lo:hi], coef,
+                                    batch.ws, vloss, d_values=dv[lo:hi])
+
+    lo, hi = batch.mbs[0]
+    ms_step = _time_calls(torch, step, warmup, reps)
+    # the two small kernels are timed as CUDA-graph replays, so that host launch overhead stays out
+    ms_gae = _time_graph(torch, gae, 10 * reps)
+    ms_val = _time_graph(torch, lambda: R.rl_value_loss_fwd_bwd(v_new[lo:hi], ret[lo:hi], batch.mask[lo:hi],
+                                                                batch.token_traj[lo:hi], coef, batch.ws, vloss,
+                                                                d_values=dv[lo:hi]), 10 * reps)
+    st, word = R.rl_query_status(batch.ws)
+    if word != 0:
+        raise RuntimeError(f"device status word {word} after the PPO timing")
+    gae_bytes = batch.T * (1 + 4 + 4 + 4) + 8 * (batch.lay.n_traj + 1) + 4 * batch.lay.n_traj
+    val_bytes = (hi - lo) * (4 + 4 + 1 + 4 + 4 + 8) + 4 * batch.lay.n_traj
+    return {"workload": "multiturn batch: values N(0.3,0.25^2), gamma = lambda = 1, skip reading, token-mean weights",
+            "ms_per_step": ms_step, "tokens_per_s": batch.T / (ms_step * 1e-3),
+            "gae_us": ms_gae * 1e3, "gae_algorithmic_bytes": gae_bytes,
+            "gae_achieved_gbs": gae_bytes / (ms_gae * 1e-3) / 1e9,
+            "value_loss_us_per_microbatch": ms_val * 1e3, "value_loss_algorithmic_bytes": val_bytes,
+            "reps": reps,
+            "note": "step = advantages/coefficients + GAE + per microbatch (policy loss with per-token advantages "
+                    "+ value loss); GAE and value loss (+ its reduction) timed as CUDA-graph replays; both are "
+                    "latency-bound (a few bytes per token)"}
+
+
 def e2e_run(torch, R, batch, dev, steps, warmup):
     """Same step through host buffers: every step copies its inputs from pinned host memory
     (metadata + each microbatch's logits) and reads back the gradient and the loss.
@@ -491,6 +550,29 @@ class HeadBatch:
                                        entropy_out=self.ent)
 
 
+def _time_graph(torch, fn, reps, replays=5):
+    """Average device time of one fn() call: reps calls captured in a CUDA graph, replayed."""
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        for _ in range(3):
+            fn()
+    torch.cuda.current_stream().wait_stream(side)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for _ in range(reps):
+            fn()
+    g.replay()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(replays):
+        g.replay()
+    b.record()
+    b.synchronize()
+    return a.elapsed_time(b) / (replays * reps)
+
+
 def _time_calls(torch, fn, warmup, reps):
     for _ in range(warmup):
         fn()
@@ -609,6 +691,7 @@ def main():
     ap.add_argument("--profile-head", type=int, default=0, metavar="TOKENS",
                     help="run a small fused-head case for a profiler capture and exit")
     ap.add_argument("--no-head", action="store_true", help="skip the fused-head measurement")
+    ap.add_argument("--no-ppo", action="store_true", help="skip the PPO-step measurement")
     args = ap.parse_args()
     if args.profile_case:
         return profile_case(args.profile_case)
@@ -688,6 +771,8 @@ def main():
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = time_oracle(host_sample(torch, batch, 2048))
 
+    ppo = None if args.no_ppo else time_ppo(torch, R, batch, dev)
+
     head = None
     if not args.no_head:
         head = time_head(torch, R, dev)
@@ -696,7 +781,7 @@ def main():
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": "f32", "data": "synthetic", "config": workload_config(batch.T, n_mb),
-                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks, "fused_head": head,
+                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks, "fused_head": head, "ppo": ppo,
                 "gpu_launches": batch.launches_per_step() * args.steps,
                 "loss_per_step": float(batch.loss.item()) / (args.warmup + args.steps)}
         print(json.dumps(line))
