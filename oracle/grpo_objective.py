@@ -31,6 +31,9 @@ Every function follows one passage of the paper (arXiv 2608.16798, "ClawGym II")
 * ``fused_head_loss_fwd_bwd``  -- the same objective with logits = hidden @ W^T
   and gradients with respect to hidden and W.
 * ``fused_head_logprobs``      -- forward-only log-probabilities of logits = hidden @ W^T.
+* ``sequence_is_weights``      -- the sequence-level importance ratio between the training
+  engine's and the rollout engine's policies, truncated at c-bar (Sec. 3.2.4, the
+  sequence-level alternative to the token-level TIS weight).
 
 Readings of the paper where it is silent (all documented with the library):
 
@@ -48,7 +51,11 @@ Readings of the paper where it is silent (all documented with the library):
   subtracted from the loss;
 * the truncated importance weight w_t scales the surrogate term only and
   carries no gradient;
-* at a ratio exactly on a clip bound the surrogate gradient passes.
+* at a ratio exactly on a clip bound the surrogate gradient passes;
+* the sequence-level ratio multiplies pi_old / pi_rollout over the trainable tokens
+  (M_t = 1) of the unit that owns them (a trajectory, or a rollout's deduplicated tree);
+  like the token-level weight it scales the surrogate only, which for a positive weight
+  is the same as scaling the advantage; c-bar <= 0 leaves it untruncated.
 
 Rows with M_t = 0, or whose trajectory has c_i = 0, contribute nothing to the
 loss and get an exactly-zero gradient row.
@@ -381,3 +388,24 @@ def fused_head_logprobs(hidden_bf16, weight_bf16, token_ids, chunk: int = 256):
         l, lp, h, _, _ = row_statistics(Z, token_ids[r0:r0 + chunk])
         lse[r0:r0 + chunk], logp[r0:r0 + chunk], H[r0:r0 + chunk] = l, lp, h
     return logp, H, lse
+
+
+# ----------------------------------------------------------------------------
+# Sequence-level importance weight (Sec. 3.2.4)
+# ----------------------------------------------------------------------------
+
+def sequence_is_weights(token_traj, mask, old_logp, rollout_logp, n_traj: int, cap: float):
+    """S_i = sum over the trainable tokens t of unit i of (log pi_old - log pi_rollout);
+    w_i = min(exp(S_i), c-bar) (no truncation when c-bar <= 0).
+
+    Returns (w float64 [n_traj], S float64 [n_traj])."""
+    tt = np.asarray(token_traj, dtype=np.int64)
+    M = np.asarray(mask) != 0
+    d = np.asarray(old_logp, dtype=np.float64) - np.asarray(rollout_logp, dtype=np.float64)
+    S = np.zeros(n_traj)
+    for i in range(n_traj):
+        S[i] = math.fsum(d[(tt == i) & M].tolist())
+    w = np.exp(S)
+    if cap > 0:
+        w = np.minimum(w, cap)
+    return w, S

@@ -413,6 +413,46 @@ def pin_token_level_advantages(O):
     assert l0 == l1 and np.array_equal(g0, g1)
 
 
+def pin_sequence_is_weights(O):
+    """The sequence-level weight is the product of the per-token ratios pi_old / pi_rollout over
+    the unit's trainable tokens, truncated at c-bar; equal policies give w = 1; a unit with one
+    trainable token gets the token-level TIS weight, and the loss with advantages scaled by w_i
+    equals the loss with that token-level weight (both scale the surrogate only)."""
+    rng = np.random.default_rng(31)
+    T, n = 40, 5
+    tt = rng.integers(0, n, T)
+    mask = (rng.random(T) < 0.7).astype(np.uint8)
+    old = rng.normal(-2, 1, T)
+    roll = old + rng.normal(0, 0.05, T)
+    w, S = O.sequence_is_weights(tt, mask, old, roll, n, cap=0.0)
+    for i in range(n):
+        prod = 1.0
+        for t in range(T):
+            if tt[t] == i and mask[t]:
+                prod *= math.exp(old[t]) / math.exp(roll[t])
+        _close([w[i]], [prod], rtol=1e-12, what=f"product of ratios {i}")
+    wc, _ = O.sequence_is_weights(tt, mask, old, roll, n, cap=1.01)
+    _close(wc, np.minimum(w, 1.01), rtol=0, atol=0, what="truncation")
+    w1, S1 = O.sequence_is_weights(tt, mask, old, old, n, cap=2.0)
+    assert np.all(w1 == 1.0) and np.all(S1 == 0.0)
+    # one trainable token per trajectory: sequence weight == token-level TIS weight
+    pr = _tiny_problem(17, n_traj=4, agg=2, alpha=0.02, beta=0.03, tis=1.5)
+    z = pr["z"]
+    Tn = z.shape[0]
+    mask1 = np.zeros(Tn, np.uint8)
+    for i in range(4):
+        mask1[np.nonzero(pr["tt"] == i)[0][0]] = 1
+    P_tok = O.LossParams(**pr["P"])
+    pr_tok = dict(pr, mask=mask1)
+    l_tok, g_tok, _, _ = _loss(O, pr_tok, z, P_tok)
+    wseq, _ = O.sequence_is_weights(pr["tt"], mask1, pr["old"], pr["roll"], 4, cap=P_tok.tis_cap)
+    P_seq = O.LossParams(**dict(pr["P"], tis_cap=0.0))
+    l_seq, g_seq, _, _ = O.policy_loss_fwd_bwd(z, "f64", pr["a"], mask1, pr["tt"], pr["adv"] * wseq, pr["coef"],
+                                               pr["old"], P_seq, pr["ref"], None)
+    _close([l_seq], [l_tok], rtol=1e-12, atol=1e-15, what="sequence weight vs token weight, loss")
+    _close(g_seq, g_tok, rtol=1e-12, atol=1e-15, what="sequence weight vs token weight, grad")
+
+
 def pin_loss_additive_and_permutation(O):
     """The loss of two microbatches adds up to the loss of the whole batch; permuting the
     rows permutes the gradient rows and keeps the loss."""

@@ -59,6 +59,11 @@ MUTANTS = {
     "head logits transposed": ("Z = Hm @ Wm.T", "Z = (Hm @ Wm.T).T"),
     "token-level adv ignored": ("A_row = adv[sel] if params.token_level_adv else adv[token_traj[sel]]",
                                 "A_row = adv[token_traj[sel]]"),
+    "seq weight includes masked tokens": ("S[i] = math.fsum(d[(tt == i) & M].tolist())",
+                                          "S[i] = math.fsum(d[tt == i].tolist())"),
+    "seq weight inverted ratio": ("d = np.asarray(old_logp, dtype=np.float64) - np.asarray(rollout_logp, dtype=np.float64)",
+                                  "d = np.asarray(rollout_logp, dtype=np.float64) - np.asarray(old_logp, dtype=np.float64)"),
+    "seq weight cap as max": ("w = np.minimum(w, cap)", "w = np.maximum(w, cap)"),
     "head logprobs chunk offset": ("Z = Hm[r0:r0 + chunk] @ Wm.T", "Z = Hm[r0 + 1:r0 + 1 + chunk] @ Wm.T"),
 }
 
