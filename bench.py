@@ -224,6 +224,12 @@ def time_ppo(torch, R, batch, dev, warmup=3, reps=20):
     ms_val = _time_graph(torch, lambda: R.rl_value_loss_fwd_bwd(v_new[lo:hi], ret[lo:hi], batch.mask[lo:hi],
                                                                 batch.token_traj[lo:hi], coef, batch.ws, vloss,
                                                                 d_values=dv[lo:hi]), 10 * reps)
+    # sequence-level importance weights over the whole batch (rollout log-probs = old + N(0, 0.02^2))
+    roll = d(W.rollout_logp_from(batch.old.cpu().numpy(), 0, std=0.02))
+    w_seq = t.empty(batch.lay.n_traj, dtype=t.float32, device=dev)
+    ms_seq = _time_graph(torch, lambda: R.rl_sequence_is_weights(batch.token_traj, batch.mask, batch.old, roll,
+                                                                 batch.lay.n_traj, batch.ws, cap=2.0,
+                                                                 weight_out=w_seq), 10 * reps)
     st, word = R.rl_query_status(batch.ws)
     if word != 0:
         raise RuntimeError(f"device status word {word} after the PPO timing")
@@ -234,6 +240,7 @@ def time_ppo(torch, R, batch, dev, warmup=3, reps=20):
             "gae_us": ms_gae * 1e3, "gae_algorithmic_bytes": gae_bytes,
             "gae_achieved_gbs": gae_bytes / (ms_gae * 1e-3) / 1e9,
             "value_loss_us_per_microbatch": ms_val * 1e3, "value_loss_algorithmic_bytes": val_bytes,
+            "sequence_is_us": ms_seq * 1e3, "sequence_is_algorithmic_bytes": batch.T * (4 + 1 + 4 + 4),
             "reps": reps,
             "note": "step = advantages/coefficients + GAE + per microbatch (policy loss with per-token advantages "
                     "+ value loss); GAE and value loss (+ its reduction) timed as CUDA-graph replays; both are "

@@ -73,7 +73,8 @@ enum {
   RL_DEV_BAD_TOKEN = 1,   /* a token id outside [0, V); that row gets no loss and a zero gradient */
   RL_DEV_BAD_TRAJ = 2,    /* token_traj outside [0, n_traj); same treatment */
   RL_DEV_BAD_OFFSETS = 4, /* group / trajectory offsets not non-decreasing within range */
-  RL_DEV_TIMEOUT = 8      /* a bounded wait for an asynchronous copy ran out */
+  RL_DEV_TIMEOUT = 8,     /* a bounded wait for an asynchronous copy ran out */
+  RL_DEV_BAD_VALUE = 16   /* a non-finite or out-of-range input value (rl_sequence_is_weights) */
 };
 
 typedef struct rl_loss_params {
@@ -295,6 +296,41 @@ rl_status rl_masked_gae(int32_t n_traj, const int64_t* traj_offsets, int64_t n_t
 rl_status rl_value_loss_fwd_bwd(int64_t rows, const float* values, const float* returns, const uint8_t* mask,
                                 const int32_t* token_traj, int32_t n_traj, const float* coef, float* d_values,
                                 double* loss_accum, void* ws, size_t ws_bytes, rl_stream_t stream);
+
+/*
+ * Sequence-level importance weights (Sec. 3.2.4: the sequence-level importance ratio
+ * between the training engine's pi_old and the rollout engine's pi_rollout, the
+ * unbiased alternative to the token-level TIS weight), truncated at c-bar:
+ *   S_i = sum over tokens t with owner i and M_t = 1 of (log pi_old(a_t) - log pi_rollout(a_t)),
+ *   w_i = min(exp(S_i), cap)   (no truncation when cap <= 0).
+ * Like the token-level weight, w_i scales the surrogate term only. For a positive weight
+ * that is the same as scaling the advantage, so the weights are applied by scaling the
+ * advantages handed to rl_policy_loss_fwd_bwd / rl_fused_head_loss_fwd_bwd (in place here,
+ * if asked); the loss entry points are unchanged.
+ *
+ *   n_traj, n_tokens   units (trajectories, or rollouts of a tree-packed batch) and tokens of
+ *                      the WHOLE batch (a unit's sum spans microbatches)
+ *   token_traj         int32 [n_tokens]: owner of each token, any order (a unit's tokens need
+ *                      not be contiguous); an owner outside [0, n_traj) on a token with
+ *                      M_t != 0 sets RL_DEV_BAD_TRAJ and the token is skipped
+ *   mask               uint8 [n_tokens]
+ *   old_logp, rollout_logp  float [n_tokens]; a difference that is not finite or above 2^22
+ *                      in magnitude sets RL_DEV_BAD_VALUE (it is clamped, NaN counts as 0)
+ *   cap                c-bar
+ *   weight_out         float [n_traj]: w_i
+ *   log_ratio_out      float [n_traj] or NULL: S_i
+ *   traj_adv_inout     float [n_traj] or NULL: A_i, multiplied by w_i in place
+ *   token_adv_inout    float [n_tokens] or NULL: A_t (per-token advantages), multiplied by
+ *                      w_{owner(t)} in place
+ *   ws, ws_bytes       workspace of at least rl_workspace_size(n_traj, 0, 0) bytes
+ * Each difference is taken in double and rounded to a multiple of 2^-40; the sums are
+ * 64-bit integer additions, so the result is independent of the order in which the GPU
+ * adds the tokens (bit-reproducible). |S_i error| <= (tokens of unit i) x 2^-41.
+ */
+rl_status rl_sequence_is_weights(int32_t n_traj, int64_t n_tokens, const int32_t* token_traj, const uint8_t* mask,
+                                 const float* old_logp, const float* rollout_logp, float cap, float* weight_out,
+                                 float* log_ratio_out, float* traj_adv_inout, float* token_adv_inout, void* ws,
+                                 size_t ws_bytes, rl_stream_t stream);
 
 /*
  * Forward-only log-probabilities through the fused LM head (the pi_old / pi_ref

@@ -22,7 +22,7 @@ RL_OK = 0
 STATUS_NAMES = {0: "RL_OK", 1: "RL_ERR_INVALID_ARG", 2: "RL_ERR_UNSUPPORTED", 3: "RL_ERR_ALIGNMENT",
                 4: "RL_ERR_WORKSPACE_TOO_SMALL", 5: "RL_ERR_CUDA", 6: "RL_ERR_DEVICE_CHECK", 7: "RL_ERR_TIMEOUT"}
 RL_BF16, RL_F32 = 0, 1
-RL_DEV_BAD_TOKEN, RL_DEV_BAD_TRAJ, RL_DEV_BAD_OFFSETS, RL_DEV_TIMEOUT = 1, 2, 4, 8
+RL_DEV_BAD_TOKEN, RL_DEV_BAD_TRAJ, RL_DEV_BAD_OFFSETS, RL_DEV_TIMEOUT, RL_DEV_BAD_VALUE = 1, 2, 4, 8, 16
 AGG_SEQ_MEAN_TOKEN_MEAN, AGG_TOKEN_MEAN, AGG_TOKEN_SUM = 0, 1, 2
 
 # C function name -> (restype, argtypes)
@@ -40,6 +40,7 @@ EXPORTS = {
                                       _P, _P, _P, _P, _SZ, _P]),
     "rl_policy_loss_fwd_bwd_noalloc": (_I32, [_P, _I32, _I64, _I64, _I64, _P, _P, _P, _I32, _P, _P, _P, _P, _P,
                                               _P, _P, _P, _P, _P, _P]),
+    "rl_sequence_is_weights": (_I32, [_I32, _I64, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P, _SZ, _P]),
     "rl_masked_gae": (_I32, [_I32, _P, _I64, _P, _P, _P, _P, _F, _F, _I32, _P, _P, _P, _SZ, _P]),
     "rl_value_loss_fwd_bwd": (_I32, [_I64, _P, _P, _P, _P, _I32, _P, _P, _P, _P, _SZ, _P]),
     "rl_fused_head_token_logprobs": (_I32, [_P, _P, _I64, _I64, _I64, _P, _P, _P, _P, _P, _SZ, _P]),
@@ -403,3 +404,30 @@ def rl_value_loss_fwd_bwd(values, returns, mask, token_traj, coef, ws, loss_accu
                                      _stream(stream))
     _check("rl_value_loss_fwd_bwd", st)
     return d_values
+
+
+def rl_sequence_is_weights(token_traj, mask, old_logp, rollout_logp, n_traj, ws, cap=0.0, weight_out=None,
+                           log_ratio_out=None, want_log_ratio=False, traj_adv_inout=None, token_adv_inout=None,
+                           stream=None):
+    """Sequence-level importance weights w_i = min(exp(sum_t M (old - rollout)), cap) over the
+    tokens each unit owns (Sec. 3.2.4); optionally scales advantages in place. Returns
+    (weight, log_ratio)."""
+    T = mask.numel()
+    dev = mask.device
+    _need(token_traj, "token_traj", torch.int32, T, device=dev)
+    _need(mask, "mask", torch.uint8, T, device=dev)
+    _need(old_logp, "old_logp", torch.float32, T, device=dev)
+    _need(rollout_logp, "rollout_logp", torch.float32, T, device=dev)
+    weight_out = torch.empty(n_traj, dtype=torch.float32, device=dev) if weight_out is None else weight_out
+    if want_log_ratio and log_ratio_out is None:
+        log_ratio_out = torch.empty(n_traj, dtype=torch.float32, device=dev)
+    _need(weight_out, "weight_out", torch.float32, n_traj, device=dev)
+    _opt(log_ratio_out, "log_ratio_out", torch.float32, n_traj, device=dev)
+    _opt(traj_adv_inout, "traj_adv_inout", torch.float32, n_traj, device=dev)
+    _opt(token_adv_inout, "token_adv_inout", torch.float32, T, device=dev)
+    _need(ws, "ws", torch.uint8, device=dev)
+    st = lib().rl_sequence_is_weights(n_traj, T, _ptr(token_traj), _ptr(mask), _ptr(old_logp), _ptr(rollout_logp),
+                                      float(cap), _ptr(weight_out), _ptr(log_ratio_out), _ptr(traj_adv_inout),
+                                      _ptr(token_adv_inout), _ptr(ws), ws.numel(), _stream(stream))
+    _check("rl_sequence_is_weights", st)
+    return weight_out, log_ratio_out

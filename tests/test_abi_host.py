@@ -215,3 +215,23 @@ def test_value_loss_argument_checks(R):
 def test_token_level_adv_flag_checks(R):
     assert _loss(R, params=_params(R, token_level_adv=2)) == 1
     assert _loss(R, params=_params(R, token_level_adv=1), adv=None, n_traj=0) == 1
+
+
+def test_sequence_is_weights_argument_checks(R):
+    L = R.lib()
+
+    def call(**over):
+        a = dict(n=4, T=100, tt=FAKE, mask=FAKE, old=FAKE, roll=FAKE, cap=2.0, w=FAKE, S=None, ta=None, tk=None,
+                 ws=FAKE, ws_bytes=1024, stream=None)
+        a.update(over)
+        return L.rl_sequence_is_weights(a["n"], a["T"], a["tt"], a["mask"], a["old"], a["roll"], a["cap"], a["w"],
+                                        a["S"], a["ta"], a["tk"], a["ws"], a["ws_bytes"], a["stream"])
+
+    assert call(n=-1) == 1
+    assert call(T=-1) == 1
+    assert call(cap=float("nan")) == 1
+    assert call(ws=None) == 1
+    assert call(n=200, ws_bytes=256 + 8 * 200 - 1) == 4
+    assert call(w=None) == 1
+    assert call(roll=None) == 1
+    assert call(n=0) == 0
