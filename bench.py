@@ -247,6 +247,47 @@ def time_ppo(torch, R, batch, dev, warmup=3, reps=20):
                     "latency-bound (a few bytes per token)"}
 
 
+def time_tree(torch, R, dev, reps=3):
+    """Tree-packed batches (Sec. 3.2.1-3.2.3): the native prefix-tree builder over the tree
+    workload's 128 rollouts on the host cores, then advantages and coefficients by owner and the
+    sequence-level weights on the packed stream (CUDA-graph replays)."""
+    t = torch
+    w = W.WORKLOADS["tree"]
+    prompts, calls, aux = W.tree_rollouts(w, seed=0)
+    captured = sum(len(x) + len(y) for cs in calls for x, y in cs)
+    threads = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else (os.cpu_count() or 1)
+    R.rl_prefix_tree_build_batch(prompts, calls, aux, max_leaves=w.tree_max_leaves, n_threads=threads)
+    t0 = time.perf_counter()
+    for _ in range(reps):
+        out = R.rl_prefix_tree_build_batch(prompts, calls, aux, max_leaves=w.tree_max_leaves, n_threads=threads)
+    host_s = (time.perf_counter() - t0) / reps
+    n = len(prompts)
+    d = lambda x: t.from_numpy(np.ascontiguousarray(x)).to(dev)  # noqa: E731
+    owner, mask = d(out["owner"]), d(out["mask"])
+    go = d(np.arange(0, n + 1, w.group_size, dtype=np.int32))
+    rewards = d((np.random.default_rng(0).random(n) < w.reward_p).astype(np.float32))
+    valid = d(np.array([s["valid"] for s in out["stats"]], np.uint8))
+    params = R.make_params(W.CLIP_EPS_LOW, W.CLIP_EPS_HIGH, 0.0, 0, 0.0, 0.0, 1e-6, 0)
+    ws = R.new_workspace(n, 0, device=dev)
+    adv, coef, L = (t.empty(n, dtype=dt, device=dev) for dt in (t.float32, t.float32, t.int32))
+    ms_adv = _time_graph(torch, lambda: R.rl_group_advantages_by_owner(go, rewards, owner, mask, params, ws,
+                                                                       traj_valid=valid, adv_out=adv, coef_out=coef,
+                                                                       n_tok_out=L), 50)
+    st, word = R.rl_query_status(ws)
+    if word != 0:
+        raise RuntimeError(f"device status word {word} after the tree timing")
+    T = len(out["tokens"])
+    return {"workload": "tree: 16 tasks x 8 rollouts of captured calls (prompt U{200..800}, 4-16 turns, tool "
+                        "outputs, 10% retries, subagent and compaction calls, 1 in 20 runaway), max 12 leaves",
+            "calls": sum(len(c) for c in calls), "captured_tokens": captured, "packed_tokens": T,
+            "trainable_tokens": int(out["mask"].sum()), "rollouts_kept": int(sum(s["valid"] for s in out["stats"])),
+            "dedup_ratio": captured / max(T, 1), "host_build_ms": host_s * 1e3, "host_threads": threads,
+            "host_captured_tokens_per_s": captured / host_s,
+            "advantages_by_owner_us": ms_adv * 1e3,
+            "note": "host build = rl_prefix_tree_build_batch (C++, one thread per rollout at a time); "
+                    "advantages by owner timed as CUDA-graph replays"}
+
+
 def e2e_run(torch, R, batch, dev, steps, warmup):
     """Same step through host buffers: every step copies its inputs from pinned host memory
     (metadata + each microbatch's logits) and reads back the gradient and the loss.
@@ -699,6 +740,7 @@ def main():
                     help="run a small fused-head case for a profiler capture and exit")
     ap.add_argument("--no-head", action="store_true", help="skip the fused-head measurement")
     ap.add_argument("--no-ppo", action="store_true", help="skip the PPO-step measurement")
+    ap.add_argument("--no-tree", action="store_true", help="skip the prefix-tree measurement")
     args = ap.parse_args()
     if args.profile_case:
         return profile_case(args.profile_case)
@@ -779,6 +821,7 @@ def main():
         cpu = time_oracle(host_sample(torch, batch, 2048))
 
     ppo = None if args.no_ppo else time_ppo(torch, R, batch, dev)
+    tree = None if args.no_tree else time_tree(torch, R, dev)
 
     head = None
     if not args.no_head:
@@ -788,7 +831,7 @@ def main():
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": "f32", "data": "synthetic", "config": workload_config(batch.T, n_mb),
-                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks, "fused_head": head, "ppo": ppo,
+                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks, "fused_head": head, "ppo": ppo, "tree": tree,
                 "gpu_launches": batch.launches_per_step() * args.steps,
                 "loss_per_step": float(batch.loss.item()) / (args.warmup + args.steps)}
         print(json.dumps(line))

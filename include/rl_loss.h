@@ -298,6 +298,46 @@ rl_status rl_value_loss_fwd_bwd(int64_t rows, const float* values, const float* 
                                 double* loss_accum, void* ws, size_t ws_bytes, rl_stream_t stream);
 
 /*
+ * rl_group_advantages for tokens in any order (tree-packed batches, Sec. 3.2.3): the owner
+ * of every token is given instead of contiguous spans, so a rollout's deduplicated prefix-tree
+ * tokens (rl_prefix_tree_build_batch) or an interleaved packing can be used directly. The
+ * advantage A_i of rollout i (Sec. 3.2.3, GRPO over the n rollouts of a task) is assigned to
+ * all its trainable token nodes, each shared prefix token once; L_i counts those nodes.
+ *
+ *   n_traj, n_groups, group_offsets, rewards, traj_valid, params, adv_out, coef_out
+ *                  as for rl_group_advantages
+ *   n_tokens       T
+ *   token_traj     int32 [T]: owner of each token (any order); an owner outside [0, n_traj)
+ *                  on a token with M_t != 0 sets RL_DEV_BAD_TRAJ and the token is not counted
+ *   mask           uint8 [T]
+ *   n_tok_out      int32 [n_traj]: L_i (overwritten; exact, independent of token order)
+ *   ws, ws_bytes   rl_workspace_size(0, 0, 0) bytes suffice
+ */
+rl_status rl_group_advantages_by_owner(int32_t n_traj, int32_t n_groups, const int32_t* group_offsets,
+                                       const float* rewards, const uint8_t* traj_valid, int64_t n_tokens,
+                                       const int32_t* token_traj, const uint8_t* mask, const rl_loss_params* params,
+                                       float* adv_out, float* coef_out, int32_t* n_tok_out, void* ws,
+                                       size_t ws_bytes, rl_stream_t stream);
+
+/*
+ * PPO advantages with gamma = lambda = 1 for tokens in any order (Sec. 2.3.4: every
+ * trajectory of a rollout receives R_i at its final token and is backed up on its own, so
+ * A_t = R_i - V(s_t); on a prefix shared by several trajectories of a tree all of them give
+ * the same value):
+ *   A_t = R_{i(t)} - V_t and G_t = R_{i(t)} for M_t != 0, A_t = G_t = 0 otherwise.
+ *
+ *   n_tokens, token_traj, mask   as for rl_group_advantages_by_owner
+ *   values         float [n_tokens]: V(s_t)
+ *   rewards        float [n_traj]: R_i
+ *   adv_out        float [n_tokens]
+ *   returns_out    float [n_tokens] or NULL
+ *   ws, ws_bytes   rl_workspace_size(0, 0, 0) bytes suffice
+ */
+rl_status rl_rollout_value_advantages(int64_t n_tokens, const int32_t* token_traj, const uint8_t* mask,
+                                      const float* values, const float* rewards, int32_t n_traj, float* adv_out,
+                                      float* returns_out, void* ws, size_t ws_bytes, rl_stream_t stream);
+
+/*
  * Sequence-level importance weights (Sec. 3.2.4: the sequence-level importance ratio
  * between the training engine's pi_old and the rollout engine's pi_rollout, the
  * unbiased alternative to the token-level TIS weight), truncated at c-bar:
@@ -385,6 +425,72 @@ rl_status rl_policy_loss_fwd_bwd_noalloc(const void* logits, rl_dtype dtype, int
                                          const float* rollout_logp, const rl_loss_params* params,
                                          void* grad_out, double* loss_accum, float* token_stats,
                                          int32_t* device_status, rl_stream_t stream);
+
+/*
+ * Rollout-level prefix trees for a batch of rollouts, packed into one deduplicated token
+ * stream (HOST function: every pointer here is a host pointer; nothing touches the GPU).
+ * Sec. 3.2.1 "Prefix Tree Construction": the captured model calls (x_i, y_i) of a rollout
+ * form a tree rooted at the initial task prompt; each call is attached to the existing node
+ * whose accumulated history is the longest prefix of x_i (the earliest node on ties), and the
+ * part of x_i past that history is the harness content in between (tool outputs, environment
+ * feedback). Sec. 3.2.2 "Trajectory Extraction and Filtering": a rollout whose tree has more
+ * than max_leaves leaves (max_leaves > 0) is discarded; auxiliary calls (subagent, context
+ * compaction) are removed with their subtrees; the root's children are grouped into segments
+ * by equal input (a compaction starts a new one) and in each segment only the leaf with the
+ * longest history is kept (the others are dead leaves of retries). Sec. 3.2.3: the kept
+ * trajectories' nodes are written once each, so shared prefixes count once in the loss.
+ *
+ *   n_rollouts
+ *   prompt_offsets, prompt_tokens  CSR [n_rollouts + 1]: rollout r's task prompt
+ *   call_offsets                   int32 [n_rollouts + 1]: rollout r owns calls
+ *                                  [call_offsets[r], call_offsets[r+1]) in capture order
+ *   x_offsets, x_tokens            CSR [n_calls + 1]: each call's input context
+ *   y_offsets, y_tokens            CSR [n_calls + 1]: each call's response
+ *   aux                            uint8 [n_calls] or NULL: 1 = auxiliary call
+ *   max_leaves                     <= 0: no limit
+ *   n_threads                      host threads (<= 1: the calling thread only)
+ *   capacity                       length of the per-token outputs
+ * Per packed token (rollouts in order, each rollout's kept nodes in depth-first preorder,
+ * children in creation order):
+ *   tokens_out     int32: token id
+ *   mask_out       uint8: 1 for response tokens, 0 for prompt and harness tokens (M_t)
+ *   parent_out     int64: position of the previous token on the token's path, -1 for the
+ *                  first prompt token (the row whose logits predicted this token)
+ *   depth_out      int32 or NULL: index of the token along its path (position id)
+ *   owner_out      int32 or NULL: rollout index (token_traj of the loss entry points)
+ *   node_call_out  int32 or NULL: global call index of the token's node, -1 for the prompt
+ * Per kept leaf (rollouts in order, preorder within a rollout), at most n_calls:
+ *   leaf_call_out  int32 or NULL: global call index of the leaf
+ *   leaf_end_out   int64 or NULL: position of the leaf's last token (-1 if its path is empty)
+ *   leaf_offsets_out int64 [n_rollouts + 1] or NULL
+ * Per rollout:
+ *   stats_out            rl_tree_stats [n_rollouts] or NULL
+ *   rollout_offsets_out  int64 [n_rollouts + 1] or NULL: rollout r's tokens are
+ *                        [rollout_offsets[r], rollout_offsets[r+1]) (empty if discarded)
+ *   n_tokens_out         total packed tokens (always written)
+ * When the packed stream is longer than capacity the call returns
+ * RL_ERR_WORKSPACE_TOO_SMALL after writing n_tokens_out, stats and offsets, so that a caller
+ * can size the outputs and call again (capacity 0 with NULL outputs is a size query).
+ * Offsets must be non-decreasing (RL_ERR_INVALID_ARG otherwise). The function allocates host
+ * memory for its temporary trees.
+ */
+typedef struct rl_tree_stats {
+  int32_t valid;          /* 0: discarded for over-branching */
+  int32_t n_leaves;       /* leaves of the whole tree (auxiliary calls included) */
+  int32_t n_kept_leaves;  /* trajectories kept for training */
+  int32_t n_unplaced;     /* calls whose input does not start with the prompt */
+  int64_t n_tokens;       /* packed tokens of the rollout */
+  int64_t n_trainable;    /* of which responses (M_t = 1) */
+} rl_tree_stats;
+
+rl_status rl_prefix_tree_build_batch(int32_t n_rollouts, const int64_t* prompt_offsets, const int32_t* prompt_tokens,
+                                     const int32_t* call_offsets, const int64_t* x_offsets, const int32_t* x_tokens,
+                                     const int64_t* y_offsets, const int32_t* y_tokens, const uint8_t* aux,
+                                     int32_t max_leaves, int32_t n_threads, int64_t capacity, int32_t* tokens_out,
+                                     uint8_t* mask_out, int64_t* parent_out, int32_t* depth_out, int32_t* owner_out,
+                                     int32_t* node_call_out, int32_t* leaf_call_out, int64_t* leaf_end_out,
+                                     int64_t* leaf_offsets_out, rl_tree_stats* stats_out,
+                                     int64_t* rollout_offsets_out, int64_t* n_tokens_out);
 
 #ifdef __cplusplus
 }

@@ -1,6 +1,7 @@
 """Build the C-ABI shared library ``librl_loss.so`` in-tree with nvcc for sm_103a.
 
-Each ``csrc/*.cu`` is compiled to an object in parallel, then linked with the
+Each ``csrc/*.cu`` (device code) and ``csrc/*.cpp`` (host code) is compiled to an object
+in parallel, then linked with the
 CUDA runtime (static) into ``paper_2608_16798_gb300/librl_loss.so``. Objects
 go to ``paper_2608_16798_gb300/_build/``. A rebuild is skipped when the
 library is newer than every source and header.
@@ -34,7 +35,7 @@ def nvcc() -> str:
 
 
 def sources():
-    return sorted(os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith(".cu"))
+    return sorted(os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith((".cu", ".cpp")))
 
 
 def _inputs():
@@ -59,7 +60,7 @@ def build(verbose: bool = False, force: bool = False, extra_flags=()) -> str:
     cc = nvcc()
 
     def compile_one(src):
-        obj = os.path.join(BUILD, os.path.basename(src)[:-3] + ".o")
+        obj = os.path.join(BUILD, os.path.splitext(os.path.basename(src))[0] + ".o")
         cmd = [cc, *ARCH, *NVCC_FLAGS, *extra_flags, "-c", src, "-o", obj]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
@@ -73,7 +74,7 @@ def build(verbose: bool = False, force: bool = False, extra_flags=()) -> str:
     tmp = LIB + ".tmp"
     cuda_lib = os.path.join(os.path.dirname(os.path.dirname(os.path.realpath(cc))), "lib64")
     cmd = [cc, *ARCH, "-shared", "-o", tmp, *objs, "-cudart", "static", "-L", cuda_lib, "-lcublasLt",
-           "-Xlinker", f"-rpath={cuda_lib}"]
+           "-lpthread", "-Xlinker", f"-rpath={cuda_lib}"]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")

@@ -46,6 +46,28 @@ __global__ void __launch_bounds__(256) traj_count_kernel(int32_t n_traj, int64_t
   if (lane == 0) n_tok_out[i] = cnt;
 }
 
+// L_i by owner, for tokens in any order (tree-packed batches, Sec. 3.2.3: each shared prefix
+// token is one token of its rollout): lanes of a warp with the same owner are counted together
+// and one integer atomic per owner and warp adds them (the counts are exact in any order).
+__global__ void __launch_bounds__(256) owner_count_kernel(int64_t n_tokens, const int32_t* __restrict__ token_traj,
+                                                          const uint8_t* __restrict__ mask, int32_t n_traj,
+                                                          int32_t* __restrict__ n_tok_out, int32_t* status) {
+  const int lane = threadIdx.x & 31;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t base = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x - lane; base < n_tokens;
+       base += stride) {
+    const int64_t t = base + lane;
+    int32_t who = -1;
+    if (t < n_tokens && mask[t] != 0) {
+      const int32_t i = token_traj[t];
+      if (i < 0 || i >= n_traj) flag_status(status, RL_DEV_BAD_TRAJ);
+      else who = i;
+    }
+    const unsigned peers = __match_any_sync(0xffffffffu, who);
+    if (who >= 0 && lane == __ffs(peers) - 1) atomicAdd(&n_tok_out[who], __popc(peers));
+  }
+}
+
 constexpr int kAdvThreads = 1024;
 
 __global__ void __launch_bounds__(kAdvThreads) group_adv_kernel(
@@ -174,5 +196,47 @@ extern "C" rl_status rl_group_advantages(int32_t n_traj, int32_t n_groups, const
                                              coef_out, status);
   e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_error(e, "rl_group_advantages: group_adv_kernel launch");
+  return RL_OK;
+}
+
+extern "C" rl_status rl_group_advantages_by_owner(int32_t n_traj, int32_t n_groups, const int32_t* group_offsets,
+                                                  const float* rewards, const uint8_t* traj_valid, int64_t n_tokens,
+                                                  const int32_t* token_traj, const uint8_t* mask,
+                                                  const rl_loss_params* params, float* adv_out, float* coef_out,
+                                                  int32_t* n_tok_out, void* ws, size_t ws_bytes,
+                                                  rl_stream_t stream) {
+  using namespace rl;
+  clear_error();
+  if (n_traj < 0 || n_groups < 0 || n_tokens < 0)
+    return set_error(RL_ERR_INVALID_ARG, "rl_group_advantages_by_owner: negative size");
+  if (!params) return set_error(RL_ERR_INVALID_ARG, "rl_group_advantages_by_owner: params is NULL");
+  if (!ws) return set_error(RL_ERR_INVALID_ARG, "rl_group_advantages_by_owner: ws is NULL");
+  if (ws_bytes < rl_workspace_size(0, 0, 0))
+    return set_error(RL_ERR_WORKSPACE_TOO_SMALL, "rl_group_advantages_by_owner: workspace too small");
+  if (params->loss_agg < RL_AGG_SEQ_MEAN_TOKEN_MEAN || params->loss_agg > RL_AGG_TOKEN_SUM)
+    return set_error(RL_ERR_INVALID_ARG, "rl_group_advantages_by_owner: unknown loss_agg");
+  if (!(params->adv_eps >= 0.f)) return set_error(RL_ERR_INVALID_ARG, "rl_group_advantages_by_owner: adv_eps < 0");
+  if (n_traj == 0) return RL_OK;
+  if (!group_offsets && n_groups > 0)
+    return set_error(RL_ERR_INVALID_ARG, "rl_group_advantages_by_owner: group_offsets is NULL");
+  if (!rewards || !adv_out || !coef_out || !n_tok_out || (n_tokens > 0 && (!token_traj || !mask)))
+    return set_error(RL_ERR_INVALID_ARG, "rl_group_advantages_by_owner: NULL array argument");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  int32_t* status = reinterpret_cast<int32_t*>(ws);
+  cudaError_t e = cudaMemsetAsync(n_tok_out, 0, static_cast<size_t>(n_traj) * sizeof(int32_t), s);
+  if (e != cudaSuccess) return cuda_error(e, "rl_group_advantages_by_owner: cudaMemsetAsync");
+  if (n_tokens > 0) {
+    int64_t blocks = (n_tokens + 255) / 256;
+    if (blocks > 152 * 8) blocks = 152 * 8;
+    owner_count_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(n_tokens, token_traj, mask, n_traj, n_tok_out,
+                                                                     status);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_error(e, "rl_group_advantages_by_owner: owner_count_kernel launch");
+  }
+  group_adv_kernel<<<1, kAdvThreads, 0, s>>>(n_traj, n_groups, group_offsets, rewards, traj_valid, n_tok_out,
+                                             static_cast<double>(params->adv_eps), params->loss_agg, adv_out,
+                                             coef_out, status);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_error(e, "rl_group_advantages_by_owner: group_adv_kernel launch");
   return RL_OK;
 }

@@ -17,6 +17,9 @@
 //   value_loss_kernel  per token: c M (V - G)^2 into the per-row loss slots, and
 //                      dV = 2 c M (V - G); the fixed-order reduction of rl_rows.cu adds
 //                      the slots into the caller's accumulator.
+//   rollout_adv_kernel A_t = R_i - V_t, G_t = R_i per token for tokens in any order (the
+//                      gamma = lambda = 1 form of Sec. 2.3.4, which also holds on the shared
+//                      prefixes of a rollout's prefix tree).
 //
 // Both touch a few bytes per token (mask, values, rewards, outputs) and are latency- or
 // launch-bound next to the logits stream.
@@ -210,6 +213,30 @@ __global__ void __launch_bounds__(256) value_loss_kernel(const ValueArgs p) {
   }
 }
 
+// A_t = R_{i(t)} - V_t and G_t = R_{i(t)} on trainable tokens, 0 elsewhere (any token order).
+__global__ void __launch_bounds__(256) rollout_adv_kernel(int64_t T, const int32_t* __restrict__ token_traj,
+                                                          const uint8_t* __restrict__ mask,
+                                                          const float* __restrict__ values,
+                                                          const float* __restrict__ rewards, int32_t n_traj,
+                                                          float* __restrict__ adv, float* __restrict__ ret,
+                                                          int32_t* status) {
+  for (int64_t t = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < T;
+       t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    float a = 0.f, g = 0.f;
+    if (mask[t] != 0) {
+      const int32_t i = token_traj[t];
+      if (i < 0 || i >= n_traj) {
+        flag_status(status, RL_DEV_BAD_TRAJ);
+      } else {
+        g = rewards[i];
+        a = g - values[t];
+      }
+    }
+    adv[t] = a;
+    if (ret) ret[t] = g;
+  }
+}
+
 static int grid_for(int64_t work, int per_block, int cap) {
   int64_t g = (work + per_block - 1) / per_block;
   if (g < 1) g = 1;
@@ -287,4 +314,25 @@ extern "C" rl_status rl_value_loss_fwd_bwd(int64_t rows, const float* values, co
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_error(e, "value_loss_kernel launch");
   return launch_reduce_loss(row_loss, rows, loss_accum, s);
+}
+
+extern "C" rl_status rl_rollout_value_advantages(int64_t n_tokens, const int32_t* token_traj, const uint8_t* mask,
+                                                 const float* values, const float* rewards, int32_t n_traj,
+                                                 float* adv_out, float* returns_out, void* ws, size_t ws_bytes,
+                                                 rl_stream_t stream) {
+  using namespace rl;
+  clear_error();
+  if (n_tokens < 0 || n_traj < 0) return set_error(RL_ERR_INVALID_ARG, "rl_rollout_value_advantages: negative size");
+  if (!ws) return set_error(RL_ERR_INVALID_ARG, "rl_rollout_value_advantages: NULL workspace");
+  if (ws_bytes < kWsHeader)
+    return set_error(RL_ERR_WORKSPACE_TOO_SMALL, "rl_rollout_value_advantages: workspace too small");
+  if (n_tokens == 0) return RL_OK;
+  if (!token_traj || !mask || !values || !adv_out || (n_traj > 0 && !rewards))
+    return set_error(RL_ERR_INVALID_ARG, "rl_rollout_value_advantages: NULL array argument");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  ppo::rollout_adv_kernel<<<ppo::grid_for(n_tokens, 256, 152 * 8), 256, 0, s>>>(
+      n_tokens, token_traj, mask, values, rewards, n_traj, adv_out, returns_out, reinterpret_cast<int32_t*>(ws));
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_error(e, "rollout_adv_kernel launch");
+  return RL_OK;
 }

@@ -13,6 +13,7 @@ from __future__ import annotations
 import ctypes
 import os
 
+import numpy as np
 import torch
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -41,6 +42,10 @@ EXPORTS = {
     "rl_policy_loss_fwd_bwd_noalloc": (_I32, [_P, _I32, _I64, _I64, _I64, _P, _P, _P, _I32, _P, _P, _P, _P, _P,
                                               _P, _P, _P, _P, _P, _P]),
     "rl_sequence_is_weights": (_I32, [_I32, _I64, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P, _SZ, _P]),
+    "rl_prefix_tree_build_batch": (_I32, [_I32, _P, _P, _P, _P, _P, _P, _P, _P, _I32, _I32, _I64, _P, _P, _P, _P,
+                                          _P, _P, _P, _P, _P, _P, _P, _P]),
+    "rl_group_advantages_by_owner": (_I32, [_I32, _I32, _P, _P, _P, _I64, _P, _P, _P, _P, _P, _P, _P, _SZ, _P]),
+    "rl_rollout_value_advantages": (_I32, [_I64, _P, _P, _P, _P, _I32, _P, _P, _P, _SZ, _P]),
     "rl_masked_gae": (_I32, [_I32, _P, _I64, _P, _P, _P, _P, _F, _F, _I32, _P, _P, _P, _SZ, _P]),
     "rl_value_loss_fwd_bwd": (_I32, [_I64, _P, _P, _P, _P, _I32, _P, _P, _P, _P, _SZ, _P]),
     "rl_fused_head_token_logprobs": (_I32, [_P, _P, _I64, _I64, _I64, _P, _P, _P, _P, _P, _SZ, _P]),
@@ -59,6 +64,11 @@ def make_params(clip_eps_low=0.2, clip_eps_high=0.28, kl_coef=0.0, kl_estimator=
                 tis_cap=0.0, adv_eps=1e-6, loss_agg=AGG_SEQ_MEAN_TOKEN_MEAN, token_level_adv=0) -> rl_loss_params:
     return rl_loss_params(clip_eps_low, clip_eps_high, kl_coef, kl_estimator, entropy_coef, tis_cap, adv_eps,
                           loss_agg, int(token_level_adv))
+
+
+class rl_tree_stats(ctypes.Structure):
+    _fields_ = [("valid", _I32), ("n_leaves", _I32), ("n_kept_leaves", _I32), ("n_unplaced", _I32),
+                ("n_tokens", _I64), ("n_trainable", _I64)]
 
 
 class RLError(RuntimeError):
@@ -431,3 +441,115 @@ def rl_sequence_is_weights(token_traj, mask, old_logp, rollout_logp, n_traj, ws,
                                       _ptr(token_adv_inout), _ptr(ws), ws.numel(), _stream(stream))
     _check("rl_sequence_is_weights", st)
     return weight_out, log_ratio_out
+
+
+def _np_ptr(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _csr(seqs, dtype, off_dtype=np.int64):
+    lens = np.fromiter((len(q) for q in seqs), dtype=np.int64, count=len(seqs))
+    offs = np.zeros(len(seqs) + 1, dtype=off_dtype)
+    np.cumsum(lens, out=offs[1:])
+    flat = np.concatenate([np.asarray(q, dtype=dtype) for q in seqs]) if len(seqs) and offs[-1] else \
+        np.zeros(1, dtype=dtype)
+    return offs, np.ascontiguousarray(flat)
+
+
+def rl_prefix_tree_build_batch(prompts, calls, aux=None, max_leaves=0, n_threads=None):
+    """Prefix trees of a batch of rollouts, packed (host arrays in, numpy arrays out).
+
+    prompts: one token sequence per rollout; calls: per rollout, a list of (x, y) token
+    sequences in capture order; aux: per rollout, a list of flags (or None). Returns a dict of
+    the packed per-token arrays (tokens, mask, parent, depth, owner, node_call), the kept
+    leaves (leaf_call, leaf_end, leaf_offsets), rollout_offsets and per-rollout stats."""
+    n = len(prompts)
+    if len(calls) != n:
+        raise ValueError("one list of calls per rollout")
+    p_off, p_tok = _csr(prompts, np.int32)
+    c_off = np.zeros(n + 1, dtype=np.int32)
+    np.cumsum([len(c) for c in calls], out=c_off[1:])
+    flat = [c for rc in calls for c in rc]
+    x_off, x_tok = _csr([c[0] for c in flat], np.int32)
+    y_off, y_tok = _csr([c[1] for c in flat], np.int32)
+    aux_arr = None
+    if aux is not None:
+        aux_arr = np.concatenate([np.asarray(a if a is not None else [0] * len(rc), dtype=np.uint8)
+                                  for a, rc in zip(aux, calls)]) if flat else np.zeros(1, np.uint8)
+    n_calls = len(flat)
+    threads = n_threads if n_threads is not None else min(16, os.cpu_count() or 1)
+    stats = (rl_tree_stats * max(n, 1))()
+    r_off = np.zeros(n + 1, dtype=np.int64)
+    l_off = np.zeros(n + 1, dtype=np.int64)
+    n_tok = ctypes.c_int64(0)
+    L = lib()
+    args = (n, _np_ptr(p_off), _np_ptr(p_tok), _np_ptr(c_off), _np_ptr(x_off), _np_ptr(x_tok), _np_ptr(y_off),
+            _np_ptr(y_tok), _np_ptr(aux_arr), int(max_leaves), int(threads))
+    st = L.rl_prefix_tree_build_batch(*args, 0, None, None, None, None, None, None, None, None, None, stats,
+                                      _np_ptr(r_off), ctypes.byref(n_tok))
+    if st not in (RL_OK, 4):
+        _check("rl_prefix_tree_build_batch", st)
+    T = n_tok.value
+    out = dict(tokens=np.empty(T, np.int32), mask=np.empty(T, np.uint8), parent=np.empty(T, np.int64),
+               depth=np.empty(T, np.int32), owner=np.empty(T, np.int32), node_call=np.empty(T, np.int32),
+               leaf_call=np.empty(max(n_calls, 1), np.int32), leaf_end=np.empty(max(n_calls, 1), np.int64))
+    st = L.rl_prefix_tree_build_batch(*args, T, *(_np_ptr(out[k]) for k in ("tokens", "mask", "parent", "depth",
+                                                                              "owner", "node_call", "leaf_call",
+                                                                              "leaf_end")),
+                                      _np_ptr(l_off), stats, _np_ptr(r_off), ctypes.byref(n_tok))
+    _check("rl_prefix_tree_build_batch", st)
+    out["leaf_call"] = out["leaf_call"][:l_off[-1]]
+    out["leaf_end"] = out["leaf_end"][:l_off[-1]]
+    out.update(leaf_offsets=l_off, rollout_offsets=r_off,
+               stats=[dict(valid=stats[r].valid, n_leaves=stats[r].n_leaves, n_kept_leaves=stats[r].n_kept_leaves,
+                           n_unplaced=stats[r].n_unplaced, n_tokens=stats[r].n_tokens,
+                           n_trainable=stats[r].n_trainable) for r in range(n)])
+    return out
+
+
+def rl_group_advantages_by_owner(group_offsets, rewards, token_traj, mask, params: rl_loss_params, ws,
+                                 traj_valid=None, adv_out=None, coef_out=None, n_tok_out=None, stream=None):
+    """rl_group_advantages with the owner of every token given (any token order)."""
+    n_traj = rewards.numel()
+    n_groups = group_offsets.numel() - 1
+    T = mask.numel()
+    dev = rewards.device
+    _need(group_offsets, "group_offsets", torch.int32, n_groups + 1, device=dev)
+    _need(rewards, "rewards", torch.float32, n_traj, device=dev)
+    _opt(traj_valid, "traj_valid", torch.uint8, n_traj, device=dev)
+    _need(token_traj, "token_traj", torch.int32, T, device=dev)
+    _need(mask, "mask", torch.uint8, T, device=dev)
+    adv_out = torch.empty(n_traj, dtype=torch.float32, device=dev) if adv_out is None else adv_out
+    coef_out = torch.empty(n_traj, dtype=torch.float32, device=dev) if coef_out is None else coef_out
+    n_tok_out = torch.empty(n_traj, dtype=torch.int32, device=dev) if n_tok_out is None else n_tok_out
+    _need(adv_out, "adv_out", torch.float32, n_traj, device=dev)
+    _need(coef_out, "coef_out", torch.float32, n_traj, device=dev)
+    _need(n_tok_out, "n_tok_out", torch.int32, n_traj, device=dev)
+    _need(ws, "ws", torch.uint8, device=dev)
+    st = lib().rl_group_advantages_by_owner(n_traj, n_groups, _ptr(group_offsets), _ptr(rewards), _ptr(traj_valid), T,
+                                            _ptr(token_traj), _ptr(mask), ctypes.byref(params), _ptr(adv_out),
+                                            _ptr(coef_out), _ptr(n_tok_out), _ptr(ws), ws.numel(), _stream(stream))
+    _check("rl_group_advantages_by_owner", st)
+    return adv_out, coef_out, n_tok_out
+
+
+def rl_rollout_value_advantages(token_traj, mask, values, rewards, ws, adv_out=None, returns_out=None,
+                                want_returns=True, stream=None):
+    """A_t = R_i - V_t, G_t = R_i on trainable tokens (Sec. 2.3.4), tokens in any order."""
+    T = mask.numel()
+    n_traj = rewards.numel()
+    dev = mask.device
+    _need(token_traj, "token_traj", torch.int32, T, device=dev)
+    _need(mask, "mask", torch.uint8, T, device=dev)
+    _need(values, "values", torch.float32, T, device=dev)
+    _need(rewards, "rewards", torch.float32, n_traj, device=dev)
+    adv_out = torch.empty(T, dtype=torch.float32, device=dev) if adv_out is None else adv_out
+    if want_returns and returns_out is None:
+        returns_out = torch.empty(T, dtype=torch.float32, device=dev)
+    _need(adv_out, "adv_out", torch.float32, T, device=dev)
+    _opt(returns_out, "returns_out", torch.float32, T, device=dev)
+    _need(ws, "ws", torch.uint8, device=dev)
+    st = lib().rl_rollout_value_advantages(T, _ptr(token_traj), _ptr(mask), _ptr(values), _ptr(rewards), n_traj,
+                                           _ptr(adv_out), _ptr(returns_out), _ptr(ws), ws.numel(), _stream(stream))
+    _check("rl_rollout_value_advantages", st)
+    return adv_out, returns_out

@@ -22,6 +22,9 @@ vocabulary):
   fusedhead  hidden bf16 [32,768 x 4,096] ~ N(0, 1), W bf16 [151,936 x 4,096] ~ N(0, 0.02^2),
              masks and rewards of the first 32,768 tokens of a multiturn batch
 
+  tree       16 tasks x 8 rollouts of captured model calls (prompt, turns with tool outputs,
+             retries, subagent and compaction calls), packed as deduplicated prefix trees
+
 For the PPO path, value predictions V(s_t) are N(0.3, 0.25^2) per token and the
 rollout reward R_i of the layout is placed at each trajectory's last trainable token;
 sparse per-token rewards can be added.
@@ -67,6 +70,7 @@ class Workload:
     equal_groups: int = 0      # groups forced to all-equal rewards (half 0, half 1)
     hidden: int = 0            # fused head only
     weight_std: float = 0.0    # fused head only
+    tree_max_leaves: int = 0   # prefix-tree workload only
     extra: dict = field(default_factory=dict)
 
 
@@ -80,10 +84,12 @@ WORKLOADS = {
     "edge": Workload("edge", 4096, 4, 32000, "f32", 2.0, 131072, ("fixed", 8), "edge", 0.5, 0.0),
     "fusedhead": Workload("fusedhead", 16, 8, 151936, "bf16", 0.0, 32768, ("uniform", 256, 2048),
                           "spans", 0.3, 0.1, hidden=4096, weight_std=0.02),
+    "tree": Workload("tree", 16, 8, 151936, "bf16", 2.0, 16384, ("calls", 4, 16), "tree", 0.3, 0.1,
+                     tree_max_leaves=12),
 }
 
 # the order in which the workloads are listed in the project's configuration
-WORKLOAD_ORDER = ["tiny", "multiturn", "longhorizon", "edge", "fusedhead"]
+WORKLOAD_ORDER = ["tiny", "multiturn", "longhorizon", "edge", "fusedhead", "tree"]
 
 
 def _rng(seed: int, *stream) -> np.random.Generator:
@@ -320,6 +326,56 @@ def rollout_logp_from(old_logp: np.ndarray, seed: int, std: float = 0.05, row0: 
     """Rollout-engine log-probs for TIS tests: old_logp + N(0, std^2)."""
     rng = _rng(seed, 99, 6, row0)
     return (np.asarray(old_logp, dtype=np.float64) + rng.normal(0.0, std, size=len(old_logp))).astype(np.float32)
+
+
+def tree_rollouts(w: Workload, seed: int = 0, n_rollouts: int | None = None):
+    """Captured model calls of black-box rollouts (Sec. 3.2.1), for the prefix-tree path.
+
+    Per rollout: a task prompt of U{200..800} tokens, then U{lo..hi} main-agent turns (the
+    workload's ``lengths`` = ("calls", lo, hi)); every turn after the first appends a tool
+    output of U{16..512} tokens to the history, and the model answers with U{16..384} tokens.
+    The input of each call is the whole history so far, as a serving proxy sees it. With
+    probability 0.1 a turn is first attempted and abandoned (a retry: same input, another
+    response that nothing continues); with probability 0.05 an auxiliary subagent call branches
+    off (history + an instruction of U{8..32} tokens, a response of U{16..128}); with
+    probability 0.06 the context is compacted: an auxiliary summariser call (history + an
+    instruction, a summary of U{64..256} tokens) and the history restarts as prompt + summary.
+    One rollout in 20 runs away with a retry on nearly every turn (more leaves than
+    ``tree_max_leaves``). Token ids are uniform on [0, vocab).
+
+    Returns (prompts, calls, aux): lists per rollout; calls are (x, y) int32 arrays."""
+    n = w.n_groups * w.group_size if n_rollouts is None else n_rollouts
+    lo, hi = w.lengths[1], w.lengths[2]
+    prompts, calls, aux = [], [], []
+    for r in range(n):
+        rng = _rng(seed, _name_id(w.name), 9, r)
+        tok = lambda k: rng.integers(0, w.vocab, int(k)).astype(np.int32)  # noqa: E731
+        prompt = tok(rng.integers(200, 801))
+        runaway = rng.random() < 0.05
+        p_retry = 0.9 if runaway else 0.1
+        hist = prompt
+        cs, ax = [], []
+        for turn in range(int(rng.integers(lo, hi + 1))):
+            x = hist if turn == 0 else np.concatenate([hist, tok(rng.integers(16, 513))])
+            if rng.random() < p_retry:
+                cs.append((x, tok(rng.integers(16, 385))))
+                ax.append(0)
+            y = tok(rng.integers(16, 385))
+            cs.append((x, y))
+            ax.append(0)
+            hist = np.concatenate([x, y])
+            if rng.random() < 0.05:
+                cs.append((np.concatenate([hist, tok(rng.integers(8, 33))]), tok(rng.integers(16, 129))))
+                ax.append(1)
+            if rng.random() < 0.06:
+                summary = tok(rng.integers(64, 257))
+                cs.append((np.concatenate([hist, tok(rng.integers(8, 33))]), summary))
+                ax.append(1)
+                hist = np.concatenate([prompt, summary])
+        prompts.append(prompt)
+        calls.append(cs)
+        aux.append(ax)
+    return prompts, calls, aux
 
 
 def value_predictions(w: Workload, seed: int, n_tokens: int, mean: float = 0.3, std: float = 0.25) -> np.ndarray:

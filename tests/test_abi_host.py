@@ -235,3 +235,25 @@ def test_sequence_is_weights_argument_checks(R):
     assert call(w=None) == 1
     assert call(roll=None) == 1
     assert call(n=0) == 0
+
+
+def test_owner_and_tree_argument_checks(R):
+    L = R.lib()
+    p = _params(R)
+    assert L.rl_group_advantages_by_owner(-1, 0, None, FAKE, None, 10, FAKE, FAKE, p, FAKE, FAKE, FAKE, FAKE, 1024,
+                                          None) == 1
+    assert L.rl_group_advantages_by_owner(4, 1, FAKE, FAKE, None, 10, None, FAKE, p, FAKE, FAKE, FAKE, FAKE, 1024,
+                                          None) == 1
+    assert L.rl_group_advantages_by_owner(4, 1, FAKE, FAKE, None, 10, FAKE, FAKE, p, FAKE, FAKE, FAKE, FAKE, 16,
+                                          None) == 4
+    assert L.rl_rollout_value_advantages(-1, FAKE, FAKE, FAKE, FAKE, 2, FAKE, None, FAKE, 1024, None) == 1
+    assert L.rl_rollout_value_advantages(10, FAKE, FAKE, FAKE, None, 2, FAKE, None, FAKE, 1024, None) == 1
+    n_tok = ctypes.c_int64(0)
+    assert L.rl_prefix_tree_build_batch(-1, *([None] * 8), 0, 1, 0, *([None] * 11), ctypes.byref(n_tok)) == 1
+    import numpy as np
+    bad = np.array([0, 3, 1], np.int64)  # decreasing offsets
+    co = np.array([0, 0, 0], np.int32)
+    ptr = lambda a: a.ctypes.data_as(ctypes.c_void_p)  # noqa: E731
+    assert L.rl_prefix_tree_build_batch(2, ptr(bad), ptr(np.zeros(4, np.int32)), ptr(co), ptr(np.zeros(1, np.int64)),
+                                        None, ptr(np.zeros(1, np.int64)), None, None, 0, 1, 0,
+                                        *([None] * 11), ctypes.byref(n_tok)) == 1
