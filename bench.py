@@ -658,9 +658,9 @@ def time_head(torch, R, dev, warmup=2, reps=5):
                         f"masks and coefficients of the first {hb.T} multiturn tokens ({hb.trained} trained)",
             "ms_per_call": ms, "tokens_per_s": hb.T / (ms * 1e-3), "bound": "tensor", "achieved": tf,
             "peak": burst, "unit": "TFLOP/s", "frac": tf / burst, "frac_of_sustained": tf / sustained,
-            "peak_source": kind, "algorithmic_flops_per_call": flops, "executed_flops_per_call": 8.0 * hb.T * hb.D * hb.V,
+            "peak_source": kind, "algorithmic_flops_per_call": flops, "executed_flops_per_call": flops,
             "reps": reps, "chunks_per_call": chunks,
-            "note": "algorithmic 6 T D V (Z, dH, dW); executed 8 T D V (Z is computed twice); dH and dW through cuBLASLt",
+            "note": "6 T D V (Z once, dH, dW); dH and dW through cuBLASLt",
             "logprobs": fwd}
 
 

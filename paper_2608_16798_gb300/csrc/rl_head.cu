@@ -2,16 +2,20 @@
 // and the output projection, with the logits Z = H W^T never written to memory.
 //
 // For each chunk of tokens:
-//   1. head_kernel<STATS>  tcgen05 GEMM tiles Z[128 x 256] = H W^T (TMA-fed shared-memory
+//   1. head_kernel<STATS_P> tcgen05 GEMM tiles Z[128 x 256] = H W^T (TMA-fed shared-memory
 //      stages, fp32 accumulators in TMEM, two accumulators so the epilogue of one tile
-//      overlaps the MMAs of the next); the epilogue folds every tile into per-row
-//      online-softmax partials for its vocabulary block.
-//   2. head_merge_kernel   one thread per token: merges the partials into lse, entropy and
+//      overlaps the MMAs of the next). The epilogue reads each tile twice from TMEM: first
+//      its row maximum m_j, then e = exp(z - m_j), which it stores (bf16) in the chunk's
+//      dZ buffer, with m_j per token and tile, and folds into per-row online-softmax
+//      partials for its vocabulary block.
+//   2. head_merge_kernel    one thread per token: merges the partials into lse, entropy and
 //      logp, evaluates the objective's per-token terms (same readings as the logits path),
 //      writes the row's loss contribution and the coefficients of dZ.
-//   3. head_kernel<DZ>     recomputes the same Z tiles; the epilogue forms
-//      dZ = c [g (delta_a - p) + alpha p (log p + H)] and stores it (bf16) for this chunk.
+//   3. head_dz_kernel       rescales the stored e in place into
+//      dZ = c [g (delta_a - p) + alpha p (log p + H)], p = e exp(m_j - lse) (HBM-bound: the
+//      logits are formed once, not twice).
 //   4. dH = dZ W and dW += dZ^T H, two plain GEMMs through cuBLASLt.
+// The forward-only call runs head_kernel<STATS> (no stores) and head_logp_merge_kernel.
 // The objective (Sec. 2.3.2, Sec. 3.2.4) is the same as for rl_policy_loss_fwd_bwd; here
 // pi_theta's logits come from the hidden states times the vocabulary projection.
 #include <cublasLt.h>
@@ -40,7 +44,7 @@ constexpr size_t kSmem = NS * STAGE_BYTES + 1024;
 constexpr int64_t kChunk = 8192;   // tokens per chunk
 constexpr size_t kLtWorkspace = 32u << 20;
 
-enum Mode { STATS = 0, DZ = 1 };
+enum Mode { STATS = 0, STATS_P = 1 };
 
 // Per-token coefficients of dZ (from head_merge_kernel).
 struct RowCoef {
@@ -60,9 +64,9 @@ struct HeadArgs {
   int32_t ent;
   const int32_t* token_ids;
   float4* partials;        // [n_vb][Tc] (m, s, u, z_a)
-  const RowCoef* rc;       // [Tc]
-  uint16_t* dz;            // [Tc x ldz] bf16
+  uint16_t* dz;            // [Tc x ldz] bf16: e = exp(z - m_j) (STATS_P)
   int64_t ldz;
+  float* tmax;             // [Tc x n_nt]: m_j per token and tile (STATS_P)
   int32_t* status;
 };
 
@@ -161,6 +165,7 @@ __global__ void __launch_bounds__(kThreads, 1) head_kernel(const __grid_constant
     // ---------------------------------------------------------------- epilogue (4 warps)
     const int q = warp & 3;  // TMEM lane quarter this warp may access
     const int rl = 32 * q + lane;
+    const float kNegInf = -__int_as_float(0x7f800000);
     uint32_t t = 0;
     bool ok = true;
     for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
@@ -168,16 +173,9 @@ __global__ void __launch_bounds__(kThreads, 1) head_kernel(const __grid_constant
       const int r = m0 + rl;  // token within the chunk
       const bool row_ok = r < p.Tc;
       const int nt1 = min((vb + 1) * VB_TILES, p.n_nt);
-      SoftmaxPartial ps{-__int_as_float(0x7f800000), 0.f, 0.f};
+      SoftmaxPartial ps{kNegInf, 0.f, 0.f};
       float za = 0.f;
-      int32_t a = -1;
-      RowCoef rc = {};
-      if (MODE == STATS) {
-        if (row_ok) a = p.token_ids[p.t0 + r];
-      } else {
-        if (row_ok) rc = p.rc[r];
-        a = rc.a;
-      }
+      const int32_t a = row_ok ? p.token_ids[p.t0 + r] : -1;
       for (int nt = vb * VB_TILES; nt < nt1; ++nt, ++t) {
         const int acc = t & 1;
         if (!mbar_wait_bounded(&accf[acc], (t >> 1) & 1)) {
@@ -187,64 +185,53 @@ __global__ void __launch_bounds__(kThreads, 1) head_kernel(const __grid_constant
         }
         tc::fence_after_sync();
         const int n0 = nt * BN;
+        const uint32_t tbase_acc = tmem + (static_cast<uint32_t>(32 * q) << 16) + acc * BN;
+        // sweep 1: the tile's row maximum and the sampled id's logit
+        float tm = kNegInf;
 #pragma unroll 1
         for (int c = 0; c < BN; c += 32) {
-          float v[32];
-          tc::tmem_ld32(tmem + (static_cast<uint32_t>(32 * q) << 16) + acc * BN + c, v);
           const int col0 = n0 + c;
           const int nvalid = min(32, p.V - col0);
-          if (nvalid <= 0) continue;  // past the vocabulary (uniform across the warp)
-          if (MODE == STATS) {
-            float vm = -__int_as_float(0x7f800000);
+          if (nvalid <= 0) break;  // past the vocabulary (uniform across the warp)
+          float v[32];
+          tc::tmem_ld32(tbase_acc + c, v);
 #pragma unroll
-            for (int j = 0; j < 32; ++j) {
-              if (j >= nvalid) v[j] = -1e30f;  // contributes exp(...) = 0
-              vm = fmaxf(vm, v[j]);
-            }
-            if (vm > ps.m) {
-              const float dd = ps.m - vm;
-              const float sc = ex2(dd * kLog2e);
-              ps.u = (ps.s == 0.f) ? 0.f : sc * fmaf(dd, ps.s, ps.u);
-              ps.s *= sc;
-              ps.m = vm;
-            }
-            const float nm = -ps.m * kLog2e;
-            float s0 = 0.f, s1 = 0.f, u0 = 0.f;
+          for (int j = 0; j < 32; ++j)
+            if (j < nvalid) tm = fmaxf(tm, v[j]);
+          const int ja = a - col0;
+          if (ja >= 0 && ja < 32) {
 #pragma unroll
-            for (int j = 0; j < 32; ++j) {
-              const float e = ex2(fmaf(v[j], kLog2e, nm));
-              if (j & 1) s1 += e; else s0 += e;
-              if (p.ent) u0 = fmaf(e, v[j] - ps.m, u0);
-            }
-            ps.s += s0 + s1;
-            ps.u += u0;
-            const int ja = a - col0;
-            if (ja >= 0 && ja < 32) {
+            for (int j = 0; j < 32; ++j)
+              if (j == ja) za = v[j];
+          }
+        }
+        // sweep 2: e = exp(z - m_j), its sums, and (STATS_P) e stored in bf16
+        const float nm = -tm * kLog2e;
+        float s0 = 0.f, s1 = 0.f, u0 = 0.f;
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+          const int col0 = n0 + c;
+          const int nvalid = min(32, p.V - col0);
+          if (nvalid <= 0) break;
+          float v[32];
+          tc::tmem_ld32(tbase_acc + c, v);
+          uint32_t w[16];
 #pragma unroll
-              for (int j = 0; j < 32; ++j)
-                if (j == ja) za = v[j];
+          for (int j = 0; j < 32; j += 2) {
+            float e2[2];
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              const bool in = j + h < nvalid;
+              const float z = in ? v[j + h] : tm;
+              const float e = in ? ex2(fmaf(z, kLog2e, nm)) : 0.f;
+              if (h) s1 += e; else s0 += e;
+              if (p.ent) u0 = fmaf(e, z - tm, u0);
+              e2[h] = e;
             }
-          } else if (row_ok) {
+            w[j / 2] = pack_bf16x2(e2[0], e2[1]);
+          }
+          if (MODE == STATS_P && row_ok) {
             uint16_t* out = p.dz + static_cast<int64_t>(r) * p.ldz + col0;
-            uint32_t w[16];
-            if (rc.active) {
-#pragma unroll
-              for (int j = 0; j < 32; j += 2) {
-                float o[2];
-#pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                  const float z = v[j + h];
-                  const float pk = ex2(fmaf(z, kLog2e, rc.nlse2));
-                  float x = p.ent ? pk * fmaf(rc.ca, z, rc.Ke) : rc.Kp * pk;
-                  if (col0 + j + h == a) x += rc.cg;
-                  o[h] = x;
-                }
-                w[j / 2] = pack_bf16x2(o[0], o[1]);
-              }
-            } else {
-#pragma unroll
-              for (int j = 0; j < 16; ++j) w[j] = 0u;
-            }
             if (nvalid == 32) {
 #pragma unroll
               for (int j = 0; j < 4; ++j)
@@ -259,9 +246,10 @@ __global__ void __launch_bounds__(kThreads, 1) head_kernel(const __grid_constant
         tc::fence_before_sync();
         __syncwarp();
         if (lane == 0) mbar_arrive(&acce[acc]);
+        if (MODE == STATS_P && row_ok) p.tmax[static_cast<int64_t>(r) * p.n_nt + nt] = tm;
+        ps = merge(ps, SoftmaxPartial{tm, s0 + s1, u0});
       }
-      if (MODE == STATS && ok && row_ok)
-        p.partials[static_cast<int64_t>(vb) * p.Tc + r] = make_float4(ps.m, ps.s, ps.u, za);
+      if (ok && row_ok) p.partials[static_cast<int64_t>(vb) * p.Tc + r] = make_float4(ps.m, ps.s, ps.u, za);
     }
   }
   tc::fence_before_sync();
@@ -365,6 +353,76 @@ __global__ void __launch_bounds__(256) head_merge_kernel(const MergeArgs p) {
   }
 }
 
+struct DzArgs {
+  int32_t Tc, V, n_nt;
+  int32_t ent;
+  const RowCoef* rc;
+  uint16_t* dz;       // in: e = exp(z - m_j) (bf16); out: dZ (bf16)
+  int64_t ldz;
+  const float* tmax;  // [Tc x n_nt]
+};
+
+constexpr int kDzThreads = 256;
+constexpr int kMaxTilesSmem = 2048;  // V up to 524,288 keeps the row's tile factors in shared memory
+
+// One CTA per token row of the chunk (grid-stride): p_v = e_v exp(m_j - lse), then
+// dZ_v = Kp p_v (+ cg at v = a), or with the entropy bonus p_v (ca z_v + Ke) (+ cg at v = a),
+// z_v = m_j + ln e_v. Rows that are not trained on become zeros. 16-byte loads and stores.
+__global__ void __launch_bounds__(kDzThreads) head_dz_kernel(const DzArgs p) {
+  __shared__ float fac[kMaxTilesSmem], zoff[kMaxTilesSmem];
+  for (int r = blockIdx.x; r < p.Tc; r += gridDim.x) {
+    const RowCoef rc = p.rc[r];
+    uint16_t* row = p.dz + static_cast<int64_t>(r) * p.ldz;
+    const int nvec = p.V / 8;
+    if (!rc.active) {
+      for (int k = threadIdx.x; k < nvec; k += kDzThreads) reinterpret_cast<uint4*>(row)[k] = make_uint4(0, 0, 0, 0);
+      for (int v = nvec * 8 + threadIdx.x; v < p.V; v += kDzThreads) row[v] = 0;
+      continue;
+    }
+    // per tile: Kp exp(m_j - lse) (no entropy) or exp(m_j - lse) and m_j (entropy)
+    for (int j = threadIdx.x; j < p.n_nt; j += kDzThreads) {
+      const float m = p.tmax[static_cast<int64_t>(r) * p.n_nt + j];
+      const float f = ex2(fmaf(m, kLog2e, rc.nlse2));
+      fac[j] = p.ent ? f : rc.Kp * f;
+      zoff[j] = fmaf(rc.ca, m, rc.Ke);  // ca m_j + Ke
+    }
+    __syncthreads();
+    for (int k = threadIdx.x; k < nvec; k += kDzThreads) {
+      uint4 w = reinterpret_cast<const uint4*>(row)[k];
+      const int j = (k * 8) / BN;
+      const float f = fac[j];
+      uint32_t* wp = reinterpret_cast<uint32_t*>(&w);
+#pragma unroll
+      for (int h = 0; h < 4; ++h) {
+        float o[2];
+#pragma unroll
+        for (int b = 0; b < 2; ++b) {
+          const float e = b ? bf16_hi(wp[h]) : bf16_lo(wp[h]);
+          float x;
+          if (p.ent) {
+            // p (ca z + Ke) with z = m_j + ln e; e = 0 contributes 0
+            x = e > 0.f ? f * e * fmaf(rc.ca, __logf(e), zoff[j]) : 0.f;
+          } else {
+            x = f * e;
+          }
+          if (k * 8 + 2 * h + b == rc.a) x += rc.cg;
+          o[b] = x;
+        }
+        wp[h] = pack_bf16x2(o[0], o[1]);
+      }
+      reinterpret_cast<uint4*>(row)[k] = w;
+    }
+    for (int v = nvec * 8 + threadIdx.x; v < p.V; v += kDzThreads) {
+      const int j = v / BN;
+      const float e = bf16_to_f32(row[v]);
+      float x = p.ent ? (e > 0.f ? fac[j] * e * fmaf(rc.ca, __logf(e), zoff[j]) : 0.f) : fac[j] * e;
+      if (v == rc.a) x += rc.cg;
+      row[v] = f32_to_bf16(x);
+    }
+    __syncthreads();  // fac / zoff are rewritten for the next row
+  }
+}
+
 struct LogpMergeArgs {
   int64_t t0;
   int32_t Tc, V, n_vb;
@@ -437,8 +495,8 @@ static rl_status make_map(CUtensorMap* m, const void* base, int64_t inner, int64
 }
 
 struct Layout {
-  int64_t Tc, n_vb, ldz;
-  size_t off_partials, off_rc, off_dz, off_lt, total;
+  int64_t Tc, n_nt, n_vb, ldz;
+  size_t off_partials, off_rc, off_tmax, off_dz, off_lt, total;
 };
 
 static size_t al256(size_t x) { return (x + 255) & ~size_t(255); }
@@ -447,6 +505,7 @@ static Layout layout(int64_t max_rows, int64_t V) {
   Layout L;
   L.Tc = std::max<int64_t>(1, std::min<int64_t>(max_rows, kChunk));
   const int64_t n_nt = (V + BN - 1) / BN;
+  L.n_nt = n_nt;
   L.n_vb = (n_nt + VB_TILES - 1) / VB_TILES;
   L.ldz = (V + 7) / 8 * 8;
   auto al = al256;
@@ -455,6 +514,8 @@ static Layout layout(int64_t max_rows, int64_t V) {
   off += al(static_cast<size_t>(L.n_vb * L.Tc) * sizeof(float4));
   L.off_rc = off;
   off += al(static_cast<size_t>(L.Tc) * sizeof(RowCoef));
+  L.off_tmax = off;
+  off += al(static_cast<size_t>(L.Tc * n_nt) * sizeof(float));
   L.off_dz = off;
   off += al(static_cast<size_t>(L.Tc * L.ldz) * 2);
   L.off_lt = off;
@@ -566,8 +627,8 @@ extern "C" rl_status rl_fused_head_loss_fwd_bwd(
   if (T < 0 || D < 64 || V < 1 || n_traj < 0)
     return set_error(RL_ERR_INVALID_ARG, "rl_fused_head_loss_fwd_bwd: need T >= 0, D >= 64, V >= 1, n_traj >= 0");
   if (D % 64 != 0) return set_error(RL_ERR_UNSUPPORTED, "rl_fused_head_loss_fwd_bwd: D must be a multiple of 64");
-  if (T > INT32_MAX || V > INT32_MAX || D > 65536)
-    return set_error(RL_ERR_UNSUPPORTED, "rl_fused_head_loss_fwd_bwd: T or V above 2^31 - 1, or D above 65536");
+  if (T > INT32_MAX || V > static_cast<int64_t>(kMaxTilesSmem) * BN || D > 65536)
+    return set_error(RL_ERR_UNSUPPORTED, "rl_fused_head_loss_fwd_bwd: T above 2^31 - 1, V above 524,288 or D above 65536");
   if (!params || !loss_accum || !ws) return set_error(RL_ERR_INVALID_ARG, "rl_fused_head_loss_fwd_bwd: NULL argument");
   if (d_hidden_dtype != RL_BF16 && d_hidden_dtype != RL_F32)
     return set_error(RL_ERR_INVALID_ARG, "rl_fused_head_loss_fwd_bwd: unknown d_hidden dtype");
@@ -593,6 +654,7 @@ extern "C" rl_status rl_fused_head_loss_fwd_bwd(
   double* row_loss = reinterpret_cast<double*>(wsb + ws_row_loss_offset());
   float4* partials = reinterpret_cast<float4*>(wsb + L.off_partials);
   RowCoef* rcs = reinterpret_cast<RowCoef*>(wsb + L.off_rc);
+  float* tmax = reinterpret_cast<float*>(wsb + L.off_tmax);
   uint16_t* dz = reinterpret_cast<uint16_t*>(wsb + L.off_dz);
   void* lt_ws = wsb + L.off_lt;
   cublasLtHandle_t lt;
@@ -622,11 +684,11 @@ extern "C" rl_status rl_fused_head_loss_fwd_bwd(
     ha.ent = ent ? 1 : 0;
     ha.token_ids = token_ids;
     ha.partials = partials;
-    ha.rc = rcs;
     ha.dz = dz;
     ha.ldz = L.ldz;
+    ha.tmax = tmax;
     ha.status = status;
-    st = launch_head<STATS>(mh, mw, ha, s);
+    st = launch_head<STATS_P>(mh, mw, ha, s);
     if (st != RL_OK) return st;
 
     MergeArgs ma = {};
@@ -658,8 +720,18 @@ extern "C" rl_status rl_fused_head_loss_fwd_bwd(
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_error(e, "head_merge_kernel launch");
 
-    st = launch_head<DZ>(mh, mw, ha, s);
-    if (st != RL_OK) return st;
+    DzArgs da = {};
+    da.Tc = Tc;
+    da.V = static_cast<int>(V);
+    da.n_nt = n_nt;
+    da.ent = ent && params->entropy_coef != 0.f ? 1 : 0;
+    da.rc = rcs;
+    da.dz = dz;
+    da.ldz = L.ldz;
+    da.tmax = tmax;
+    head_dz_kernel<<<std::min(Tc, 148 * 16), kDzThreads, 0, s>>>(da);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_error(e, "head_dz_kernel launch");
 
     // dH[t0 : t0 + Tc] = dZ W    (column-major: dH^T [D x Tc] = W^T [D x V] dZ^T [V x Tc])
     void* dh = static_cast<char*>(d_hidden) + t0 * D * (d_hidden_dtype == RL_BF16 ? 2 : 4);

@@ -1,11 +1,15 @@
 """Fused LM head (logits = hidden @ W^T never materialised) against the float64 oracle.
 
-The library rounds the logits' gradient dZ to bf16 before the two products
-dH = dZ W and dW = dZ^T H, so their elements carry independent rounding errors of at
-most 2^-9 relative per term: the bound used is 6 * 2^-9 * sqrt(sum of squared terms)
-(computed exactly in float64) plus 1e-4 of the element and 1e-6 of the largest
-element for the float32 parts. Loss, clip flags and per-token statistics use the
-logits-path tolerances.
+The library keeps exp(z - m_j) of each 256-wide tile in bf16 between its tensor-core pass
+and the formation of dZ, and rounds dZ itself to bf16 before the two products dH = dZ W and
+dW = dZ^T H: each term of those products carries two independent roundings of at most 2^-8
+relative (bf16's unit roundoff; plus, with the entropy bonus, alpha c p 2^-8 from the
+logarithm of the rounded value). Rounding errors of independent terms add like a random
+walk (standard deviation about 2^-7 / sqrt(3) of the root of the summed squared terms), so
+the bound used is 2^-6 * sqrt(sum of squared terms) (computed exactly in float64), about 3.5
+standard deviations, plus 1e-4 of the element and 1e-6 of the largest element for the
+float32 parts; a bf16 d_hidden adds its own rounding, 2^-8 of the element. Loss, clip flags
+and per-token statistics use the logits-path tolerances.
 """
 
 import dataclasses
@@ -83,7 +87,8 @@ def run_head(R, c, dh_dtype=torch.float32):
 
 
 def check_product(got, ref, S, what):
-    tol = 6 * 2.0 ** -9 * S + 1e-4 * np.abs(ref) + 1e-6 * np.abs(ref).max() + 1e-30
+    tol = 2.0 ** -6 * S + 1e-4 * np.abs(ref) + 1e-6 * np.abs(ref).max() + 1e-30
+    print(f"{what}: max error / bound = {float((np.abs(got - ref) / tol).max()):.3f}")
     bad = np.abs(got - ref) > tol
     if bad.any():
         i, j = np.argwhere(bad)[0]
@@ -107,7 +112,7 @@ def compare_head(c, out, dh_bf16=False):
     S_h = np.sqrt((dZ ** 2) @ (Wm ** 2))
     S_w = np.sqrt((dZ.T ** 2) @ (Hm ** 2))
     if dh_bf16:
-        S_h = S_h + 2.0 ** 8 * np.abs(dH) / 6  # plus half an ulp of the bf16 output
+        S_h = S_h + np.abs(dH) / 4  # 2^-6 |dH| / 4 = 2^-8 |dH|: the bf16 output's rounding
     check_product(out["dH"], dH, S_h, "d_hidden")
     check_product(out["dW"], dW, S_w, "d_weight")
     assert np.all(out["dH"][~active] == 0.0), "tokens that are not trained on must get zero d_hidden rows"
