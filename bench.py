@@ -181,6 +181,34 @@ class DeviceBatch:
         return 2 + 2 * len(self.mbs)
 
 
+def time_logits_extras(torch, R, batch, dev, peak, reps=20):
+    """Forward-only log-probs over the batch's microbatches (the pi_old / pi_ref recompute; one
+    read of each logits row, V x 2 bytes), with and without the entropy, and the advantages
+    alone (CUDA-graph replays)."""
+    t = torch
+    logp = t.empty(batch.T, dtype=t.float32, device=dev)
+    ent = t.empty_like(logp)
+    out = {}
+    for name, want_ent in (("token_logprobs", False), ("token_logprobs_entropy", True)):
+        def run():
+            for lo, hi in batch.mbs:
+                R.rl_token_logprobs(batch.logits[lo:hi], batch.ids[lo:hi], batch.ws, logp_out=logp[lo:hi],
+                                    entropy_out=ent[lo:hi] if want_ent else None)
+        ms = _time_calls(torch, run, 3, reps)
+        gbs = batch.T * batch.V * 2 / (ms * 1e-3) / 1e9
+        out[name] = {"ms_per_batch": ms, "tokens_per_s": batch.T / (ms * 1e-3), "achieved_gbs": gbs,
+                     "frac": gbs / peak, "frac_of_nominal_8tbs": gbs / 8000.0,
+                     "algorithmic_bytes_per_token": batch.V * 2}
+    params = R.make_params(W.CLIP_EPS_LOW, W.CLIP_EPS_HIGH, 0.0, 0, 0.0, 0.0, 1e-6, 0)
+    ms_adv = _time_graph(torch, lambda: R.rl_group_advantages(batch.group_offsets, batch.rewards, batch.traj_offsets,
+                                                              batch.mask, params, batch.ws, traj_valid=batch.valid,
+                                                              adv_out=batch.adv, coef_out=batch.coef,
+                                                              n_tok_out=batch.n_tok, token_traj_out=batch.token_traj),
+                         50)
+    out["group_advantages_us"] = ms_adv * 1e3
+    return out
+
+
 def time_ppo(torch, R, batch, dev, warmup=3, reps=20):
     """PPO step on the same batch (Sec. 2.3.1, Sec. 2.3.4): token-mean coefficients, masked GAE over
     the whole batch (skip reading, gamma = lambda = 1, R_i at each trajectory's last trainable token,
@@ -808,7 +836,17 @@ def main():
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                 "traffic": profiled_traffic(), "peak_source": peak_kind,
                 "kernel": "rows_kernel<bf16> via rl_policy_loss_fwd_bwd (+ 1-CTA loss reduction)",
-                "algorithmic_bytes_per_launch": per_launch_bytes, "avg_launch_ms": avg_launch_ms}
+                "algorithmic_bytes_per_launch": per_launch_bytes, "avg_launch_ms": avg_launch_ms,
+                "frac_of_nominal_8tbs": achieved / 8000.0}
+    # per microbatch: median and best launch over the timed steps, and each one's GB/s
+    per_mb = []
+    for k in range(n_mb):
+        ts = [kern_ms[s * n_mb + k] for s in range(args.steps)]
+        per_mb.append({"rows": batch.mbs[k][1] - batch.mbs[k][0], "median_ms": statistics.median(ts),
+                       "best_ms": min(ts), "median_gbs": batch.mb_bytes[k] / (statistics.median(ts) * 1e-3) / 1e9})
+    extras = time_logits_extras(torch, R, batch, dev, peak)
+    extras["loss_microbatches"] = per_mb
+    extras["loss_batch_sum_ms"] = sum(m["median_ms"] for m in per_mb)
 
     e2e = None
     if not args.no_e2e:
@@ -831,7 +869,7 @@ def main():
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": "f32", "data": "synthetic", "config": workload_config(batch.T, n_mb),
-                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks, "fused_head": head, "ppo": ppo, "tree": tree,
+                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks, "logits_path": extras, "fused_head": head, "ppo": ppo, "tree": tree,
                 "gpu_launches": batch.launches_per_step() * args.steps,
                 "loss_per_step": float(batch.loss.item()) / (args.warmup + args.steps)}
         print(json.dumps(line))
