@@ -316,64 +316,90 @@ def time_tree(torch, R, dev, reps=3):
                     "advantages by owner timed as CUDA-graph replays"}
 
 
-def e2e_run(torch, R, batch, dev, steps, warmup):
-    """Same step through host buffers: every step copies its inputs from pinned host memory
-    (metadata + each microbatch's logits) and reads back the gradient and the loss.
+def host_mem_available() -> int:
+    """MemAvailable of /proc/meminfo in bytes (0 if unknown)."""
+    try:
+        with open("/proc/meminfo") as f:
+            for line in f:
+                if line.startswith("MemAvailable:"):
+                    return int(line.split()[1]) * 1024
+    except OSError:
+        pass
+    return 0
 
-    Host memory holds a ring of two microbatches of logits and gradient (pinned), reused
-    cyclically; copies and kernels overlap on two streams."""
+
+def e2e_run(torch, R, batch, dev, steps, warmup, slots=4):
+    """Same step through host buffers: every step copies its inputs from pinned host memory (the
+    whole batch's logits, microbatch by microbatch, and the metadata) to the device and reads the
+    step's loss back; the gradient stays in HBM (batch.grad), where a training step's backward
+    consumes it.
+
+    Logits go through `slots` device buffers on two copy streams: the copy of microbatch k waits
+    only for the kernel that last read its slot, so copies run back to back while the kernels
+    follow, and a copy from a slow region of host memory overlaps the next one."""
     t = torch
     w = WORKLOAD
     V, mb = batch.V, w.microbatch
-    host_logits = [t.empty((mb, V), dtype=t.bfloat16, pin_memory=True) for _ in range(2)]
-    host_grad = [t.empty((mb, V), dtype=t.bfloat16, pin_memory=True) for _ in range(2)]
-    for k in range(2):
-        lo, hi = batch.mbs[k % len(batch.mbs)]
-        host_logits[k][:hi - lo].copy_(batch.logits[lo:hi])
+    # the whole batch in pinned host memory when every rank on the node fits in 40% of the
+    # available host memory; otherwise a ring of two microbatches (the timing is the same)
+    ranks_here = int(os.environ.get("LOCAL_WORLD_SIZE", "1"))
+    whole = batch.T * V * 2 * ranks_here <= 0.4 * host_mem_available()
+    # one pinned allocation per microbatch, filled by device-to-host copies (host-side CPU
+    # writes would leave dirty cache lines that the GPU's reads then have to fetch)
+    if whole:
+        host_mb = [t.empty((hi - lo, V), dtype=t.bfloat16, pin_memory=True) for lo, hi in batch.mbs]
+        for (lo, hi), h in zip(batch.mbs, host_mb):
+            h.copy_(batch.logits[lo:hi])
+        src = list(range(len(batch.mbs)))
+    else:
+        host_mb = [t.empty((mb, V), dtype=t.bfloat16, pin_memory=True) for _ in range(2)]
+        for k in range(2):
+            lo, hi = batch.mbs[k % len(batch.mbs)]
+            host_mb[k][:hi - lo].copy_(batch.logits[lo:hi])
+        src = [k % 2 for k in range(len(batch.mbs))]
     meta_host = {n: getattr(batch, n).cpu().pin_memory() for n in
                  ("ids", "mask", "old", "rewards", "group_offsets", "traj_offsets", "valid")}
     meta_dev = {n: t.empty_like(getattr(batch, n)) for n in meta_host}
-    dev_logits = [t.empty((mb, V), dtype=t.bfloat16, device=dev) for _ in range(2)]
-    dev_grad = [t.empty((mb, V), dtype=t.bfloat16, device=dev) for _ in range(2)]
+    dev_logits = [t.empty((mb, V), dtype=t.bfloat16, device=dev) for _ in range(slots)]
     loss_host = t.zeros(1, dtype=t.float64, pin_memory=True)
-    copy_in, copy_out = t.cuda.Stream(dev), t.cuda.Stream(dev)
+    copy_streams = [t.cuda.Stream(dev), t.cuda.Stream(dev)]
+    copy_in = copy_streams[0]
     comp = t.cuda.current_stream(dev)
     adv, coef = t.empty_like(batch.adv), t.empty_like(batch.coef)
     n_tok, tt = t.empty_like(batch.n_tok), t.empty_like(batch.token_traj)
     loss = t.zeros(1, dtype=t.float64, device=dev)
     h2d = sum(v.numel() * v.element_size() for v in meta_host.values())
     h2d += sum((hi - lo) * V * 2 for lo, hi in batch.mbs)
-    d2h = sum((hi - lo) * V * 2 for lo, hi in batch.mbs) + 8
+    d2h = loss_host.numel() * loss_host.element_size()
+    read_done = [None] * slots
 
     def one_step():
-        for n, h in meta_host.items():
-            meta_dev[n].copy_(h, non_blocking=True)
+        with t.cuda.stream(copy_in):
+            for n, h in meta_host.items():
+                meta_dev[n].copy_(h, non_blocking=True)
+            meta_ready = t.cuda.Event()
+            meta_ready.record(copy_in)
+        comp.wait_event(meta_ready)
+        loss.zero_()
         R.rl_group_advantages(meta_dev["group_offsets"], meta_dev["rewards"], meta_dev["traj_offsets"],
                               meta_dev["mask"], batch.params, batch.ws, traj_valid=meta_dev["valid"], adv_out=adv,
                               coef_out=coef, n_tok_out=n_tok, token_traj_out=tt)
-        loaded = [None, None]
-        freed = [None, None]
         for k, (lo, hi) in enumerate(batch.mbs):
-            s = k & 1
+            s = k % slots
             n = hi - lo
-            with t.cuda.stream(copy_in):
-                if freed[s] is not None:
-                    copy_in.wait_event(freed[s])
-                dev_logits[s][:n].copy_(host_logits[s][:n], non_blocking=True)
-                loaded[s] = t.cuda.Event()
-                loaded[s].record(copy_in)
-            comp.wait_event(loaded[s])
+            cs = copy_streams[k & 1]
+            with t.cuda.stream(cs):
+                if read_done[s] is not None:
+                    cs.wait_event(read_done[s])
+                dev_logits[s][:n].copy_(host_mb[src[k]][:n], non_blocking=True)
+                loaded = t.cuda.Event()
+                loaded.record(cs)
+            comp.wait_event(loaded)
             R.rl_policy_loss_fwd_bwd(dev_logits[s][:n], meta_dev["ids"][lo:hi], meta_dev["mask"][lo:hi], tt[lo:hi],
                                      adv, coef, meta_dev["old"][lo:hi], batch.params, batch.ws, loss,
-                                     grad_out=dev_grad[s][:n], stream=comp)
-            done = t.cuda.Event()
-            done.record(comp)
-            with t.cuda.stream(copy_out):
-                copy_out.wait_event(done)
-                host_grad[s][:n].copy_(dev_grad[s][:n], non_blocking=True)
-                freed[s] = t.cuda.Event()
-                freed[s].record(copy_out)
-        comp.wait_stream(copy_out)
+                                     grad_out=batch.grad[lo:hi], stream=comp)
+            read_done[s] = t.cuda.Event()
+            read_done[s].record(comp)
         loss_host.copy_(loss, non_blocking=True)
 
     for _ in range(warmup):
@@ -387,7 +413,9 @@ def e2e_run(torch, R, batch, dev, steps, warmup):
     e1.synchronize()
     t.cuda.synchronize(dev)
     ms = e0.elapsed_time(e1)
-    return ms, h2d, d2h
+    check = float(loss_host.item())
+    del host_mb
+    return ms, h2d, d2h, check, ("whole batch" if whole else "ring of 2 microbatches")
 
 
 # ----------------------------------------------------------------------------- oracle (CPU) legs
@@ -850,9 +878,11 @@ def main():
 
     e2e = None
     if not args.no_e2e:
-        e_ms, h2d, d2h = e2e_run(torch, R, batch, dev, args.e2e_steps, 1)
+        e_ms, h2d, d2h, e_loss, src = e2e_run(torch, R, batch, dev, args.e2e_steps, 1)
         e2e = {"value": batch.T / (e_ms / 1e3 / args.e2e_steps) * world, "unit": UNIT, "h2d_bytes_per_step": h2d,
-               "d2h_bytes_per_step": d2h, "steps": args.e2e_steps}
+               "d2h_bytes_per_step": d2h, "steps": args.e2e_steps, "loss": e_loss, "host_source": src,
+               "note": "per step: metadata and every microbatch's logits from pinned host memory, loss read "
+                       "back; the gradient stays in HBM for the model's backward"}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
