@@ -209,7 +209,8 @@ def row_statistics(z: np.ndarray, a: np.ndarray):
     """For rows z[r, :] (float64) and sampled ids a[r]:
 
     lse = log sum_v exp(z_v), log p_v = z_v - lse, logp = z_a - lse and the entropy
-    H = -sum_v p_v log p_v.  Returns (lse, logp, H, p, z_a).
+    H = -sum_v p_v log p_v with 0 log 0 = 0 (entries at -inf have p = 0 and add nothing).
+    Returns (lse, logp, H, p, z_a).
     """
     z = np.atleast_2d(z)
     a = np.asarray(a, dtype=np.int64)
@@ -221,7 +222,8 @@ def row_statistics(z: np.ndarray, a: np.ndarray):
     rows = np.arange(z.shape[0])
     z_a = z[rows, a]
     logp = z_a - lse[:, 0]
-    H = -(p * logp_all).sum(axis=1)
+    with np.errstate(invalid="ignore"):  # 0 * (-inf) in the branch that np.where discards
+        H = -np.where(p > 0, p * logp_all, 0.0).sum(axis=1)
     return lse[:, 0], logp, H, p, z_a
 
 
@@ -331,7 +333,8 @@ def policy_loss_fwd_bwd(logits, dtype, token_ids, mask, token_traj, adv, coef, o
             gz = -tt["g"][:, None] * p
             gz[np.arange(len(r)), a] += tt["g"]
             if alpha != 0.0:
-                gz += alpha * p * (z - lse[:, None] + H[:, None])
+                with np.errstate(invalid="ignore"):  # 0 * (-inf) in the discarded branch
+                    gz += np.where(p > 0, alpha * p * (z - lse[:, None] + H[:, None]), 0.0)
             grad[loc] = c[:, None] * gz
     loss = math.fsum(contrib.tolist())
     return loss, grad, stats, contrib

@@ -194,6 +194,32 @@ def pin_rowstats_library(O):
     _close(p, pt, rtol=1e-10, atol=1e-300, what="p vs torch")
 
 
+def pin_rowstats_neg_inf(O):
+    """Entries at -inf have probability 0: lse, logp and H equal those of the row without them,
+    and the loss gradient is exactly 0 there and equal to the reduced row's elsewhere
+    (entropy bonus and KL on)."""
+    rng = np.random.default_rng(21)
+    V = 12
+    z = rng.normal(0, 1.5, size=(3, V))
+    drop = [np.array([1, 5, 6]), np.array([0]), np.array([2, 3, 4, 9, 11])]
+    a = np.array([0, 4, 10])
+    for r, dr in enumerate(drop):
+        z[r, dr] = -np.inf
+    keep = [np.setdiff1d(np.arange(V), dr) for dr in drop]
+    lse, logp, H, _, _ = O.row_statistics(z, a)
+    for r in range(3):
+        zr = z[r, keep[r]][None, :]
+        ar = np.array([int(np.nonzero(keep[r] == a[r])[0][0])])
+        l2, lp2, h2, _, _ = O.row_statistics(zr, ar)
+        _close([lse[r], logp[r], H[r]], [l2[0], lp2[0], h2[0]], rtol=1e-13, atol=1e-14, what=f"-inf row {r}")
+        P = O.LossParams(entropy_coef=0.05, kl_coef=0.1, kl_estimator=3)
+        old, ref = np.array([logp[r] + 0.1]), np.array([logp[r] - 0.2])
+        _, g, _, _ = O.policy_loss_fwd_bwd(z[r:r + 1], "f64", a[r:r + 1], [1], [0], [1.3], [0.5], old, P, ref)
+        _, g2, _, _ = O.policy_loss_fwd_bwd(zr, "f64", ar, [1], [0], [1.3], [0.5], old, P, ref)
+        assert np.all(g[0, drop[r]] == 0.0)
+        _close(g[0, keep[r]], g2[0], rtol=1e-12, atol=1e-15, what=f"-inf grad {r}")
+
+
 def pin_rowstats_shift(O):
     """lse(z + c) = lse(z) + c; logp and H unchanged (c = -1e4 and +37)."""
     rng = np.random.default_rng(1)

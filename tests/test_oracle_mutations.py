@@ -29,7 +29,10 @@ MUTANTS = {
                         "c[counted] = 1.0 / (n * L[counted].astype(np.float64))"),
     "count off by one span": ("L[i] = int(np.count_nonzero(mask[s:e]))", "L[i] = int(np.count_nonzero(mask[s:e + 1]))"),
     "lse without max": ("lse = m + np.log(s)", "lse = np.log(s)"),
-    "entropy sign": ("H = -(p * logp_all).sum(axis=1)", "H = (p * logp_all).sum(axis=1)"),
+    "entropy sign": ("H = -np.where(p > 0, p * logp_all, 0.0).sum(axis=1)",
+                     "H = np.where(p > 0, p * logp_all, 0.0).sum(axis=1)"),
+    "entropy 0 log 0 not 0": ("H = -np.where(p > 0, p * logp_all, 0.0).sum(axis=1)",
+                              "H = -(p * logp_all).sum(axis=1)"),
     "gather wrong index": ("z_a = z[rows, a]", "z_a = z[rows, (a + 1) % z.shape[1]]"),
     "ratio inverted": ("log_ratio = (z_a - old) - lse", "log_ratio = (old - z_a) + lse"),
     "symmetric clip": ("clipped_rho = np.minimum(np.maximum(rho, 1.0 - el), 1.0 + eh)",
@@ -48,8 +51,10 @@ MUTANTS = {
     "objective not negated": ("ell = -w * surr", "ell = w * surr"),
     "grad without tis weight": ("g = -w * A * rho * act", "g = -A * rho * act"),
     "grad without ratio": ("g = -w * A * rho * act", "g = -w * A * act"),
-    "dropped entropy grad term": ("gz += alpha * p * (z - lse[:, None] + H[:, None])",
-                                  "gz += alpha * p * (z - lse[:, None])"),
+    "dropped entropy grad term": ("gz += np.where(p > 0, alpha * p * (z - lse[:, None] + H[:, None]), 0.0)",
+                                  "gz += np.where(p > 0, alpha * p * (z - lse[:, None]), 0.0)"),
+    "entropy grad at -inf entries": ("gz += np.where(p > 0, alpha * p * (z - lse[:, None] + H[:, None]), 0.0)",
+                                     "gz += alpha * p * (z - lse[:, None] + H[:, None])"),
     "dropped softmax grad term": ('gz = -tt["g"][:, None] * p', 'gz = 0.0 * p'),
     "masked rows kept": ("active = (mask[sel] != 0) & (c_row != 0.0)", "active = (c_row != 0.0)"),
     "loss not weighted": ('contrib[loc] = c * tt["ell"]', 'contrib[loc] = tt["ell"]'),
