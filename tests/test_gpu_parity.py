@@ -6,6 +6,8 @@ vocabulary tails, unaligned leading dimensions and the degenerate cases.
 Full-size workloads are in test_gpu_fullsize.py.
 """
 
+import dataclasses
+
 import numpy as np
 import pytest
 import torch
@@ -249,3 +251,52 @@ def test_end_to_end_advantages_then_loss(R):
     l_ref, g_ref, _, contrib = oracle_loss(case)
     check_loss(loss.item(), l_ref, contrib, "end to end")
     check_grad(grad_to_np(g), g_ref, "bf16", "end to end")
+
+
+# ----------------------------------------------------------------------------- logits at -inf
+
+def neg_inf_case(name, rows, seed=6, entropy=False):
+    """Rows with vocabulary entries masked to -inf (never the sampled one): 30% of the entries
+    in half the rows, all but three entries in one row. old_logp and ref_logp follow from the
+    masked rows' log-probabilities, so the ratio band around the clip bounds still holds."""
+    c = make_case(name, seed=seed, rows=rows)
+    raw = c.raw.copy()
+    V = raw.shape[1]
+    rng = np.random.default_rng(seed + 100)
+    ninf = np.uint16(0xFF80) if c.w.dtype == "bf16" else np.float32(-np.inf)
+    for r in range(0, c.rows, 2):
+        cols = rng.random(V) < 0.3
+        cols[c.ids[r]] = False
+        raw[r, cols] = ninf
+    r = 1
+    cols = np.ones(V, bool)
+    cols[[c.ids[r], (c.ids[r] + 1) % V, (c.ids[r] + 7) % V]] = False
+    raw[r, cols] = ninf
+    logp, _, _ = O.token_logprobs(raw, c.w.dtype, c.ids)
+    old = W.old_logp_from(logp, c.w, seed, c.row0)
+    ref = W.ref_logp_from(logp, c.w, seed, c.row0) if c.w.ref_noise_std else None
+    P = dataclasses.replace(c.P, entropy_coef=1e-2) if entropy else c.P
+    return dataclasses.replace(c, raw=raw, old=old, ref=ref, P=P)
+
+
+@pytest.mark.parametrize("name,entropy", [("longhorizon", False), ("multiturn", True), ("edge", True),
+                                          ("multiturn", False)])
+def test_policy_loss_neg_inf_logits(R, name, entropy):
+    case = neg_inf_case(name, 64, entropy=entropy)
+    out = run_loss(R, case)
+    compare(case, out, f"{name} -inf entries, entropy={entropy}")
+    assert np.isfinite(out["grad"]).all()
+
+
+@pytest.mark.parametrize("name", ["multiturn", "edge"])
+def test_token_logprobs_neg_inf_logits(R, name):
+    case = neg_inf_case(name, 48)
+    V = case.raw.shape[1]
+    ws = R.new_workspace(case.rows, V)
+    logp, H, lse = R.rl_token_logprobs(logits_to_dev(case), to_dev(case.ids), ws, want_entropy=True, want_lse=True)
+    assert R.rl_query_status(ws)[1] == 0
+    lp_ref, H_ref, lse_ref = O.token_logprobs(case.raw, case.w.dtype, case.ids)
+    lp, Hd, ls = (x.cpu().numpy().astype(np.float64) for x in (logp, H, lse))
+    assert np.all(np.abs(lp - lp_ref) <= 1e-5 + 2.0 ** -22 * np.abs(lp_ref)), np.abs(lp - lp_ref).max()
+    assert np.all(np.abs(ls - lse_ref) <= 1e-5 + 2.0 ** -22 * np.abs(lse_ref)), np.abs(ls - lse_ref).max()
+    assert np.all(np.abs(Hd - H_ref) <= 5e-5 + 2e-5 * np.abs(H_ref)), np.abs(Hd - H_ref).max()
