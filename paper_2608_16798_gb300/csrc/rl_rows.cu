@@ -29,6 +29,7 @@
 #include <map>
 #include <mutex>
 #include <tuple>
+#include <type_traits>
 
 #include "rl_device.cuh"
 #include "rl_host.h"
@@ -286,41 +287,51 @@ __device__ __forceinline__ void fold_block(SoftmaxPartial& ps, const uint4 (&x)[
     if (!(m0 > -1e38f)) return;
     ps.m = m0;
   }
-  auto exps = [&](const uint4 w, float2& s0, float2& s1, float2& u0) {
+  // x = (z - m) log2(e) by one fused multiply-add against nm = fl(-m log2(e)); with the
+  // entropy, u accumulates e x (log2 units, scaled by ln 2 at the end). A logit at -inf gives
+  // e = 0 and e x = NaN: such a block is redone on the clamped path (CLAMP), where z counts as
+  // -1e30. The rounding of nm shifts every x of the block by the same err = -m log2(e) - nm
+  // (exact by one fma); the block's sums are corrected for it once at the end.
+  auto exps = [&](auto clamp, const uint4 w, float2& s0, float2& s1, float2& u0) {
+    constexpr bool CLAMP = decltype(clamp)::value;
     const float nm = -ps.m * kLog2e;
-    const float2 l2 = make_float2(kLog2e, kLog2e), nm2 = make_float2(nm, nm), mm = make_float2(-ps.m, -ps.m);
+    const float2 l2 = make_float2(kLog2e, kLog2e), nm2 = make_float2(nm, nm);
     float2 q[NP];
     Vec<T>::pairs(w, q);
 #pragma unroll
     for (int i = 0; i < NP; ++i) {
-      if (ENT) {
-        const float2 t = __fadd2_rn(make_float2(fmaxf(q[i].x, -1e30f), fmaxf(q[i].y, -1e30f)), mm);
-        const float2 xx = __fmul2_rn(t, l2);
-        const float2 e = make_float2(ex2(xx.x), ex2(xx.y));
-        if (i & 1) s1 = __fadd2_rn(s1, e); else s0 = __fadd2_rn(s0, e);
-        u0 = __ffma2_rn(e, t, u0);
-      } else {
-        const float2 xx = __ffma2_rn(q[i], l2, nm2);
-        const float2 e = make_float2(ex2(xx.x), ex2(xx.y));
-        if (i & 1) s1 = __fadd2_rn(s1, e); else s0 = __fadd2_rn(s0, e);
-      }
+      const float2 qi = CLAMP ? make_float2(fmaxf(q[i].x, -1e30f), fmaxf(q[i].y, -1e30f)) : q[i];
+      const float2 xx = __ffma2_rn(qi, l2, nm2);
+      const float2 e = make_float2(ex2(xx.x), ex2(xx.y));
+      if (i & 1) s1 = __fadd2_rn(s1, e); else s0 = __fadd2_rn(s0, e);
+      if (ENT) u0 = __ffma2_rn(e, xx, u0);
     }
   };
+  using Fast = std::integral_constant<bool, false>;
+  using Clamped = std::integral_constant<bool, true>;
   const float2 z2 = make_float2(0.f, 0.f);
   float2 s0 = z2, s1 = z2, u0 = z2;
 #pragma unroll
-  for (int k = 0; k < NV; ++k) exps(x[k], s0, s1, u0);
+  for (int k = 0; k < NV; ++k) exps(Fast{}, x[k], s0, s1, u0);
   float2 sacc = __fadd2_rn(s0, s1);
   float se = sacc.x + sacc.y;
-  if (!(se <= 1e30f)) {  // rare: move the reference up to the exact maximum and redo from shared memory
-    raise_max<ENT>(ps, all_max());
+  float ue = ENT ? u0.x + u0.y : 0.f;
+  if (!(se <= 1e30f) || (ENT && ue != ue)) {
+    // rare: a value far above the reference (move it up to the exact maximum) or a logit at
+    // -inf with the entropy on; redo from shared memory on the clamped path
+    if (!(se <= 1e30f)) raise_max<ENT>(ps, all_max());
     s0 = z2; s1 = z2; u0 = z2;
-    for (int k = 0; k < NV; ++k) exps(reload(k), s0, s1, u0);
+    for (int k = 0; k < NV; ++k) exps(Clamped{}, reload(k), s0, s1, u0);
     sacc = __fadd2_rn(s0, s1);
     se = sacc.x + sacc.y;
+    ue = ENT ? u0.x + u0.y : 0.f;
   }
-  ps.s += se;
-  if (ENT) ps.u += u0.x + u0.y;
+  // e_true = e 2^err and x_true = x + err, with |err| <= 2^-24 |m log2(e)|: first order in err
+  const float nm = -ps.m * kLog2e;
+  const float err = fmaf(-ps.m, kLog2e, -nm);
+  const float f = fmaf(err, kLn2, 1.f);
+  if (ENT) ps.u = fmaf(fmaf(err, se, ue) * f, kLn2, ps.u);
+  ps.s = fmaf(se, f, ps.s);
 }
 
 template <typename T, int NW, bool ENT, bool BWD, int HOLDV>
@@ -572,9 +583,14 @@ __global__ void __launch_bounds__((NW + 1) * 32, 2) rows_kernel(const RowArgs p)
         }
         const float ell = -w * surr + p.beta * kl - p.alpha * H;
         const float g = (cut ? 0.f : -w * A * rho) + p.beta * dkl;
-        const float cg = c * g, ca = c * p.alpha;
-        const float Kp = -cg;                    // gradient = Kp p_v (+ cg at v = a)
-        const float Ke = -cg + ca * (H - lse);   // entropy: p_v (ca z_v + Ke)
+        const float cg = c * g, ca0 = c * p.alpha;
+        // p_v = 2^(z_v log2(e) + nl) with nl = fl(-lse log2(e)); its rounding scales every p_v of
+        // the row by 2^errl (errl exact by one fma), folded into the coefficients below
+        const float nl = -lse * kLog2e;
+        const float fl = fmaf(fmaf(-lse, kLog2e, -nl), kLn2, 1.f);
+        const float Kp = -cg * fl;                      // gradient = Kp p_v (+ cg at v = a)
+        const float ca = ca0 * fl;                      // entropy: p_v (ca z_v + Ke)
+        const float Ke = (-cg + ca0 * (H - lse)) * fl;
         if (rank == 0 && warp == 0 && lane == 0) {
           p.row_loss[r] = static_cast<double>(c) * static_cast<double>(ell);
           if (p.token_stats) {
@@ -583,7 +599,6 @@ __global__ void __launch_bounds__((NW + 1) * 32, 2) rows_kernel(const RowArgs p)
           }
         }
         // ---- pass 2: gradient from the on-chip slice
-        const float nl = -lse * kLog2e;
         T* g_row = grad + r * ld + s0;
         auto grad_vec = [&](const float (&v)[EPV], int j) {
           float o[EPV];
