@@ -31,6 +31,9 @@ Every function follows one passage of the paper (arXiv 2608.16798, "ClawGym II")
 * ``fused_head_loss_fwd_bwd``  -- the same objective with logits = hidden @ W^T
   and gradients with respect to hidden and W.
 * ``fused_head_logprobs``      -- forward-only log-probabilities of logits = hidden @ W^T.
+* ``stats_summary``            -- batch sums of the per-token statistics (trained tokens,
+  clipped tokens, entropy, KL, ratio): the clip fraction and the mean policy entropy that
+  the paper tracks during training (Sec. 4, training dynamics).
 * ``sequence_is_weights``      -- the sequence-level importance ratio between the training
   engine's and the rollout engine's policies, truncated at c-bar (Sec. 3.2.4, the
   sequence-level alternative to the token-level TIS weight).
@@ -412,3 +415,17 @@ def sequence_is_weights(token_traj, mask, old_logp, rollout_logp, n_traj: int, c
     if cap > 0:
         w = np.minimum(w, cap)
     return w, S
+
+
+# ----------------------------------------------------------------------------
+# Batch summaries of the per-token statistics (monitoring)
+# ----------------------------------------------------------------------------
+
+def stats_summary(stats, mask, token_traj, coef):
+    """Over the trained tokens (M_t != 0 and c_{i(t)} != 0): (count, number clipped, sum of H,
+    sum of KL, sum of rho) from per-token stats rows (logp, rho, clipped, H, KL)."""
+    st = np.asarray(stats, dtype=np.float64).reshape(-1, 5)
+    c = np.asarray(coef, dtype=np.float64)[np.asarray(token_traj, dtype=np.int64)]
+    act = (np.asarray(mask) != 0) & (c != 0)
+    return np.array([float(act.sum()), math.fsum(st[act, STAT_CLIPPED]), math.fsum(st[act, STAT_ENTROPY]),
+                     math.fsum(st[act, STAT_KL]), math.fsum(st[act, STAT_RATIO])])

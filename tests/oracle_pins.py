@@ -479,6 +479,28 @@ def pin_sequence_is_weights(O):
     _close(g_seq, g_tok, rtol=1e-12, atol=1e-15, what="sequence weight vs token weight, grad")
 
 
+def pin_stats_summary(O):
+    """Hand-worked: three trained tokens (one clipped), one masked and one of a zero-coefficient
+    trajectory are left out; and the summary of a loss call's stats at rho = 1 counts every
+    trained token with ratio 1 and none clipped."""
+    stats = np.array([[-1.0, 1.5, 1.0, 2.0, 0.1], [-2.0, 0.9, 0.0, 1.0, 0.2], [-0.5, 1.0, 0.0, 3.0, 0.0],
+                      [-9.0, 7.0, 1.0, 9.0, 9.0], [-9.0, 7.0, 1.0, 9.0, 9.0]])
+    mask = [1, 1, 1, 0, 1]
+    tt = [0, 0, 1, 1, 2]
+    coef = [0.5, 0.25, 0.0]
+    _close(O.stats_summary(stats, mask, tt, coef), [3.0, 1.0, 6.0, 0.3, 3.4], rtol=1e-15, what="summary")
+    pr = _tiny_problem(23, n_traj=5, agg=1, alpha=0.0, beta=0.0, tis=0.0)
+    z = pr["z"]
+    T = z.shape[0]
+    zmax = z.max(axis=1)
+    logp = z[np.arange(T), pr["a"]] - (zmax + np.log(np.exp(z - zmax[:, None]).sum(axis=1)))
+    P = O.LossParams(**pr["P"])
+    _, _, st, _ = O.policy_loss_fwd_bwd(z, "f64", pr["a"], pr["mask"], pr["tt"], pr["adv"], pr["coef"], logp, P)
+    sm = O.stats_summary(st, pr["mask"], pr["tt"], pr["coef"])
+    n_act = int(((pr["mask"] != 0) & (pr["coef"][pr["tt"]] != 0)).sum())
+    _close(sm[[0, 1, 4]], [n_act, 0.0, n_act], rtol=1e-12, what="rho = 1 summary")
+
+
 def pin_loss_additive_and_permutation(O):
     """The loss of two microbatches adds up to the loss of the whole batch; permuting the
     rows permutes the gradient rows and keeps the loss."""

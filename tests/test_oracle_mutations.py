@@ -69,6 +69,8 @@ MUTANTS = {
     "seq weight inverted ratio": ("d = np.asarray(old_logp, dtype=np.float64) - np.asarray(rollout_logp, dtype=np.float64)",
                                   "d = np.asarray(rollout_logp, dtype=np.float64) - np.asarray(old_logp, dtype=np.float64)"),
     "seq weight cap as max": ("w = np.minimum(w, cap)", "w = np.maximum(w, cap)"),
+    "summary counts masked tokens": ("act = (np.asarray(mask) != 0) & (c != 0)", "act = c != 0"),
+    "summary sums the wrong column": ("math.fsum(st[act, STAT_ENTROPY])", "math.fsum(st[act, STAT_LOGP])"),
     "head logprobs chunk offset": ("Z = Hm[r0:r0 + chunk] @ Wm.T", "Z = Hm[r0 + 1:r0 + 1 + chunk] @ Wm.T"),
 }
 
