@@ -46,13 +46,13 @@ KERNEL_SRC = os.path.join(ROOT, "paper_2608_16798_gb300", "csrc", "rl_rows.cu")
 FALLBACK_HBM_GBS = 6800.0
 
 
-def workload_config(T, n_mb):
+def workload_config(T, n_mb, inputs_sha256=None):
     w = WORKLOAD
     return {"workload": f"multiturn: {w.n_groups} groups x {w.group_size} trajectories, lengths U{{256..2048}}, "
                         f"~40% masked in spans, V={w.vocab}, bf16 logits N(0,2^2), {w.microbatch}-row microbatches",
             "tokens_per_step": int(T), "microbatches": int(n_mb), "vocab": w.vocab, "logits": "bf16",
             "l2": "no flush: resident inputs (logits + gradient) far larger than L2",
-            "parallelism": "replicas"}
+            "parallelism": "replicas", "seed": 0, "inputs_sha256": inputs_sha256}
 
 
 def measured_peaks():
@@ -159,6 +159,13 @@ class DeviceBatch:
         self.n_tok = t.empty(self.lay.n_traj, dtype=t.int32, device=dev)
         self.token_traj = t.empty(self.T, dtype=t.int32, device=dev)
         self.loss = t.zeros(1, dtype=t.float64, device=dev)
+        h = hashlib.sha256()
+        for a in (self.lay.traj_offsets, self.lay.group_offsets, self.lay.rewards, self.lay.mask,
+                  self.ids.cpu().numpy(), self.old.cpu().numpy()):
+            h.update(np.ascontiguousarray(a).tobytes())
+        for r in (0, self.T // 2, self.T - 1):
+            h.update(self.logits[r].view(t.int16).cpu().numpy().tobytes())
+        self.inputs_sha256 = h.hexdigest()
         m = self.lay.mask.astype(np.int64)
         es = 2
         # algorithmic bytes per microbatch launch: trainable rows read + write, other rows write only
@@ -206,6 +213,74 @@ def time_logits_extras(torch, R, batch, dev, peak, reps=20):
                                                               n_tok_out=batch.n_tok, token_traj_out=batch.token_traj),
                          50)
     out["group_advantages_us"] = ms_adv * 1e3
+    return out
+
+
+def time_other_workloads(torch, R, dev, peak, reps=10):
+    """rl_policy_loss_fwd_bwd on the long-horizon workload (bf16, entropy + k3 KL, two resident
+    32,768-row microbatches: the first and the middle one) and the edge workload (fp32,
+    V = 32,000, the whole 131,072-row batch as one microbatch), timed with CUDA events around
+    `reps` launches after two warm-up launches. The logits stay resident (20 and 17 GB, far
+    above L2); pi_old comes from the library's forward pass plus the workload's noise."""
+    t = torch
+    out = {}
+    for name, picks in (("longhorizon", (0, None)), ("edge", (0,))):
+        w = W.WORKLOADS[name]
+        lay = W.make_layout(w, 0)
+        mbs = W.microbatches(lay, w.microbatch)
+        chosen = [mbs[0] if k == 0 else mbs[len(mbs) // 2] for k in picks]
+        dt = t.bfloat16 if w.dtype == "bf16" else t.float32
+        es = 2 if w.dtype == "bf16" else 4
+        d = lambda x: t.from_numpy(np.ascontiguousarray(x)).to(dev)  # noqa: E731
+        kl = 3 if w.kl_coef else 0
+        params = R.make_params(W.CLIP_EPS_LOW, W.CLIP_EPS_HIGH, w.kl_coef, kl, w.entropy_coef, 0.0, 1e-6, 0)
+        ws = R.new_workspace(w.microbatch, w.vocab, device=dev)
+        adv, coef, n_tok, tt = R.rl_group_advantages(d(lay.group_offsets), d(lay.rewards), d(lay.traj_offsets),
+                                                     d(lay.mask), params, ws, traj_valid=d(lay.traj_valid))
+        coef_h, tt_h = coef.cpu().numpy(), tt.cpu().numpy()
+        items, nbytes, rows_total = [], 0, 0
+        for lo, hi in chosen:
+            n = hi - lo
+            logits = t.empty((n, w.vocab), dtype=dt, device=dev)
+            W.logits_rows_torch(w, 0, lo, n, logits)
+            ids = W.sample_tokens_torch(logits, 0, lo, w)
+            logp, _, _ = R.rl_token_logprobs(logits, ids, ws)
+            lp = logp.cpu().numpy()
+            old = d(W.old_logp_from(lp, w, 0, lo))
+            ref = d(W.ref_logp_from(lp, w, 0, lo)) if w.ref_noise_std else None
+            grad = t.empty_like(logits)
+            trained = (lay.mask[lo:hi] != 0) & (coef_h[tt_h[lo:hi]] != 0)
+            nbytes += int((trained.astype(np.int64) + 1).sum()) * w.vocab * es
+            rows_total += n
+            items.append((logits, ids, d(lay.mask[lo:hi]), tt[lo:hi], old, ref, grad))
+        loss = t.zeros(1, dtype=t.float64, device=dev)
+
+        def launch(k):
+            lg, ids, m, tk, old, ref, g = items[k % len(items)]
+            R.rl_policy_loss_fwd_bwd(lg, ids, m, tk, adv, coef, old, params, ws, loss, grad_out=g, ref_logp=ref)
+
+        for k in range(2):
+            launch(k)
+        t.cuda.synchronize(dev)
+        a, b = t.cuda.Event(enable_timing=True), t.cuda.Event(enable_timing=True)
+        a.record()
+        for k in range(reps):
+            launch(k)
+        b.record()
+        b.synchronize()
+        st, word = R.rl_query_status(ws)
+        if word != 0:
+            raise RuntimeError(f"device status word {word} after the {name} timing")
+        ms = a.elapsed_time(b) / reps
+        per_launch_bytes = nbytes / len(items)
+        rows_per_launch = rows_total / len(items)
+        gbs = per_launch_bytes / (ms * 1e-3) / 1e9
+        out[name] = {"rows_per_launch": rows_per_launch, "vocab": w.vocab, "dtype": w.dtype,
+                     "entropy_coef": w.entropy_coef, "kl_coef": w.kl_coef, "ms_per_launch": ms,
+                     "tokens_per_s": rows_per_launch / (ms * 1e-3), "algorithmic_bytes_per_launch": per_launch_bytes,
+                     "achieved_gbs": gbs, "frac": gbs / peak, "reps": reps}
+        del items
+        t.cuda.empty_cache()
     return out
 
 
@@ -797,6 +872,7 @@ def main():
     ap.add_argument("--no-head", action="store_true", help="skip the fused-head measurement")
     ap.add_argument("--no-ppo", action="store_true", help="skip the PPO-step measurement")
     ap.add_argument("--no-tree", action="store_true", help="skip the prefix-tree measurement")
+    ap.add_argument("--no-other", action="store_true", help="skip the long-horizon and edge workloads")
     args = ap.parse_args()
     if args.profile_case:
         return profile_case(args.profile_case)
@@ -873,6 +949,8 @@ def main():
         per_mb.append({"rows": batch.mbs[k][1] - batch.mbs[k][0], "median_ms": statistics.median(ts),
                        "best_ms": min(ts), "median_gbs": batch.mb_bytes[k] / (statistics.median(ts) * 1e-3) / 1e9})
     extras = time_logits_extras(torch, R, batch, dev, peak)
+    if not args.no_other:
+        extras["other_workloads"] = time_other_workloads(torch, R, dev, peak)
     extras["loss_microbatches"] = per_mb
     extras["loss_batch_sum_ms"] = sum(m["median_ms"] for m in per_mb)
 
@@ -898,7 +976,7 @@ def main():
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
-                "vs_baseline": None, "dtype": "f32", "data": "synthetic", "config": workload_config(batch.T, n_mb),
+                "vs_baseline": None, "dtype": "f32", "data": "synthetic", "config": workload_config(batch.T, n_mb, batch.inputs_sha256),
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks, "logits_path": extras, "fused_head": head, "ppo": ppo, "tree": tree,
                 "gpu_launches": batch.launches_per_step() * args.steps,
                 "loss_per_step": float(batch.loss.item()) / (args.warmup + args.steps)}

@@ -244,6 +244,25 @@ rl_status rl_fused_head_loss_fwd_bwd(const void* hidden, const void* weight, int
                                      size_t ws_bytes, rl_stream_t stream);
 
 /*
+ * Batch summary of the per-token statistics written by rl_policy_loss_fwd_bwd /
+ * rl_fused_head_loss_fwd_bwd (token_stats rows (logp, rho, clipped, H, KL)): over the trained
+ * tokens (M_t != 0, owner in range, c_{i(t)} != 0) it ADDS to summary_accum
+ *   [0] the number of trained tokens, [1] the number clipped, [2] sum of H_t,
+ *   [3] sum of KL_t, [4] sum of rho_t
+ * (the clip fraction and the mean policy entropy tracked during training, Sec. 4). Call it
+ * once per microbatch with the same accumulator; divide by [0] for the means.
+ *
+ *   rows, token_stats  float [rows x 5]
+ *   mask, token_traj, n_traj, coef   as for rl_policy_loss_fwd_bwd
+ *   summary_accum      double [5] on the device
+ *   ws, ws_bytes       rl_workspace_size(0, 0, 0) bytes suffice (status word)
+ * One CTA in a fixed order, in double precision: deterministic.
+ */
+rl_status rl_token_stats_summary(int64_t rows, const float* token_stats, const uint8_t* mask,
+                                 const int32_t* token_traj, int32_t n_traj, const float* coef,
+                                 double* summary_accum, void* ws, size_t ws_bytes, rl_stream_t stream);
+
+/*
  * Masked generalised advantage estimation for PPO (Sec. 2.3.1, masked GAE and TD
  * residual; Sec. 2.3.4, PPO with each trajectory backed up on its own), per
  * trajectory of the packed stream:

@@ -1,0 +1,69 @@
+// Batch summaries of the per-token statistics that rl_policy_loss_fwd_bwd and
+// rl_fused_head_loss_fwd_bwd write: the number of trained tokens, of clipped ones, and the
+// sums of entropy, KL and ratio over them (the clip fraction and the mean policy entropy that
+// are tracked during training, Sec. 4). One CTA, fixed assignment of rows to threads and a
+// fixed reduction order in double precision: the sums are the same on every run.
+#include <cstdint>
+
+#include "rl_device.cuh"
+#include "rl_host.h"
+
+namespace rl {
+
+constexpr int kSumThreads = 1024;
+
+__global__ void __launch_bounds__(kSumThreads) stats_summary_kernel(int64_t rows, const float* __restrict__ st,
+                                                                    const uint8_t* __restrict__ mask,
+                                                                    const int32_t* __restrict__ token_traj,
+                                                                    int32_t n_traj, const float* __restrict__ coef,
+                                                                    double* __restrict__ out, int32_t* status) {
+  __shared__ double part[kSumThreads / 32][5];
+  double acc[5] = {0.0, 0.0, 0.0, 0.0, 0.0};
+  for (int64_t r = threadIdx.x; r < rows; r += kSumThreads) {
+    if (mask[r] == 0) continue;
+    const int32_t i = token_traj[r];
+    if (i < 0 || i >= n_traj) {
+      flag_status(status, RL_DEV_BAD_TRAJ);
+      continue;
+    }
+    if (coef[i] == 0.f) continue;
+    const float* s = st + r * 5;
+    acc[0] += 1.0;
+    acc[1] += static_cast<double>(s[2]);
+    acc[2] += static_cast<double>(s[3]);
+    acc[3] += static_cast<double>(s[4]);
+    acc[4] += static_cast<double>(s[1]);
+  }
+#pragma unroll
+  for (int k = 0; k < 5; ++k) acc[k] = warp_sum(acc[k]);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (lane == 0)
+    for (int k = 0; k < 5; ++k) part[warp][k] = acc[k];
+  __syncthreads();
+  if (threadIdx.x < 5) {
+    double sum = 0.0;
+    for (int w = 0; w < kSumThreads / 32; ++w) sum += part[w][threadIdx.x];
+    out[threadIdx.x] += sum;
+  }
+}
+
+}  // namespace rl
+
+extern "C" rl_status rl_token_stats_summary(int64_t rows, const float* token_stats, const uint8_t* mask,
+                                            const int32_t* token_traj, int32_t n_traj, const float* coef,
+                                            double* summary_accum, void* ws, size_t ws_bytes, rl_stream_t stream) {
+  using namespace rl;
+  clear_error();
+  if (rows < 0 || n_traj < 0) return set_error(RL_ERR_INVALID_ARG, "rl_token_stats_summary: negative size");
+  if (!summary_accum || !ws) return set_error(RL_ERR_INVALID_ARG, "rl_token_stats_summary: NULL argument");
+  if (ws_bytes < kWsHeader) return set_error(RL_ERR_WORKSPACE_TOO_SMALL, "rl_token_stats_summary: workspace too small");
+  if (rows == 0) return RL_OK;
+  if (!token_stats || !mask || !token_traj || (n_traj > 0 && !coef))
+    return set_error(RL_ERR_INVALID_ARG, "rl_token_stats_summary: NULL array argument");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  stats_summary_kernel<<<1, kSumThreads, 0, s>>>(rows, token_stats, mask, token_traj, n_traj, coef, summary_accum,
+                                                 reinterpret_cast<int32_t*>(ws));
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_error(e, "stats_summary_kernel launch");
+  return RL_OK;
+}

@@ -46,6 +46,7 @@ EXPORTS = {
                                           _P, _P, _P, _P, _P, _P, _P, _P]),
     "rl_group_advantages_by_owner": (_I32, [_I32, _I32, _P, _P, _P, _I64, _P, _P, _P, _P, _P, _P, _P, _SZ, _P]),
     "rl_rollout_value_advantages": (_I32, [_I64, _P, _P, _P, _P, _I32, _P, _P, _P, _SZ, _P]),
+    "rl_token_stats_summary": (_I32, [_I64, _P, _P, _P, _I32, _P, _P, _P, _SZ, _P]),
     "rl_masked_gae": (_I32, [_I32, _P, _I64, _P, _P, _P, _P, _F, _F, _I32, _P, _P, _P, _SZ, _P]),
     "rl_value_loss_fwd_bwd": (_I32, [_I64, _P, _P, _P, _P, _I32, _P, _P, _P, _P, _SZ, _P]),
     "rl_fused_head_token_logprobs": (_I32, [_P, _P, _I64, _I64, _I64, _P, _P, _P, _P, _P, _SZ, _P]),
@@ -553,3 +554,23 @@ def rl_rollout_value_advantages(token_traj, mask, values, rewards, ws, adv_out=N
                                            _ptr(adv_out), _ptr(returns_out), _ptr(ws), ws.numel(), _stream(stream))
     _check("rl_rollout_value_advantages", st)
     return adv_out, returns_out
+
+
+def rl_token_stats_summary(token_stats, mask, token_traj, coef, ws, summary_accum=None, stream=None):
+    """Adds (trained tokens, clipped, sum H, sum KL, sum rho) over the trained tokens to
+    ``summary_accum`` (float64 [5], created if None) and returns it."""
+    rows = mask.numel()
+    n_traj = coef.numel()
+    dev = mask.device
+    _need(token_stats, "token_stats", torch.float32, rows * 5, device=dev)
+    _need(mask, "mask", torch.uint8, rows, device=dev)
+    _need(token_traj, "token_traj", torch.int32, rows, device=dev)
+    _need(coef, "coef", torch.float32, n_traj, device=dev)
+    if summary_accum is None:
+        summary_accum = torch.zeros(5, dtype=torch.float64, device=dev)
+    _need(summary_accum, "summary_accum", torch.float64, 5, device=dev)
+    _need(ws, "ws", torch.uint8, device=dev)
+    st = lib().rl_token_stats_summary(rows, _ptr(token_stats), _ptr(mask), _ptr(token_traj), n_traj, _ptr(coef),
+                                      _ptr(summary_accum), _ptr(ws), ws.numel(), _stream(stream))
+    _check("rl_token_stats_summary", st)
+    return summary_accum

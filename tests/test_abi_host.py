@@ -257,3 +257,13 @@ def test_owner_and_tree_argument_checks(R):
     assert L.rl_prefix_tree_build_batch(2, ptr(bad), ptr(np.zeros(4, np.int32)), ptr(co), ptr(np.zeros(1, np.int64)),
                                         None, ptr(np.zeros(1, np.int64)), None, None, 0, 1, 0,
                                         *([None] * 11), ctypes.byref(n_tok)) == 1
+
+
+
+def test_stats_summary_argument_checks(R):
+    L = R.lib()
+    assert L.rl_token_stats_summary(-1, FAKE, FAKE, FAKE, 2, FAKE, FAKE, FAKE, 1024, None) == 1
+    assert L.rl_token_stats_summary(10, FAKE, FAKE, FAKE, 2, FAKE, None, FAKE, 1024, None) == 1
+    assert L.rl_token_stats_summary(10, FAKE, FAKE, FAKE, 2, FAKE, FAKE, FAKE, 16, None) == 4
+    assert L.rl_token_stats_summary(10, None, FAKE, FAKE, 2, FAKE, FAKE, FAKE, 1024, None) == 1
+    assert L.rl_token_stats_summary(0, None, None, None, 0, None, FAKE, FAKE, 1024, None) == 0

@@ -40,13 +40,21 @@ def run_loss(R, case, adv32=None, coef32=None, ld=None, in_place=False, stats=Tr
     coef32 = case.coef64.astype(np.float32) if coef32 is None else coef32
     ws = R.new_workspace(case.rows, case.raw.shape[1]) if ws is None else ws
     loss = torch.zeros(1, dtype=torch.float64, device=dev)
-    st = torch.zeros(case.rows * 5, dtype=torch.float32, device=dev) if stats else None
+    st = torch.full((case.rows * 5,), float("nan"), dtype=torch.float32, device=dev) if stats else None
+    # the gradient buffer starts as NaN everywhere (padding columns included): an element the
+    # library should write and does not stays NaN and fails the comparison
+    poison = torch.full_like(logits, float("nan")) if logits.is_contiguous() else None
+    if not in_place and poison is None:
+        full = torch.full((case.rows, logits.stride(0)), float("nan"), dtype=logits.dtype, device=dev)
+        poison = full[:, :logits.shape[1]]
     g = R.rl_policy_loss_fwd_bwd(logits, to_dev(case.ids), to_dev(case.mask), to_dev(case.tt.astype(np.int32)),
                                  to_dev(adv32), to_dev(coef32), to_dev(case.old), cuda_params(R, case.P), ws, loss,
-                                 grad_out=logits if in_place else None,
+                                 grad_out=logits if in_place else poison,
                                  ref_logp=None if case.ref is None else to_dev(case.ref),
                                  rollout_logp=None if case.roll is None else to_dev(case.roll), token_stats=st)
     status, word = R.rl_query_status(ws)
+    if not in_place and not logits.is_contiguous():  # columns past V are never written
+        assert torch.isnan(full[:, logits.shape[1]:]).all()
     return dict(loss=float(loss.item()), grad=grad_to_np(g), stats=None if st is None else st.view(-1, 5).cpu().numpy(),
                 status=status, word=word)
 
@@ -300,3 +308,54 @@ def test_token_logprobs_neg_inf_logits(R, name):
     assert np.all(np.abs(lp - lp_ref) <= 1e-5 + 2.0 ** -22 * np.abs(lp_ref)), np.abs(lp - lp_ref).max()
     assert np.all(np.abs(ls - lse_ref) <= 1e-5 + 2.0 ** -22 * np.abs(lse_ref)), np.abs(ls - lse_ref).max()
     assert np.all(np.abs(Hd - H_ref) <= 5e-5 + 2e-5 * np.abs(H_ref)), np.abs(Hd - H_ref).max()
+
+
+
+# ----------------------------------------------------------------------------- NaN logits, batch summaries
+
+def test_nan_logits_stay_in_their_rows(R):
+    """A NaN logit makes its own row's loss term and gradient NaN and nothing else: every other
+    row matches the oracle, and the loss (a sum over rows) is NaN."""
+    case = make_case("multiturn", seed=8, row0=2000, rows=40)
+    raw = case.raw.copy()
+    bad = [int(r) for r in np.nonzero((case.mask != 0) & (case.coef64[case.tt] != 0))[0][:3]]
+    for r in bad:
+        raw[r, (case.ids[r] + 11) % raw.shape[1]] = np.uint16(0x7FC0)  # bf16 NaN
+    c2 = dataclasses.replace(case, raw=raw)
+    out = run_loss(R, c2)
+    assert np.isnan(out["loss"])
+    ok = np.ones(case.rows, bool)
+    ok[bad] = False
+    assert np.isnan(out["grad"][bad]).any(axis=1).all()
+    adv32 = case.adv64.astype(np.float32).astype(np.float64)
+    coef32 = case.coef64.astype(np.float32).astype(np.float64)
+    rows = np.nonzero(ok)[0]
+    _, g_ref, st_ref, _ = O.policy_loss_fwd_bwd(case.raw, case.w.dtype, case.ids, case.mask, case.tt, adv32, coef32,
+                                                case.old, case.P, case.ref, case.roll, rows=rows)
+    check_grad(out["grad"][rows], g_ref, case.w.dtype, "rows without NaN")
+
+
+def test_stats_summary(R):
+    """Summaries of the loss call's statistics: counts exact, sums equal the float64 sum of the
+    same float32 values (order-independent to 1e-12), and within the statistics' own tolerances
+    of the oracle's summary."""
+    case = make_case("longhorizon", seed=9, row0=3000, rows=96, tis=True)
+    out = run_loss(R, case)
+    st_dev = torch.from_numpy(out["stats"].reshape(-1).astype(np.float32)).cuda()
+    coef32 = case.coef64.astype(np.float32)
+    ws = R.new_workspace(0, 0)
+    acc = R.rl_token_stats_summary(st_dev, to_dev(case.mask), to_dev(case.tt.astype(np.int32)), to_dev(coef32), ws)
+    acc = R.rl_token_stats_summary(st_dev, to_dev(case.mask), to_dev(case.tt.astype(np.int32)), to_dev(coef32), ws,
+                                   summary_accum=acc)  # accumulates
+    assert R.rl_query_status(ws)[1] == 0
+    got = acc.cpu().numpy() / 2
+    mine = O.stats_summary(out["stats"].astype(np.float64), case.mask, case.tt, coef32)
+    assert got[0] == mine[0] and got[1] == mine[1]
+    assert np.allclose(got[2:], mine[2:], rtol=1e-12, atol=1e-12)
+    _, _, st_ref, _ = oracle_loss(case, case.adv64.astype(np.float32).astype(np.float64),
+                                  coef32.astype(np.float64), want_grad=False)
+    ref = O.stats_summary(st_ref, case.mask, case.tt, coef32)
+    assert got[0] == ref[0] and got[1] == ref[1]
+    act = (case.mask != 0) & (coef32[case.tt] != 0)
+    tolH = float((5e-5 + 2e-5 * np.abs(st_ref[act, 3])).sum())
+    assert abs(got[2] - ref[2]) <= tolH and abs(got[4] - ref[4]) <= float((2e-5 * st_ref[act, 1]).sum())
