@@ -182,6 +182,8 @@ rl_status rl_token_logprobs(const void* logits, rl_dtype dtype, int64_t rows, in
  *   g = -w A rho act + beta (1 - exp(r - logp)), act = 0 iff
  *   (A > 0 and rho > 1 + eps_high) or (A < 0 and rho < 1 - eps_low).
  * Every other row gets an exactly-zero gradient row and contributes nothing.
+ * Logits at -inf have probability 0 (and a zero gradient); a NaN logit makes its own row's
+ * loss term, statistics and gradient NaN (so the loss is NaN) and leaves the other rows alone.
  *
  *   logits        [rows x ld] of `dtype`, base 16-byte aligned
  *   rows, V, ld   rows >= 0, 1 <= V <= ld

@@ -141,13 +141,18 @@ struct Vec<float> {
 };
 
 #define RL_NEG_INF (-__int_as_float(0x7f800000))
+
+// Pass 1: -inf (and anything below -1e30) becomes -1e30, so that e = 0 and e (z - m) = 0
+// instead of NaN; a NaN stays NaN (a comparison, not fmaxf, which would drop it) and poisons
+// its row. Pass 2 clamps with fmaxf: there p = 2^(NaN) is NaN already.
+__device__ __forceinline__ float clamp_ninf(float z) { return z < -1e30f ? -1e30f : z; }
 constexpr uint32_t kBulkChunk = 32768;
 
 // fold one value into a per-thread online-softmax partial whose max is already >= z
 template <bool ENT>
 __device__ __forceinline__ void accumulate(SoftmaxPartial& ps, float z, float neg_m_l2e) {
   if (ENT) {
-    const float t = fmaxf(z, -1e30f) - ps.m;  // -inf logits contribute 0, not NaN
+    const float t = clamp_ninf(z) - ps.m;  // -inf logits contribute 0, not NaN
     const float e = ex2(t * kLog2e);
     ps.s += e;
     ps.u = fmaf(e, t, ps.u);
@@ -222,7 +227,7 @@ __device__ __forceinline__ void fold(SoftmaxPartial& ps, const float (&v)[EPV]) 
 #pragma unroll
     for (int k = 0; k < EPV; ++k) {
       if (ENT) {
-        t[k] = fmaxf(v[k], -1e30f) - ps.m;  // -inf logits contribute 0, not NaN
+        t[k] = clamp_ninf(v[k]) - ps.m;  // -inf logits contribute 0, not NaN
         e[k] = ex2(t[k] * kLog2e);
       } else {
         e[k] = ex2(fmaf(v[k], kLog2e, nm));
@@ -290,8 +295,9 @@ __device__ __forceinline__ void fold_block(SoftmaxPartial& ps, const uint4 (&x)[
   // x = (z - m) log2(e) by one fused multiply-add against nm = fl(-m log2(e)); with the
   // entropy, u accumulates e x (log2 units, scaled by ln 2 at the end). A logit at -inf gives
   // e = 0 and e x = NaN: such a block is redone on the clamped path (CLAMP), where z counts as
-  // -1e30. The rounding of nm shifts every x of the block by the same err = -m log2(e) - nm
-  // (exact by one fma); the block's sums are corrected for it once at the end.
+  // -1e30 (a NaN stays NaN). The rounding of nm shifts every x of the block by the same
+  // err = -m log2(e) - nm (exact by one fma); the block's sums are corrected for it once at
+  // the end.
   auto exps = [&](auto clamp, const uint4 w, float2& s0, float2& s1, float2& u0) {
     constexpr bool CLAMP = decltype(clamp)::value;
     const float nm = -ps.m * kLog2e;
@@ -300,7 +306,7 @@ __device__ __forceinline__ void fold_block(SoftmaxPartial& ps, const uint4 (&x)[
     Vec<T>::pairs(w, q);
 #pragma unroll
     for (int i = 0; i < NP; ++i) {
-      const float2 qi = CLAMP ? make_float2(fmaxf(q[i].x, -1e30f), fmaxf(q[i].y, -1e30f)) : q[i];
+      const float2 qi = CLAMP ? make_float2(clamp_ninf(q[i].x), clamp_ninf(q[i].y)) : q[i];
       const float2 xx = __ffma2_rn(qi, l2, nm2);
       const float2 e = make_float2(ex2(xx.x), ex2(xx.y));
       if (i & 1) s1 = __fadd2_rn(s1, e); else s0 = __fadd2_rn(s0, e);
