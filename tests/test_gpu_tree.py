@@ -124,3 +124,27 @@ def test_tree_sequence_weights(R, packed):
     w_ref, _ = O.sequence_is_weights(out["owner"], out["mask"], old, roll, n, 3.0)
     n_i = np.bincount(out["owner"][out["mask"] != 0], minlength=n)
     assert np.all(np.abs(wt.cpu().numpy() - w_ref) <= (n_i * 2.0 ** -40 + 2.0 ** -23) * w_ref + 1e-30)
+
+
+def test_full_tree_workload_by_owner(R):
+    """The benchmark's tree batch (128 rollouts, 652K packed tokens): counts by owner bit-exact
+    against the oracle, A_i and c_i within one float32 rounding, sequence weights too."""
+    w = W.WORKLOADS["tree"]
+    prompts, calls, aux = W.tree_rollouts(w, seed=0)
+    out = R.rl_prefix_tree_build_batch(prompts, calls, aux, max_leaves=w.tree_max_leaves)
+    n = len(prompts)
+    rewards = (np.random.default_rng(0).random(n) < w.reward_p).astype(np.float32)
+    valid = np.array([s["valid"] for s in out["stats"]], np.uint8)
+    go = np.arange(0, n + 1, w.group_size, dtype=np.int32)
+    P = O.LossParams(loss_agg=0)
+    ws = R.new_workspace(n, 0)
+    adv, coef, L = R.rl_group_advantages_by_owner(to_dev(go), to_dev(rewards), to_dev(out["owner"]),
+                                                  to_dev(out["mask"]), cuda_params(R, P), ws,
+                                                  traj_valid=to_dev(valid))
+    assert R.rl_query_status(ws)[1] == 0
+    L_ref = np.bincount(out["owner"][out["mask"] != 0], minlength=n)  # plain count by owner
+    assert np.array_equal(L.cpu().numpy(), L_ref)
+    a_ref, c_ref, L2 = PT.advantages_and_coefficients_by_owner(rewards, go, out["owner"], out["mask"], n, valid, P)
+    assert np.array_equal(L2, L_ref)
+    assert _ulp_close(adv.cpu().numpy().astype(np.float64), a_ref)
+    assert _ulp_close(coef.cpu().numpy().astype(np.float64), c_ref)
