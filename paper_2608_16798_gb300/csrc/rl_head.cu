@@ -608,6 +608,9 @@ size_t head_workspace_bytes(int64_t max_rows, int64_t V, int64_t D) {
 
 // The forward-only call needs the status word and one chunk's partials, which sit at the
 // same offset as in the loss layout's header; rl_workspace_size(T, V, D) always suffices.
+// It keeps the loss call's chunk of 8,192 tokens: the chunk's hidden states (64 MB at
+// D = 4,096) and one 4,096-entry block of W (32 MB) then stay in L2 together; with chunks
+// of 32,768 tokens the hidden states (256 MB) evict W's tiles and the call took 22% longer.
 static size_t head_logp_workspace_bytes(int64_t T, int64_t V) {
   const head::Layout L = head::layout(T, V);
   return kWsHeader + head::al256(static_cast<size_t>(L.n_vb * L.Tc) * sizeof(float4));
