@@ -780,7 +780,7 @@ def time_head(torch, R, dev, warmup=2, reps=5):
         burst, sustained, kind = float(pk["bf16_tflops"]), float(pk["bf16_tflops_sustained"]), "measured"
     flops = 6.0 * hb.T * hb.D * hb.V
     tf = flops / (ms * 1e-3) / 1e12
-    chunks = (hb.T + 8191) // 8192
+    chunks = (hb.T + 4095) // 4096
     tf_fwd = 2.0 * hb.T * hb.D * hb.V / (ms_fwd * 1e-3) / 1e12
     fwd = {"ms_per_call": ms_fwd, "tokens_per_s": hb.T / (ms_fwd * 1e-3), "achieved": tf_fwd, "frac": tf_fwd / burst,
            "frac_of_sustained": tf_fwd / sustained, "algorithmic_flops_per_call": 2.0 * hb.T * hb.D * hb.V,

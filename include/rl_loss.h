@@ -102,7 +102,7 @@ const char* rl_last_error_message(void);
  * vocabulary V (D = hidden size of the fused head, 0 if unused). The
  * workspace holds the device status word and per-row loss contributions; with
  * D > 0 it also holds the fused head's per-chunk buffers (about
- * min(max_rows, 8192) * V * 2 bytes plus 32 MiB). */
+ * min(max_rows, 4096) * V * 2 bytes plus 32 MiB). */
 size_t rl_workspace_size(int64_t max_rows, int64_t V, int64_t D);
 
 /* Zero the workspace's status word. Call once after allocating a workspace,
@@ -231,9 +231,9 @@ rl_status rl_policy_loss_fwd_bwd(const void* logits, rl_dtype dtype, int64_t row
  *                 (overwritten; zero rows for tokens that are not trained on)
  *   d_weight      float [V x D]: d loss / d W is ADDED to it
  *   ws, ws_bytes  workspace of at least rl_workspace_size(T, V, D) bytes; it holds,
- *                 among others, the gradient of the logits for one chunk of 8,192
+ *                 among others, the gradient of the logits for one chunk of 4,096
  *                 tokens (bf16), consumed by the dH and dW products of that chunk
- * Tokens are processed in chunks of 8,192: per chunk, a tensor-core pass forms the
+ * Tokens are processed in chunks of 4,096: per chunk, a tensor-core pass forms the
  * softmax statistics, a second pass recomputes the logits and forms their gradient,
  * and two GEMMs (cuBLASLt) produce dH and accumulate dW.
  */
@@ -406,9 +406,9 @@ rl_status rl_sequence_is_weights(int32_t n_traj, int64_t n_tokens, const int32_t
  *   entropy_out  float [T] or NULL (entropy work is skipped when NULL)
  *   lse_out      float [T] or NULL
  *   ws, ws_bytes workspace; rl_workspace_size(T, V, D) bytes always suffice (the
- *                call uses the status word and 16 * ceil(V / 4096) * min(T, 8192)
+ *                call uses the status word and 16 * ceil(V / 4096) * min(T, 4096)
  *                bytes of per-block softmax partials after it)
- * One tensor-core pass per chunk of 8,192 tokens, then a per-token merge of the
+ * One tensor-core pass per chunk of 4,096 tokens, then a per-token merge of the
  * vocabulary blocks' partials in fixed order (deterministic).
  */
 rl_status rl_fused_head_token_logprobs(const void* hidden, const void* weight, int64_t T, int64_t D, int64_t V,

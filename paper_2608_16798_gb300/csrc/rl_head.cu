@@ -41,7 +41,10 @@ constexpr int VB_TILES = 16;       // N tiles per work item (a vocabulary block 
 constexpr uint32_t A_BYTES = BM * BK * 2, B_BYTES = BN * BK * 2, STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int kThreads = 192;      // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
 constexpr size_t kSmem = NS * STAGE_BYTES + 1024;
-constexpr int64_t kChunk = 8192;   // tokens per chunk
+#ifndef RL_HEAD_CHUNK
+#define RL_HEAD_CHUNK 4096
+#endif
+constexpr int64_t kChunk = RL_HEAD_CHUNK;  // tokens per chunk (tuning knob, compile time)
 constexpr size_t kLtWorkspace = 32u << 20;
 
 enum Mode { STATS = 0, STATS_P = 1 };
@@ -608,9 +611,11 @@ size_t head_workspace_bytes(int64_t max_rows, int64_t V, int64_t D) {
 
 // The forward-only call needs the status word and one chunk's partials, which sit at the
 // same offset as in the loss layout's header; rl_workspace_size(T, V, D) always suffices.
-// It keeps the loss call's chunk of 8,192 tokens: the chunk's hidden states (64 MB at
-// D = 4,096) and one 4,096-entry block of W (32 MB) then stay in L2 together; with chunks
-// of 32,768 tokens the hidden states (256 MB) evict W's tiles and the call took 22% longer.
+// It keeps the loss call's chunk of 4,096 tokens: the chunk's hidden states (32 MB at
+// D = 4,096) and the W tiles in use then stay in L2 together. Measured at 32,768 x 4,096 x
+// 151,936: chunks of 4,096 tokens give 24.8 ms per forward-only call (70.9 ms per loss call),
+// 3,072 and 6,144 are within 2%, 8,192 takes 26.7 ms (73.1), and 32,768 takes 31.5 ms: the
+// hidden states (256 MB) then evict W's tiles from the 129 MB L2.
 static size_t head_logp_workspace_bytes(int64_t T, int64_t V) {
   const head::Layout L = head::layout(T, V);
   return kWsHeader + head::al256(static_cast<size_t>(L.n_vb * L.Tc) * sizeof(float4));

@@ -166,8 +166,8 @@ def test_fused_head_logprobs_argument_checks(R):
     # (logp=None makes a call that passed the workspace check stop at the next one)
     big = dict(T=20000, V=151936, logp=None)
     assert call(ws_bytes=R.rl_workspace_size(20000, 151936, 4096), **big) == 1
-    assert call(ws_bytes=256 + 16 * 38 * 8192, **big) == 1
-    assert call(ws_bytes=256 + 16 * 38 * 8192 - 1, **big) == 4
+    assert call(ws_bytes=256 + 16 * 38 * 4096, **big) == 1
+    assert call(ws_bytes=256 + 16 * 38 * 4096 - 1, **big) == 4
 
 
 def test_masked_gae_argument_checks(R):

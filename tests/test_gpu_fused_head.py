@@ -132,7 +132,7 @@ def test_fused_head_parity(R, T, D, V, agg, ent, tis):
 
 
 def test_fused_head_two_chunks_bf16_grad(R):
-    """More than 8,192 tokens: two chunks, dW accumulated across them; bf16 d_hidden."""
+    """More than 8,192 tokens: three chunks of 4,096, dW accumulated across them; bf16 d_hidden."""
     c = make_head_case(8192 + 77, 128, 1100, seed=5, agg=2)
     out = run_head(R, c, dh_dtype=torch.bfloat16)
     compare_head(c, out, dh_bf16=True)
@@ -189,7 +189,7 @@ def run_logprobs(R, c, want_entropy=True, ids=None):
     (300, 256, 1000),        # ragged M tile and vocabulary tile
     (256, 128, 8292),        # three vocabulary blocks, ragged last block
     (130, 64, 513),          # smallest D
-    (8192 + 77, 128, 1100),  # two chunks
+    (8192 + 77, 128, 1100),  # three chunks
 ])
 def test_fused_head_logprobs_parity(R, T, D, V):
     c = make_head_case(T, D, V, seed=3 * T + V)
