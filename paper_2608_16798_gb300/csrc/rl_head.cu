@@ -37,7 +37,10 @@ constexpr int BM = 128;            // tokens per tile (TMEM lanes)
 constexpr int BN = 256;            // vocabulary entries per tile (TMEM columns per accumulator)
 constexpr int BK = 64;             // hidden elements per stage (one 128-byte swizzle row)
 constexpr int NS = 4;              // shared-memory stages
-constexpr int VB_TILES = 16;       // N tiles per work item (a vocabulary block of 4,096)
+#ifndef RL_HEAD_VB_TILES
+#define RL_HEAD_VB_TILES 16
+#endif
+constexpr int VB_TILES = RL_HEAD_VB_TILES;  // N tiles per work item (16: a vocabulary block of 4,096)
 constexpr uint32_t A_BYTES = BM * BK * 2, B_BYTES = BN * BK * 2, STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int kThreads = 192;      // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
 constexpr size_t kSmem = NS * STAGE_BYTES + 1024;
