@@ -223,7 +223,8 @@ rl_status rl_policy_loss_fwd_bwd(const void* logits, rl_dtype dtype, int64_t row
  *
  *   hidden        bf16 [T x D], row-major, 16-byte aligned
  *   weight        bf16 [V x D], row-major (row v = output embedding of token v)
- *   T, D, V       T >= 0, D >= 64 and a multiple of 64, V >= 1
+ *   T, D, V       T >= 0, D >= 64 and a multiple of 64 (at most 65,536), 1 <= V <= 524,288
+ *                 (RL_ERR_UNSUPPORTED otherwise)
  *   token_ids, mask, token_traj, n_traj, adv, coef, old_logp, ref_logp,
  *   rollout_logp, params, loss_accum, token_stats
  *                 as for rl_policy_loss_fwd_bwd, with one row per token

@@ -267,3 +267,20 @@ def test_stats_summary_argument_checks(R):
     assert L.rl_token_stats_summary(10, FAKE, FAKE, FAKE, 2, FAKE, FAKE, FAKE, 16, None) == 4
     assert L.rl_token_stats_summary(10, None, FAKE, FAKE, 2, FAKE, FAKE, FAKE, 1024, None) == 1
     assert L.rl_token_stats_summary(0, None, None, None, 0, None, FAKE, FAKE, 1024, None) == 0
+
+
+
+def test_fused_head_loss_shape_limits(R):
+    L = R.lib()
+    p = _params(R)
+    loss = FAKE
+
+    def call(T=16, D=128, V=1000):
+        return L.rl_fused_head_loss_fwd_bwd(FAKE, FAKE, T, D, V, FAKE, FAKE, FAKE, 2, FAKE, FAKE, FAKE, None, None, p,
+                                            FAKE, R.RL_BF16, FAKE, loss, None, FAKE, 1 << 40, None)
+
+    assert call(D=96) == 2          # not a multiple of 64
+    assert call(D=32) == 1
+    assert call(V=524_289) == 2     # above the fix-up kernel's shared-memory tile factors
+    assert call(D=65_600) == 2
+    assert call(T=-1) == 1
