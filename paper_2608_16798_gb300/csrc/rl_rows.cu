@@ -382,79 +382,105 @@ __global__ void __launch_bounds__((NW + 1) * 32, 2) rows_kernel(const RowArgs p)
 
   if (warp == NW) {
     // =============================================================== producer warp
+    // Row metadata is fetched 32 rows at a time, one row per lane (independent loads, one
+    // latency per batch), then handed row by row to the staging loop with shuffles.
     uint32_t it = 0;
     bool failed = false, stored = false;
-    for (int64_t r = cid; r < rows && !failed; r += ncl) {
-      RowMeta m;
-      bool active = true;
-      m.r = r;
-      m.a = p.token_ids[r];
-      if (BWD) {
-        active = p.mask[r] != 0;
-        if (active) {
-          const int32_t i = p.token_traj[r];
-          if (i < 0 || i >= p.n_traj) {
-            if (rank == 0 && lane == 0) flag_status(p.status, RL_DEV_BAD_TRAJ);
-            active = false;
-          } else {
-            m.c = p.coef[i];
-            m.A = p.adv_per_row ? p.adv[r] : p.adv[i];
-            active = m.c != 0.f;
-            if (active && (m.a < 0 || m.a >= V)) {
-              if (rank == 0 && lane == 0) flag_status(p.status, RL_DEV_BAD_TOKEN);
+    for (int64_t base = cid; base < rows && !failed; base += 32 * ncl) {
+      const int64_t my = base + static_cast<int64_t>(lane) * ncl;
+      const bool have = my < rows;
+      int32_t la = 0, li = -1;
+      uint32_t lm = 0;
+      float lc = 0.f, lA = 0.f, lold = 0.f, lref = 0.f, lroll = 0.f;
+      if (have) {
+        la = p.token_ids[my];
+        if (BWD) {
+          lm = p.mask[my];
+          li = p.token_traj[my];
+          lold = p.old_logp[my];
+          if (p.ref_logp) lref = p.ref_logp[my];
+          if (p.rollout_logp) lroll = p.rollout_logp[my];
+          if (p.adv_per_row) lA = p.adv[my];
+        }
+      }
+      if (BWD && have && lm != 0 && li >= 0 && li < p.n_traj) {
+        lc = p.coef[li];
+        if (!p.adv_per_row) lA = p.adv[li];
+      }
+      const int nb = static_cast<int>(min(static_cast<int64_t>(32), (rows - base + ncl - 1) / ncl));
+      for (int jr = 0; jr < nb && !failed; ++jr) {
+        const int64_t r = base + static_cast<int64_t>(jr) * ncl;
+        RowMeta m;
+        bool active = true;
+        m.r = r;
+        m.a = __shfl_sync(0xffffffffu, la, jr);
+        if (BWD) {
+          active = __shfl_sync(0xffffffffu, lm, jr) != 0;
+          if (active) {
+            const int32_t i = __shfl_sync(0xffffffffu, li, jr);
+            if (i < 0 || i >= p.n_traj) {
+              if (rank == 0 && lane == 0) flag_status(p.status, RL_DEV_BAD_TRAJ);
               active = false;
+            } else {
+              m.c = __shfl_sync(0xffffffffu, lc, jr);
+              m.A = __shfl_sync(0xffffffffu, lA, jr);
+              active = m.c != 0.f;
+              if (active && (m.a < 0 || m.a >= V)) {
+                if (rank == 0 && lane == 0) flag_status(p.status, RL_DEV_BAD_TOKEN);
+                active = false;
+              }
             }
           }
-        }
-        if (!active) {
-          // zero this CTA's slice of gradient row r
-          T* g = grad + r * ld + s0;
-          if (p.tma) {
-            if (lane == 0) {
-              const uint32_t bytes = tma_bytes;
-              for (uint32_t off = 0; off < bytes; off += kZeroBytes)
-                bulk_s2g(reinterpret_cast<char*>(g) + off, zeros, min(static_cast<uint32_t>(kZeroBytes), bytes - off));
-              bulk_commit();
-              stored = true;
+          if (!active) {
+            // zero this CTA's slice of gradient row r
+            T* g = grad + r * ld + s0;
+            if (p.tma) {
+              if (lane == 0) {
+                const uint32_t bytes = tma_bytes;
+                for (uint32_t off = 0; off < bytes; off += kZeroBytes)
+                  bulk_s2g(reinterpret_cast<char*>(g) + off, zeros, min(static_cast<uint32_t>(kZeroBytes), bytes - off));
+                bulk_commit();
+                stored = true;
+              }
+              for (int e = nv * EPV + lane; e < n; e += 32) g[e] = T(0);
+            } else {
+              for (int e = lane; e < n; e += 32) g[e] = T(0);
             }
-            for (int e = nv * EPV + lane; e < n; e += 32) g[e] = T(0);
+            if (rank == 0 && lane == 0) {
+              p.row_loss[r] = 0.0;
+              if (p.token_stats)
+                for (int k = 0; k < 5; ++k) p.token_stats[r * 5 + k] = 0.f;
+            }
+            continue;
+          }
+          m.old = __shfl_sync(0xffffffffu, lold, jr);
+          m.ref = __shfl_sync(0xffffffffu, lref, jr);
+          m.roll = __shfl_sync(0xffffffffu, lroll, jr);
+        }
+        const int b = it % NB;
+        const uint32_t use = it / NB;
+        if (use > 0 && !mbar_wait_bounded(&empty_bar[b], (use - 1) & 1)) {
+          failed = true;
+          if (lane == 0) flag_status(p.status, RL_DEV_TIMEOUT);
+          break;
+        }
+        T* buf = buf_base + b * p.buf_elems;
+        const T* src = logits + r * ld + s0;
+        for (int e = first_scalar + lane; e < n; e += 32) buf[e] = src[e];
+        __syncwarp();
+        if (lane == 0) {
+          meta[b] = m;
+          if (tma_bytes > 0) {
+            mbar_arrive_expect_tx(&full_bar[b], tma_bytes);
+            for (uint32_t off = 0; off < tma_bytes; off += kBulkChunk)
+              bulk_g2s(reinterpret_cast<char*>(buf) + off, reinterpret_cast<const char*>(src) + off,
+                       min(kBulkChunk, tma_bytes - off), &full_bar[b]);
           } else {
-            for (int e = lane; e < n; e += 32) g[e] = T(0);
+            mbar_arrive(&full_bar[b]);
           }
-          if (rank == 0 && lane == 0) {
-            p.row_loss[r] = 0.0;
-            if (p.token_stats)
-              for (int k = 0; k < 5; ++k) p.token_stats[r * 5 + k] = 0.f;
-          }
-          continue;
         }
-        m.old = p.old_logp[r];
-        m.ref = p.ref_logp ? p.ref_logp[r] : 0.f;
-        m.roll = p.rollout_logp ? p.rollout_logp[r] : 0.f;
+        ++it;
       }
-      const int b = it % NB;
-      const uint32_t use = it / NB;
-      if (use > 0 && !mbar_wait_bounded(&empty_bar[b], (use - 1) & 1)) {
-        failed = true;
-        if (lane == 0) flag_status(p.status, RL_DEV_TIMEOUT);
-        break;
-      }
-      T* buf = buf_base + b * p.buf_elems;
-      const T* src = logits + r * ld + s0;
-      for (int e = first_scalar + lane; e < n; e += 32) buf[e] = src[e];
-      __syncwarp();
-      if (lane == 0) {
-        meta[b] = m;
-        if (tma_bytes > 0) {
-          mbar_arrive_expect_tx(&full_bar[b], tma_bytes);
-          for (uint32_t off = 0; off < tma_bytes; off += kBulkChunk)
-            bulk_g2s(reinterpret_cast<char*>(buf) + off, reinterpret_cast<const char*>(src) + off,
-                     min(kBulkChunk, tma_bytes - off), &full_bar[b]);
-        } else {
-          mbar_arrive(&full_bar[b]);
-        }
-      }
-      ++it;
     }
     if (!failed) {
       // end of stream
