@@ -382,33 +382,51 @@ __global__ void __launch_bounds__((NW + 1) * 32, 2) rows_kernel(const RowArgs p)
 
   if (warp == NW) {
     // =============================================================== producer warp
-    // Row metadata is fetched 32 rows at a time, one row per lane (independent loads, one
-    // latency per batch), then handed row by row to the staging loop with shuffles.
+    // Row metadata is fetched 32 rows at a time, one row per lane, and handed row by row to the
+    // staging loop with shuffles. The loads of the next batch are issued while the current one
+    // is staged (its owners' coefficients once the owners have arrived), so their latency is
+    // hidden behind the copies.
     uint32_t it = 0;
     bool failed = false, stored = false;
-    for (int64_t base = cid; base < rows && !failed; base += 32 * ncl) {
-      const int64_t my = base + static_cast<int64_t>(lane) * ncl;
-      const bool have = my < rows;
-      int32_t la = 0, li = -1;
-      uint32_t lm = 0;
-      float lc = 0.f, lA = 0.f, lold = 0.f, lref = 0.f, lroll = 0.f;
-      if (have) {
-        la = p.token_ids[my];
+    struct Batch {
+      int32_t a, i;
+      uint32_t m;
+      float c, A, old, ref, roll;
+    };
+    auto load_primary = [&](int64_t b0, Batch& q) {
+      const int64_t my = b0 + static_cast<int64_t>(lane) * ncl;
+      q = Batch{0, -1, 0u, 0.f, 0.f, 0.f, 0.f, 0.f};
+      if (my < rows) {
+        q.a = p.token_ids[my];
         if (BWD) {
-          lm = p.mask[my];
-          li = p.token_traj[my];
-          lold = p.old_logp[my];
-          if (p.ref_logp) lref = p.ref_logp[my];
-          if (p.rollout_logp) lroll = p.rollout_logp[my];
-          if (p.adv_per_row) lA = p.adv[my];
+          q.m = p.mask[my];
+          q.i = p.token_traj[my];
+          q.old = p.old_logp[my];
+          if (p.ref_logp) q.ref = p.ref_logp[my];
+          if (p.rollout_logp) q.roll = p.rollout_logp[my];
+          if (p.adv_per_row) q.A = p.adv[my];
         }
       }
-      if (BWD && have && lm != 0 && li >= 0 && li < p.n_traj) {
-        lc = p.coef[li];
-        if (!p.adv_per_row) lA = p.adv[li];
+    };
+    auto load_dependent = [&](Batch& q) {
+      if (BWD && q.m != 0 && q.i >= 0 && q.i < p.n_traj) {
+        q.c = p.coef[q.i];
+        if (!p.adv_per_row) q.A = p.adv[q.i];
       }
+    };
+    Batch cur, nxt = Batch{0, -1, 0u, 0.f, 0.f, 0.f, 0.f, 0.f};
+    load_primary(cid, cur);
+    load_dependent(cur);
+    for (int64_t base = cid; base < rows && !failed; base += 32 * ncl) {
+      const int64_t next_base = base + 32 * ncl;
+      const bool has_next = next_base < rows;
+      if (has_next) load_primary(next_base, nxt);
+      const int32_t la = cur.a, li = cur.i;
+      const uint32_t lm = cur.m;
+      const float lc = cur.c, lA = cur.A, lold = cur.old, lref = cur.ref, lroll = cur.roll;
       const int nb = static_cast<int>(min(static_cast<int64_t>(32), (rows - base + ncl - 1) / ncl));
       for (int jr = 0; jr < nb && !failed; ++jr) {
+        if (jr == 1 && has_next) load_dependent(nxt);  // the next batch's owners have arrived by now
         const int64_t r = base + static_cast<int64_t>(jr) * ncl;
         RowMeta m;
         bool active = true;
@@ -481,6 +499,8 @@ __global__ void __launch_bounds__((NW + 1) * 32, 2) rows_kernel(const RowArgs p)
         }
         ++it;
       }
+      if (has_next && nb <= 1) load_dependent(nxt);
+      cur = nxt;
     }
     if (!failed) {
       // end of stream
