@@ -856,6 +856,49 @@ def profile_case(rows):
     return 0 if word == 0 else 1
 
 
+def profile_ppo(steps):
+    """The PPO step of the benchmark on the whole multi-turn batch, `steps` times without timing
+    (for a profiler's launch list): advantages and coefficients, masked GAE, then per microbatch
+    the policy loss with per-token advantages and the value loss; then sequence-level weights."""
+    import torch
+
+    from paper_2608_16798_gb300 import build as B
+
+    B.build()
+    import paper_2608_16798_gb300.rl_loss as R
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    batch = DeviceBatch(torch, R, dev)
+    t = torch
+    d = lambda x: t.from_numpy(np.ascontiguousarray(x)).to(dev)  # noqa: E731
+    values = d(W.value_predictions(WORKLOAD, 0, batch.T))
+    v_new = values + 0.05
+    params = R.make_params(W.CLIP_EPS_LOW, W.CLIP_EPS_HIGH, 0.0, 0, 0.0, 0.0, 1e-6, 1, token_level_adv=1)
+    coef, adv_traj = t.empty_like(batch.coef), t.empty_like(batch.adv)
+    adv, ret, dv = (t.empty(batch.T, dtype=t.float32, device=dev) for _ in range(3))
+    loss, vloss = t.zeros(1, dtype=t.float64, device=dev), t.zeros(1, dtype=t.float64, device=dev)
+    roll = d(W.rollout_logp_from(batch.old.cpu().numpy(), 0, std=0.02))
+    w_seq = t.empty(batch.lay.n_traj, dtype=t.float32, device=dev)
+    for _ in range(steps):
+        R.rl_group_advantages(batch.group_offsets, batch.rewards, batch.traj_offsets, batch.mask, params, batch.ws,
+                              traj_valid=batch.valid, adv_out=adv_traj, coef_out=coef, n_tok_out=batch.n_tok,
+                              token_traj_out=batch.token_traj)
+        R.rl_masked_gae(batch.traj_offsets, batch.mask, values, batch.ws, 1.0, 1.0, True,
+                        traj_rewards=batch.rewards.float(), adv_out=adv, returns_out=ret)
+        for lo, hi in batch.mbs:
+            R.rl_policy_loss_fwd_bwd(batch.logits[lo:hi], batch.ids[lo:hi], batch.mask[lo:hi],
+                                     batch.token_traj[lo:hi], adv[lo:hi], coef, batch.old[lo:hi], params, batch.ws,
+                                     loss, grad_out=batch.grad[lo:hi])
+            R.rl_value_loss_fwd_bwd(v_new[lo:hi], ret[lo:hi], batch.mask[lo:hi], batch.token_traj[lo:hi], coef,
+                                    batch.ws, vloss, d_values=dv[lo:hi])
+        R.rl_sequence_is_weights(batch.token_traj, batch.mask, batch.old, roll, batch.lay.n_traj, batch.ws, cap=2.0,
+                                 weight_out=w_seq)
+    st, word = R.rl_query_status(batch.ws)
+    print(json.dumps({"profile_ppo_steps": steps, "tokens_per_step": batch.T, "status": word}))
+    return 0 if word == 0 else 1
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -869,6 +912,8 @@ def main():
                     help="run a small slice of the workload for a profiler capture and exit")
     ap.add_argument("--profile-head", type=int, default=0, metavar="TOKENS",
                     help="run a small fused-head case for a profiler capture and exit")
+    ap.add_argument("--profile-ppo", type=int, default=0, metavar="STEPS",
+                    help="run the PPO step on the batch STEPS times for a profiler's launch list and exit")
     ap.add_argument("--no-head", action="store_true", help="skip the fused-head measurement")
     ap.add_argument("--no-ppo", action="store_true", help="skip the PPO-step measurement")
     ap.add_argument("--no-tree", action="store_true", help="skip the prefix-tree measurement")
@@ -878,6 +923,8 @@ def main():
         return profile_case(args.profile_case)
     if args.profile_head:
         return profile_head(args.profile_head)
+    if args.profile_ppo:
+        return profile_ppo(args.profile_ppo)
     if args.impl == "reference":
         return run_reference(args)
     args.warmup = max(3, args.warmup)
