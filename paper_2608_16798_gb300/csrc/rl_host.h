@@ -13,7 +13,9 @@ namespace rl {
 
 // Workspace layout (offsets in bytes from the caller's workspace pointer):
 //   [0, 256)                 header: int32 device status word at offset 0
-//   [256, 256 + 8 * rows)    double per-row loss contributions c_i * l_t
+//   [256, 256 + 8 * rows)    double loss contributions: one per cluster of the logits-path
+//                            loss kernel (its rows' c_i * l_t added in row order), one per
+//                            row for the fused head and the value loss
 constexpr size_t kWsHeader = 256;
 
 inline size_t ws_row_loss_offset() { return kWsHeader; }
@@ -22,7 +24,7 @@ rl_status set_error(rl_status st, const std::string& msg);
 rl_status cuda_error(cudaError_t e, const char* what);
 void clear_error();
 
-// Fixed-order sum of per-row loss contributions into *loss_accum (rl_rows.cu).
+// Fixed-order sum of `rows` loss contributions into *loss_accum (rl_stats.cu).
 rl_status launch_reduce_loss(const double* row_loss, int64_t rows, double* loss_accum, cudaStream_t s);
 // Workspace of the fused LM head for up to max_rows tokens (rl_head.cu).
 size_t head_workspace_bytes(int64_t max_rows, int64_t V, int64_t D);

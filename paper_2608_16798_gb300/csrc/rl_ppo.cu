@@ -14,9 +14,9 @@
 //                                         Vn_{t+1} the value of the next trainable token,
 //                                         itself the suffix scan of the selection map
 //                                         x_t = M_t ? V_t : x_{t+1} (exact in fp32)
-//   value_loss_kernel  per token: c M (V - G)^2 into the per-row loss slots, and
-//                      dV = 2 c M (V - G); the fixed-order reduction of rl_rows.cu adds
-//                      the slots into the caller's accumulator.
+//   value_loss_kernel  per token: c M (V - G)^2, added per CTA in a fixed order into one
+//                      partial per CTA, and dV = 2 c M (V - G); the fixed-order reduction
+//                      adds the partials into the caller's accumulator.
 //   rollout_adv_kernel A_t = R_i - V_t, G_t = R_i per token for tokens in any order (the
 //                      gamma = lambda = 1 form of Sec. 2.3.4, which also holds on the shared
 //                      prefixes of a rollout's prefix tree).
@@ -197,7 +197,11 @@ struct ValueArgs {
   int32_t* status;
 };
 
+// Each CTA adds its rows' terms in a fixed order (thread-strided, then warp and CTA) and leaves
+// one partial per CTA in row_loss[blockIdx.x]; the reduction then adds the partials in order.
 __global__ void __launch_bounds__(256) value_loss_kernel(const ValueArgs p) {
+  __shared__ double part[8];
+  double acc = 0.0;
   for (int64_t t = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < p.rows;
        t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
     float c = 0.f;
@@ -209,7 +213,15 @@ __global__ void __launch_bounds__(256) value_loss_kernel(const ValueArgs p) {
     const float d = p.values[t] - p.returns[t];
     const float cd = c * d;
     p.d_values[t] = c != 0.f ? 2.f * cd : 0.f;
-    p.row_loss[t] = c != 0.f ? static_cast<double>(cd) * static_cast<double>(d) : 0.0;
+    if (c != 0.f) acc += static_cast<double>(cd) * static_cast<double>(d);
+  }
+  acc = warp_sum(acc);
+  if ((threadIdx.x & 31) == 0) part[threadIdx.x >> 5] = acc;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double t = 0.0;
+    for (int w = 0; w < 8; ++w) t += part[w];
+    p.row_loss[blockIdx.x] = t;
   }
 }
 
@@ -310,10 +322,11 @@ extern "C" rl_status rl_value_loss_fwd_bwd(int64_t rows, const float* values, co
   a.row_loss = row_loss;
   a.status = reinterpret_cast<int32_t*>(ws);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  ppo::value_loss_kernel<<<ppo::grid_for(rows, 256, 152 * 16), 256, 0, s>>>(a);
+  const int blocks = ppo::grid_for(rows, 256, 152 * 16);  // <= rows: one partial per CTA fits
+  ppo::value_loss_kernel<<<blocks, 256, 0, s>>>(a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_error(e, "value_loss_kernel launch");
-  return launch_reduce_loss(row_loss, rows, loss_accum, s);
+  return launch_reduce_loss(row_loss, blocks, loss_accum, s);
 }
 
 extern "C" rl_status rl_rollout_value_advantages(int64_t n_tokens, const int32_t* token_traj, const uint8_t* mask,

@@ -464,11 +464,8 @@ __global__ void __launch_bounds__((NW + 1) * 32, 2) rows_kernel(const RowArgs p)
             } else {
               for (int e = lane; e < n; e += 32) g[e] = T(0);
             }
-            if (rank == 0 && lane == 0) {
-              p.row_loss[r] = 0.0;
-              if (p.token_stats)
-                for (int k = 0; k < 5; ++k) p.token_stats[r * 5 + k] = 0.f;
-            }
+            if (rank == 0 && lane == 0 && p.token_stats)
+              for (int k = 0; k < 5; ++k) p.token_stats[r * 5 + k] = 0.f;
             continue;
           }
           m.old = __shfl_sync(0xffffffffu, lold, jr);
@@ -516,6 +513,9 @@ __global__ void __launch_bounds__((NW + 1) * 32, 2) rows_kernel(const RowArgs p)
     if (lane == 0 && stored) bulk_wait_read_all();
   } else {
     // =============================================================== consumer warps
+    // the cluster's loss contributions, added in the order of its rows (rank 0, warp 0, lane 0
+    // keeps the sum; one partial per cluster goes to the workspace at the end)
+    double cl_loss = 0.0;
     for (uint32_t it = 0;; ++it) {
       const int b = it % NB;
       if (!mbar_wait_bounded(&full_bar[b], (it / NB) & 1)) {
@@ -644,7 +644,7 @@ __global__ void __launch_bounds__((NW + 1) * 32, 2) rows_kernel(const RowArgs p)
         const float ca = ca0 * fl;                      // entropy: p_v (ca z_v + Ke)
         const float Ke = (-cg + ca0 * (H - lse)) * fl;
         if (rank == 0 && warp == 0 && lane == 0) {
-          p.row_loss[r] = static_cast<double>(c) * static_cast<double>(ell);
+          cl_loss += static_cast<double>(c) * static_cast<double>(ell);
           if (p.token_stats) {
             float* st = p.token_stats + r * 5;
             st[0] = logp; st[1] = rho; st[2] = cut ? 1.f : 0.f; st[3] = H; st[4] = kl;
@@ -727,6 +727,7 @@ __global__ void __launch_bounds__((NW + 1) * 32, 2) rows_kernel(const RowArgs p)
         if (lane == 0) mbar_arrive(&empty_bar[b]);
       }
     }
+    if (BWD && rank == 0 && warp == 0 && lane == 0) p.row_loss[cid] = cl_loss;  // cid < clusters <= rows
   }
   __syncthreads();
   // no CTA leaves while a peer may still write into its mailbox
@@ -898,30 +899,7 @@ __global__ void __launch_bounds__((NW + 1) * 32, 2) stream_logprobs_kernel(const
   }
 }
 
-// Fixed-order sum of the per-row contributions into the caller's accumulator.
-__global__ void __launch_bounds__(1024) reduce_loss_kernel(const double* __restrict__ row_loss, int64_t rows,
-                                                           double* loss_accum) {
-  __shared__ double part[32];
-  double acc = 0.0;
-  for (int64_t r = threadIdx.x; r < rows; r += 1024) acc += row_loss[r];
-  acc = warp_sum(acc);
-  if ((threadIdx.x & 31) == 0) part[threadIdx.x >> 5] = acc;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    double t = 0.0;
-    for (int w = 0; w < 32; ++w) t += part[w];
-    *loss_accum += t;
-  }
-}
-
 // ------------------------------------------------------------------ host side
-
-rl_status launch_reduce_loss(const double* row_loss, int64_t rows, double* loss_accum, cudaStream_t s) {
-  reduce_loss_kernel<<<1, 1024, 0, s>>>(row_loss, rows, loss_accum);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return cuda_error(e, "reduce_loss_kernel launch");
-  return RL_OK;
-}
 
 constexpr int kConsumerWarps = RL_CONSUMER_WARPS;
 constexpr int kRowThreads = (RL_CONSUMER_WARPS + 1) * 32;
@@ -970,7 +948,7 @@ static rl_status configure(const void* kern, int dev, size_t smem) {
 }
 
 template <typename T, bool ENT, int HOLDV>
-static rl_status launch_rows(const RowArgs& args, const Plan& plan, cudaStream_t s) {
+static rl_status launch_rows(const RowArgs& args, const Plan& plan, cudaStream_t s, int64_t* n_clusters_out) {
   auto kern = rows_kernel<T, kConsumerWarps, ENT, true, HOLDV>;
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -1020,18 +998,22 @@ static rl_status launch_rows(const RowArgs& args, const Plan& plan, cudaStream_t
   cfg.numAttrs = 1;
   e = cudaLaunchKernelEx(&cfg, kern, args);
   if (e != cudaSuccess) return cuda_error(e, "cudaLaunchKernelEx(rows_kernel)");
+  if (n_clusters_out) *n_clusters_out = n_clusters;
   return RL_OK;
 }
 
 // Registers hold the slice when it fits kHoldVecs 16-byte vectors per consumer thread.
 constexpr int kHoldVecs = 11;
 
+// Launches the loss kernel; *n_clusters receives the number of clusters, each of which leaves
+// one loss partial at the head of the per-row loss area.
 template <typename T>
-static rl_status dispatch_loss(bool ent, const RowArgs& args, const Plan& plan, cudaStream_t s) {
+static rl_status dispatch_loss(bool ent, const RowArgs& args, const Plan& plan, cudaStream_t s, int64_t* n_clusters) {
   const bool hold = plan.slice * static_cast<int64_t>(sizeof(T)) / 16 <= int64_t(kHoldVecs) * kConsumerWarps * 32;
   if (hold)
-    return ent ? launch_rows<T, true, kHoldVecs>(args, plan, s) : launch_rows<T, false, kHoldVecs>(args, plan, s);
-  return ent ? launch_rows<T, true, 0>(args, plan, s) : launch_rows<T, false, 0>(args, plan, s);
+    return ent ? launch_rows<T, true, kHoldVecs>(args, plan, s, n_clusters)
+               : launch_rows<T, false, kHoldVecs>(args, plan, s, n_clusters);
+  return ent ? launch_rows<T, true, 0>(args, plan, s, n_clusters) : launch_rows<T, false, 0>(args, plan, s, n_clusters);
 }
 
 constexpr int kFwdWarps = 8;
@@ -1180,7 +1162,9 @@ extern "C" rl_status rl_policy_loss_fwd_bwd(const void* logits, rl_dtype dtype, 
   a.tma = ((ld * es) % 16) == 0;
   const bool ent = params->entropy_coef != 0.f || token_stats != nullptr;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  st = dtype == RL_BF16 ? dispatch_loss<uint16_t>(ent, a, plan, s) : dispatch_loss<float>(ent, a, plan, s);
+  int64_t n_clusters = 0;
+  st = dtype == RL_BF16 ? dispatch_loss<uint16_t>(ent, a, plan, s, &n_clusters)
+                        : dispatch_loss<float>(ent, a, plan, s, &n_clusters);
   if (st != RL_OK) return st;
-  return launch_reduce_loss(row_loss, rows, loss_accum, s);
+  return launch_reduce_loss(row_loss, n_clusters, loss_accum, s);
 }

@@ -1,4 +1,5 @@
-// Batch summaries of the per-token statistics that rl_policy_loss_fwd_bwd and
+// Fixed-order reductions: the loss sum behind every loss entry point, and batch summaries of
+// the per-token statistics that rl_policy_loss_fwd_bwd and
 // rl_fused_head_loss_fwd_bwd write: the number of trained tokens, of clipped ones, and the
 // sums of entropy, KL and ratio over them (the clip fraction and the mean policy entropy that
 // are tracked during training, Sec. 4). One CTA, fixed assignment of rows to threads and a
@@ -9,6 +10,39 @@
 #include "rl_host.h"
 
 namespace rl {
+
+// Fixed-order sum of per-row loss contributions into the caller's accumulator (every loss
+// entry point ends with it). Thread k adds rows k, k + 1024, ... into eight accumulators in
+// turn, so eight independent loads are in flight per thread (one memory latency per 8,192
+// rows instead of per 1,024); the accumulators, the warps and the CTA are then combined in a
+// fixed order: the sum is the same on every run.
+__global__ void __launch_bounds__(1024) reduce_loss_kernel(const double* __restrict__ row_loss, int64_t rows,
+                                                           double* loss_accum) {
+  __shared__ double part[32];
+  double acc[8] = {0.0, 0.0, 0.0, 0.0, 0.0, 0.0, 0.0, 0.0};
+  int64_t r = threadIdx.x;
+  for (; r + 7 * 1024 < rows; r += 8 * 1024) {
+#pragma unroll
+    for (int k = 0; k < 8; ++k) acc[k] += row_loss[r + k * 1024];
+  }
+  for (int k = 0; r < rows; r += 1024, ++k) acc[k] += row_loss[r];
+  double a = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+  a = warp_sum(a);
+  if ((threadIdx.x & 31) == 0) part[threadIdx.x >> 5] = a;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double t = 0.0;
+    for (int w = 0; w < 32; ++w) t += part[w];
+    *loss_accum += t;
+  }
+}
+
+rl_status launch_reduce_loss(const double* row_loss, int64_t rows, double* loss_accum, cudaStream_t s) {
+  reduce_loss_kernel<<<1, 1024, 0, s>>>(row_loss, rows, loss_accum);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_error(e, "reduce_loss_kernel launch");
+  return RL_OK;
+}
 
 constexpr int kSumThreads = 1024;
 
