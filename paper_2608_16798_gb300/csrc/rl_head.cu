@@ -486,7 +486,7 @@ static rl_status encoder(EncodeTiledFn* out) {
 
 // bf16 matrix [rows x inner] (row stride inner), tiles of box_rows x 64 with the 128-byte swizzle.
 static rl_status make_map(CUtensorMap* m, const void* base, int64_t inner, int64_t rows, uint32_t box_rows) {
-  EncodeTiledFn enc;
+  EncodeTiledFn enc = nullptr;
   rl_status st = encoder(&enc);
   if (st != RL_OK) return st;
   cuuint64_t dims[2] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(rows)};
@@ -668,7 +668,7 @@ extern "C" rl_status rl_fused_head_loss_fwd_bwd(
   float* tmax = reinterpret_cast<float*>(wsb + L.off_tmax);
   uint16_t* dz = reinterpret_cast<uint16_t*>(wsb + L.off_dz);
   void* lt_ws = wsb + L.off_lt;
-  cublasLtHandle_t lt;
+  cublasLtHandle_t lt = nullptr;
   rl_status st = lt_handle(&lt);
   if (st != RL_OK) return st;
   const bool kl_on = params->kl_estimator == 3 && params->kl_coef != 0.f && ref_logp != nullptr;
