@@ -284,3 +284,19 @@ def test_fused_head_loss_shape_limits(R):
     assert call(V=524_289) == 2     # above the fix-up kernel's shared-memory tile factors
     assert call(D=65_600) == 2
     assert call(T=-1) == 1
+
+
+def test_binding_fails_loudly_without_the_library(R, monkeypatch):
+    """No CPU fallback: with the shared library absent every entry point raises."""
+    import pytest as _pytest
+    import torch
+
+    monkeypatch.setattr(R, "_lib", None)
+    monkeypatch.setattr(R, "LIB_PATH", R.LIB_PATH + ".absent")
+    with _pytest.raises(RuntimeError, match="missing"):
+        R.lib()
+    with _pytest.raises(RuntimeError, match="missing"):
+        R.rl_workspace_size(16, 128)
+    # host tensors are refused outright: there is no CPU path to fall back to
+    with _pytest.raises(ValueError, match="CUDA tensor"):
+        R.rl_token_logprobs(torch.zeros((2, 8)), torch.zeros(2, dtype=torch.int32), torch.zeros(1024, dtype=torch.uint8))
