@@ -14,13 +14,23 @@
  *   - the token-level truncated importance weight w_t = min(exp(log pi_old -
  *     log pi_rollout), c-bar) (Sec. 3.2.4, TIS equation);
  *   - log pi(a_t | s_t) of the sampled token, a log-softmax over the vocabulary
- *     (Sec. 2.3, the policy pi_theta(a_t | s_t)).
+ *     (Sec. 2.3, the policy pi_theta(a_t | s_t)), from logits rows or through a
+ *     fused LM head (logits = hidden W^T formed on the tensor cores, never stored);
+ *   - PPO's masked GAE, per-token advantages and masked value loss (Sec. 2.3.1,
+ *     Sec. 2.3.4);
+ *   - rollout-level prefix trees of captured model calls, packed once per shared
+ *     prefix, and the advantages and counts of their tokens in any order
+ *     (Sec. 3.2.1-3.2.3);
+ *   - sequence-level importance weights (Sec. 3.2.4) and batch summaries of the
+ *     per-token statistics (entropy, clip fraction; Sec. 4).
  *
  * Conventions shared by every entry point:
- *   - Array arguments are DEVICE pointers owned by the caller. The library
- *     never allocates, frees or synchronises (except rl_query_status, which
- *     synchronises the given stream). All work is enqueued on `stream`
- *     (a cudaStream_t; NULL is the legacy default stream).
+ *   - Array arguments are DEVICE pointers owned by the caller (the one
+ *     exception, rl_prefix_tree_build_batch, is a host function on host
+ *     pointers). The library never allocates device memory, frees or
+ *     synchronises (except rl_query_status, which synchronises the given
+ *     stream). All work is enqueued on `stream` (a cudaStream_t; NULL is the
+ *     legacy default stream).
  *   - Argument errors that the host can see return a status before anything is
  *     launched; rl_last_error_message() then describes the problem.
  *   - Errors that only the device can see (a token id outside [0, V), a
