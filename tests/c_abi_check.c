@@ -1,0 +1,153 @@
+/* A plain C caller of the library (no Python, no torch): it includes only rl_loss.h and
+ * links librl_loss.so. Argument "host" runs the host-side checks; argument "gpu" also runs
+ * the advantages and the policy loss on a small batch whose result has a closed form:
+ * uniform logits (all 0) give logp = -ln V for every token; with old_logp = logp the ratio
+ * is 1, nothing is clipped, and the loss is -sum_i c_i L_i A_i, which is 0 for complete
+ * groups under RL_AGG_SEQ_MEAN_TOKEN_MEAN; every trained gradient row is
+ * -c_i A_i (onehot_a - 1/V). Exit status 0 on success. */
+#include <math.h>
+#include <stdint.h>
+#include <stdio.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include "rl_loss.h"
+
+/* The CUDA runtime calls this check needs, declared here so that the file needs no CUDA
+ * header: they are resolved from libcudart at link time. */
+typedef int cudaError_t;
+extern cudaError_t cudaMalloc(void** p, size_t n);
+extern cudaError_t cudaFree(void* p);
+extern cudaError_t cudaMemcpy(void* dst, const void* src, size_t n, int kind);
+extern cudaError_t cudaMemset(void* p, int v, size_t n);
+enum { H2D = 1, D2H = 2 };
+
+static int fails = 0;
+#define CHECK(cond, ...)                      \
+  do {                                        \
+    if (!(cond)) {                            \
+      fprintf(stderr, "FAIL: " __VA_ARGS__); \
+      fprintf(stderr, "\n");                  \
+      ++fails;                                \
+    }                                         \
+  } while (0)
+
+static int host_checks(void) {
+  CHECK(rl_version() >= 10000, "rl_version");
+  CHECK(rl_workspace_size(0, 0, 0) == 256, "workspace header");
+  CHECK(rl_workspace_size(16384, 151936, 0) == 256 + 16384 * 8, "workspace rows");
+  rl_loss_params p;
+  memset(&p, 0, sizeof p);
+  p.clip_eps_low = 0.2f;
+  p.clip_eps_high = 0.28f;
+  p.adv_eps = 1e-6f;
+  void* fake = (void*)(uintptr_t)0x10000;
+  double* lacc = (double*)fake;
+  /* a bad dtype, a misaligned gradient, a small workspace: errors before any launch */
+  CHECK(rl_policy_loss_fwd_bwd(fake, (rl_dtype)7, 4, 8, 8, fake, fake, fake, 2, fake, fake, fake, NULL, NULL, &p,
+                               fake, lacc, NULL, fake, 1 << 20, NULL) == RL_ERR_INVALID_ARG,
+        "bad dtype");
+  CHECK(rl_policy_loss_fwd_bwd(fake, RL_BF16, 4, 8, 8, fake, fake, fake, 2, fake, fake, fake, NULL, NULL, &p,
+                               (char*)fake + 8, lacc, NULL, fake, 1 << 20, NULL) == RL_ERR_ALIGNMENT,
+        "misaligned gradient");
+  CHECK(rl_policy_loss_fwd_bwd(fake, RL_BF16, 4, 8, 8, fake, fake, fake, 2, fake, fake, fake, NULL, NULL, &p, fake,
+                               lacc, NULL, fake, 100, NULL) == RL_ERR_WORKSPACE_TOO_SMALL,
+        "small workspace");
+  CHECK(strstr(rl_last_error_message(), "rl_policy_loss_fwd_bwd") != NULL, "error message");
+  return fails;
+}
+
+static int gpu_checks(void) {
+  enum { G = 2, PER = 4, N = G * PER, LEN = 24, T = N * LEN, V = 1000 };
+  const int32_t go[G + 1] = {0, PER, 2 * PER};
+  float rewards[N];
+  int64_t offs[N + 1];
+  uint8_t mask[T];
+  int32_t ids[T];
+  float old[T];
+  for (int i = 0; i < N; ++i) rewards[i] = (float)((i * 7) % 3);
+  for (int i = 0; i <= N; ++i) offs[i] = (int64_t)i * LEN;
+  for (int t = 0; t < T; ++t) {
+    mask[t] = (uint8_t)((t % 5) != 0); /* every trajectory keeps trained tokens */
+    ids[t] = (t * 37) % V;
+    old[t] = (float)(-log((double)V));
+  }
+  rl_loss_params p;
+  memset(&p, 0, sizeof p);
+  p.clip_eps_low = 0.2f;
+  p.clip_eps_high = 0.28f;
+  p.adv_eps = 1e-6f;
+  p.loss_agg = RL_AGG_SEQ_MEAN_TOKEN_MEAN;
+
+  void *d_go, *d_rw, *d_offs, *d_mask, *d_ids, *d_old, *d_adv, *d_coef, *d_ntok, *d_tt, *d_logits, *d_grad, *d_loss,
+      *d_ws;
+  const size_t ws_bytes = rl_workspace_size(T, V, 0);
+  int bad = 0;
+  bad |= cudaMalloc(&d_go, sizeof go) | cudaMalloc(&d_rw, sizeof rewards) | cudaMalloc(&d_offs, sizeof offs);
+  bad |= cudaMalloc(&d_mask, sizeof mask) | cudaMalloc(&d_ids, sizeof ids) | cudaMalloc(&d_old, sizeof old);
+  bad |= cudaMalloc(&d_adv, N * 4) | cudaMalloc(&d_coef, N * 4) | cudaMalloc(&d_ntok, N * 4) | cudaMalloc(&d_tt, T * 4);
+  bad |= cudaMalloc(&d_logits, (size_t)T * V * 4) | cudaMalloc(&d_grad, (size_t)T * V * 4);
+  bad |= cudaMalloc(&d_loss, 8) | cudaMalloc(&d_ws, ws_bytes);
+  if (bad) {
+    fprintf(stderr, "FAIL: cudaMalloc\n");
+    return 1;
+  }
+  cudaMemcpy(d_go, go, sizeof go, H2D);
+  cudaMemcpy(d_rw, rewards, sizeof rewards, H2D);
+  cudaMemcpy(d_offs, offs, sizeof offs, H2D);
+  cudaMemcpy(d_mask, mask, sizeof mask, H2D);
+  cudaMemcpy(d_ids, ids, sizeof ids, H2D);
+  cudaMemcpy(d_old, old, sizeof old, H2D);
+  cudaMemset(d_logits, 0, (size_t)T * V * 4); /* uniform rows */
+  cudaMemset(d_loss, 0, 8);
+  CHECK(rl_workspace_init(d_ws, ws_bytes, NULL) == RL_OK, "workspace init");
+  CHECK(rl_group_advantages(N, G, d_go, d_rw, NULL, T, d_offs, d_mask, &p, d_adv, d_coef, d_ntok, d_tt, d_ws,
+                            ws_bytes, NULL) == RL_OK,
+        "rl_group_advantages: %s", rl_last_error_message());
+  CHECK(rl_policy_loss_fwd_bwd(d_logits, RL_F32, T, V, V, d_ids, d_mask, d_tt, N, d_adv, d_coef, d_old, NULL, NULL,
+                               &p, d_grad, d_loss, NULL, d_ws, ws_bytes, NULL) == RL_OK,
+        "rl_policy_loss_fwd_bwd: %s", rl_last_error_message());
+  int32_t word = -1;
+  CHECK(rl_query_status(d_ws, NULL, &word) == RL_OK && word == 0, "device status %d", word);
+
+  float adv[N], coef[N];
+  int32_t ntok[N];
+  double loss = 0.0;
+  cudaMemcpy(adv, d_adv, sizeof adv, D2H);
+  cudaMemcpy(coef, d_coef, sizeof coef, D2H);
+  cudaMemcpy(ntok, d_ntok, sizeof ntok, D2H);
+  cudaMemcpy(&loss, d_loss, 8, D2H);
+  double expect = 0.0, scale = 0.0;
+  for (int i = 0; i < N; ++i) {
+    expect -= (double)coef[i] * ntok[i] * adv[i];
+    scale += fabs((double)coef[i] * ntok[i] * adv[i]);
+  }
+  CHECK(fabs(loss - expect) <= 1e-5 * scale + 1e-12, "loss %.9g, closed form %.9g", loss, expect);
+  CHECK(fabs(expect) <= 1e-6 * scale + 1e-12, "complete groups: the closed form is 0 (%.3g)", expect);
+  /* gradient rows: -c A (onehot - 1/V) on trained tokens, zero elsewhere */
+  float* row = (float*)malloc(V * sizeof(float));
+  for (int t = 0; t < T; t += 7) {
+    cudaMemcpy(row, (char*)d_grad + (size_t)t * V * 4, V * sizeof(float), D2H);
+    const int i = t / LEN;
+    const double g = mask[t] ? -(double)coef[i] * adv[i] : 0.0;
+    for (int v = 0; v < V; ++v) {
+      const double ref = g * ((v == ids[t] ? 1.0 : 0.0) - 1.0 / V);
+      if (fabs(row[v] - ref) > 1e-6 * fabs(g) + 1e-12) {
+        fprintf(stderr, "FAIL: grad[%d][%d] = %.9g, closed form %.9g\n", t, v, row[v], ref);
+        ++fails;
+        break;
+      }
+    }
+  }
+  free(row);
+  void* all[] = {d_go, d_rw, d_offs, d_mask, d_ids, d_old, d_adv, d_coef, d_ntok, d_tt, d_logits, d_grad, d_loss, d_ws};
+  for (size_t k = 0; k < sizeof all / sizeof all[0]; ++k) cudaFree(all[k]);
+  return fails;
+}
+
+int main(int argc, char** argv) {
+  int f = host_checks();
+  if (argc > 1 && strcmp(argv[1], "gpu") == 0) f += gpu_checks();
+  if (f == 0) printf("c_abi_check ok\n");
+  return f == 0 ? 0 : 1;
+}
