@@ -18,6 +18,9 @@
 #include <algorithm>
 #include <cstdint>
 #include <cstring>
+#include <exception>
+#include <mutex>
+#include <new>
 #include <string>
 #include <thread>
 #include <unordered_map>
@@ -62,12 +65,10 @@ static inline int64_t own_len(const Node& n, int64_t parent_hist) { return n.x.n
 // Is the accumulated history of `child` a prefix of x, given that its parent's is?
 static bool child_matches(const Node& child, int64_t parent_hist, const Span& x) {
   if (child.hist_len > x.n) return false;
-  const int64_t len = own_len(child, parent_hist);
   // own tokens are child.x[parent_hist:] then child.y; compare with x[parent_hist:]
   const int64_t nx = child.x.n - parent_hist;
   if (nx > 0 && std::memcmp(child.x.p + parent_hist, x.p + parent_hist, nx * sizeof(int32_t)) != 0) return false;
   if (child.y.n > 0 && std::memcmp(child.y.p, x.p + child.x.n, child.y.n * sizeof(int32_t)) != 0) return false;
-  (void)len;
   return true;
 }
 
@@ -232,24 +233,54 @@ static void emit(const Rollout& R, int32_t r, int64_t base, int64_t lbase, const
   }
 }
 
+// Runs f(0..n-1) on up to `threads` host threads. An exception in a worker is kept and
+// rethrown after every thread has joined; so is a failure to start a thread (the threads
+// already started are joined first).
 template <class F>
 static void parallel_for(int32_t n, int32_t threads, F f) {
   if (threads <= 1 || n <= 1) {
     for (int32_t i = 0; i < n; ++i) f(i);
     return;
   }
-  std::vector<std::thread> pool;
+  std::mutex mu;
+  std::exception_ptr first;
   const int32_t T = std::min(threads, n);
-  for (int32_t w = 0; w < T; ++w)
-    pool.emplace_back([=, &f] {
+  auto work = [&](int32_t w) {
+    try {
       for (int32_t i = w; i < n; i += T) f(i);
-    });
+    } catch (...) {
+      std::lock_guard<std::mutex> lock(mu);
+      if (!first) first = std::current_exception();
+    }
+  };
+  std::vector<std::thread> pool;
+  try {
+    for (int32_t w = 0; w < T; ++w) pool.emplace_back(work, w);
+  } catch (...) {
+    for (auto& th : pool) th.join();
+    throw;
+  }
   for (auto& th : pool) th.join();
+  if (first) std::rethrow_exception(first);
 }
 
 }  // namespace tree
 }  // namespace rl
 
+namespace rl {
+namespace tree {
+static rl_status build_batch(int32_t n_rollouts, const int64_t* prompt_offsets, const int32_t* prompt_tokens,
+                             const int32_t* call_offsets, const int64_t* x_offsets, const int32_t* x_tokens,
+                             const int64_t* y_offsets, const int32_t* y_tokens, const uint8_t* aux, int32_t max_leaves,
+                             int32_t n_threads, int64_t capacity, int32_t* tokens_out, uint8_t* mask_out,
+                             int64_t* parent_out, int32_t* depth_out, int32_t* owner_out, int32_t* node_call_out,
+                             int32_t* leaf_call_out, int64_t* leaf_end_out, int64_t* leaf_offsets_out,
+                             rl_tree_stats* stats_out, int64_t* rollout_offsets_out, int64_t* n_tokens_out);
+}  // namespace tree
+}  // namespace rl
+
+// C entry point: no C++ exception (an allocation or a thread that cannot be created) may
+// cross the C ABI; it becomes an error status instead.
 extern "C" rl_status rl_prefix_tree_build_batch(
     int32_t n_rollouts, const int64_t* prompt_offsets, const int32_t* prompt_tokens, const int32_t* call_offsets,
     const int64_t* x_offsets, const int32_t* x_tokens, const int64_t* y_offsets, const int32_t* y_tokens,
@@ -257,8 +288,27 @@ extern "C" rl_status rl_prefix_tree_build_batch(
     uint8_t* mask_out, int64_t* parent_out, int32_t* depth_out, int32_t* owner_out, int32_t* node_call_out,
     int32_t* leaf_call_out, int64_t* leaf_end_out, int64_t* leaf_offsets_out, rl_tree_stats* stats_out,
     int64_t* rollout_offsets_out, int64_t* n_tokens_out) {
-  using namespace rl;
-  using namespace rl::tree;
+  try {
+    return rl::tree::build_batch(n_rollouts, prompt_offsets, prompt_tokens, call_offsets, x_offsets, x_tokens,
+                                 y_offsets, y_tokens, aux, max_leaves, n_threads, capacity, tokens_out, mask_out,
+                                 parent_out, depth_out, owner_out, node_call_out, leaf_call_out, leaf_end_out,
+                                 leaf_offsets_out, stats_out, rollout_offsets_out, n_tokens_out);
+  } catch (const std::bad_alloc&) {
+    return rl::set_error(RL_ERR_UNSUPPORTED, "rl_prefix_tree_build_batch: out of host memory");
+  } catch (const std::exception& e) {
+    return rl::set_error(RL_ERR_UNSUPPORTED, std::string("rl_prefix_tree_build_batch: ") + e.what());
+  } catch (...) {
+    return rl::set_error(RL_ERR_UNSUPPORTED, "rl_prefix_tree_build_batch: unexpected host error");
+  }
+}
+
+static rl_status rl::tree::build_batch(
+    int32_t n_rollouts, const int64_t* prompt_offsets, const int32_t* prompt_tokens, const int32_t* call_offsets,
+    const int64_t* x_offsets, const int32_t* x_tokens, const int64_t* y_offsets, const int32_t* y_tokens,
+    const uint8_t* aux, int32_t max_leaves, int32_t n_threads, int64_t capacity, int32_t* tokens_out,
+    uint8_t* mask_out, int64_t* parent_out, int32_t* depth_out, int32_t* owner_out, int32_t* node_call_out,
+    int32_t* leaf_call_out, int64_t* leaf_end_out, int64_t* leaf_offsets_out, rl_tree_stats* stats_out,
+    int64_t* rollout_offsets_out, int64_t* n_tokens_out) {
   clear_error();
   if (n_rollouts < 0) return set_error(RL_ERR_INVALID_ARG, "rl_prefix_tree_build_batch: n_rollouts < 0");
   if (!n_tokens_out) return set_error(RL_ERR_INVALID_ARG, "rl_prefix_tree_build_batch: n_tokens_out is NULL");
