@@ -198,6 +198,12 @@ def check_grad(g_dev, g_ref, dtype, what="", row_scale=None, absolute=True):
     rs = np.abs(g_ref).max(axis=1, keepdims=True) if g_ref.size else np.zeros((g_ref.shape[0], 1))
     row_scale = rs if row_scale is None else np.maximum(rs, row_scale)
     tol = (fmt + 2e-5) * np.abs(g_ref) + 2e-5 * row_scale + 1e-30
+    if g_ref.size:
+        # relative to the row's scale (its largest element, or the coefficient size when the
+        # exact row is 0, e.g. V = 1)
+        rel = d.max(axis=1, keepdims=True) / np.maximum(row_scale, 1e-30)
+        print(f"{what}: max per-row relative error {float(rel.max()):.3e}, "
+              f"max error / bound {float((d / tol).max()):.3f}")
     bad = d > tol
     if bad.any():
         r, v = np.argwhere(bad)[0]

@@ -43,7 +43,8 @@ def _host_raw(logits, dtype):
     return logits.cpu().numpy()
 
 
-@pytest.mark.parametrize("name,mb", [("multiturn", 0), ("multiturn", -1), ("longhorizon", 1), ("edge", 0)])
+@pytest.mark.parametrize("name,mb", [("multiturn", 0), ("multiturn", -1), ("longhorizon", 0), ("longhorizon", 1),
+                                     ("longhorizon", -1), ("edge", 0)])
 def test_full_microbatch(R, name, mb):
     w = W.WORKLOADS[name]
     seed = 0
