@@ -391,46 +391,49 @@ def time_tree(torch, R, dev, reps=3):
                     "advantages by owner timed as CUDA-graph replays"}
 
 
-class HugePinned:
-    """Host memory for the end-to-end leg: an anonymous mapping advised to use transparent huge
-    pages, touched, then registered with the CUDA runtime (page-locked, visible to copies).
-    On the box, pinned allocations made of small pages copy at 18-110 GB/s from some regions;
-    these copy at 211 GB/s from every region. Falls back to torch's pinned allocator when the
-    mapping or the registration is refused."""
+class StagedPinned:
+    """Host memory for the end-to-end leg: a HostStagingBuffer (one mapping with transparent huge
+    pages, registered with the CUDA runtime) whose units are qualified by timing a copy from each
+    to the device; units that copy far below the median are replaced before any timed work. On
+    the box, a few physical huge pages in some processes copy at 8-72 GB/s against 210 GB/s from
+    the rest. Falls back to torch's pinned allocator when the mapping or registration is refused."""
 
-    def __init__(self, torch, rows, cols, dtype):
-        import mmap
+    def __init__(self, torch, rows, cols, dtype, dev):
+        from paper_2608_16798_gb300.host_staging import HostStagingBuffer
 
-        self.torch, self.mm, self.addr = torch, None, None
+        self.buf, self.qualified = None, None
         nbytes = rows * cols * torch.empty((), dtype=dtype).element_size()
+        cr = torch.cuda.cudart()
         try:
-            self.mm = mmap.mmap(-1, nbytes, flags=mmap.MAP_PRIVATE | mmap.MAP_ANONYMOUS)
-            if hasattr(mmap, "MADV_HUGEPAGE"):
-                self.mm.madvise(mmap.MADV_HUGEPAGE)
-            raw = np.frombuffer(self.mm, dtype=np.uint8)
-            raw[::4096] = 0  # touch every page before registering
-            addr = raw.ctypes.data
-            if torch.cuda.cudart().cudaHostRegister(addr, nbytes, 0) != torch.cuda.cudart().cudaError.success:
-                raise RuntimeError("cudaHostRegister refused")
-            self.addr = addr
-            self.tensor = torch.frombuffer(self.mm, dtype=dtype).view(rows, cols)
-            self.kind = "huge pages, registered"
+            self.buf = HostStagingBuffer(nbytes, lambda a, n: cr.cudaHostRegister(a, n, 0) == cr.cudaError.success,
+                                         lambda a: cr.cudaHostUnregister(a))
+            units = torch.frombuffer(self.buf.buffer(whole_units=True), dtype=torch.uint8)
+            scratch = torch.empty(self.buf.unit, dtype=torch.uint8, device=dev)
+            s = torch.cuda.Stream(dev)
+
+            def probe(off, n):
+                a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                with torch.cuda.stream(s):
+                    a0.record(s)
+                    scratch[:n].copy_(units[off:off + n], non_blocking=True)
+                    a1.record(s)
+                a1.synchronize()
+                return n / a0.elapsed_time(a1) / 1e6
+
+            self.qualified = self.buf.qualify(probe)
+            del units, scratch
+            self.tensor = torch.frombuffer(self.buf.buffer(), dtype=dtype).view(rows, cols)
+            self.kind = "huge pages, registered, qualified"
         except Exception:
             self.close()
             self.tensor = torch.empty((rows, cols), dtype=dtype, pin_memory=True)
             self.kind = "torch pinned"
 
     def close(self):
-        if self.addr is not None:
-            self.torch.cuda.cudart().cudaHostUnregister(self.addr)
-            self.addr = None
         self.tensor = None
-        if self.mm is not None:
-            try:
-                self.mm.close()
-            except BufferError:  # a view still exists: the mapping goes with the process
-                pass
-            self.mm = None
+        if self.buf is not None:
+            self.buf.close()
+            self.buf = None
 
 
 def host_mem_available() -> int:
@@ -466,12 +469,12 @@ def e2e_run(torch, R, batch, dev, steps, warmup, slots=4):
     # one mapping for the whole host source (separate per-microbatch mappings measured 3-73 GB/s
     # from some of them, one mapping 211 GB/s from nearly all of its microbatches)
     if whole:
-        pinned = HugePinned(t, batch.T, V, t.bfloat16)
+        pinned = StagedPinned(t, batch.T, V, t.bfloat16, dev)
         for lo, hi in batch.mbs:
             pinned.tensor[lo:hi].copy_(batch.logits[lo:hi])
         host_mb = [pinned.tensor[lo:hi] for lo, hi in batch.mbs]
     else:
-        pinned = HugePinned(t, 2 * mb, V, t.bfloat16)
+        pinned = StagedPinned(t, 2 * mb, V, t.bfloat16, dev)
         for k in range(2):
             lo, hi = batch.mbs[k % len(batch.mbs)]
             pinned.tensor[k * mb:k * mb + hi - lo].copy_(batch.logits[lo:hi])
@@ -523,6 +526,17 @@ def e2e_run(torch, R, batch, dev, steps, warmup, slots=4):
             read_done[s].record(comp)
         loss_host.copy_(loss, non_blocking=True)
 
+    # each microbatch's copy timed alone: the host source's bandwidth, which bounds the step
+    alone = []
+    for k, (lo, hi) in enumerate(batch.mbs):
+        a0, a1 = t.cuda.Event(enable_timing=True), t.cuda.Event(enable_timing=True)
+        with t.cuda.stream(copy_in):
+            a0.record(copy_in)
+            dev_logits[0][:hi - lo].copy_(host_mb[src[k]][:hi - lo], non_blocking=True)
+            a1.record(copy_in)
+        a1.synchronize()
+        alone.append((hi - lo) * V * 2 / a0.elapsed_time(a1) / 1e6)
+    t.cuda.synchronize(dev)
     for _ in range(warmup):
         one_step()
     t.cuda.synchronize(dev)
@@ -537,7 +551,9 @@ def e2e_run(torch, R, batch, dev, steps, warmup, slots=4):
     check = float(loss_host.item())
     del host_mb
     pinned.close()
-    return ms, h2d, d2h, check, ("whole batch" if whole else "ring of 2 microbatches") + ", " + host_kind
+    copy_gbs = {"min": min(alone), "median": statistics.median(alone), "max": max(alone),
+                "in_steps": h2d * steps / (ms * 1e-3) / 1e9, "staging": pinned.qualified}
+    return ms, h2d, d2h, check, ("whole batch" if whole else "ring of 2 microbatches") + ", " + host_kind, copy_gbs
 
 
 # ----------------------------------------------------------------------------- oracle (CPU) legs
@@ -1050,9 +1066,10 @@ def main():
 
     e2e = None
     if not args.no_e2e:
-        e_ms, h2d, d2h, e_loss, src = e2e_run(torch, R, batch, dev, args.e2e_steps, 1)
+        e_ms, h2d, d2h, e_loss, src, copy_gbs = e2e_run(torch, R, batch, dev, args.e2e_steps, 2)
         e2e = {"value": batch.T / (e_ms / 1e3 / args.e2e_steps) * world, "unit": UNIT, "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "steps": args.e2e_steps, "loss": e_loss, "host_source": src,
+               "h2d_gbs": copy_gbs,
                "note": "per step: metadata and every microbatch's logits from pinned host memory, loss read "
                        "back; the gradient stays in HBM for the model's backward"}
 
