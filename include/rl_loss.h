@@ -111,8 +111,9 @@ const char* rl_last_error_message(void);
 /* Workspace bytes needed by calls on at most `max_rows` logits rows of
  * vocabulary V (D = hidden size of the fused head, 0 if unused). The
  * workspace holds the device status word and per-row loss contributions; with
- * D > 0 it also holds the fused head's per-chunk buffers (about
- * min(max_rows, 4096) * V * 2 bytes plus 32 MiB). */
+ * D > 0 it also holds the fused head's buffers (about
+ * min(max_rows, 32768) * V * 2 bytes plus 32 MiB: the bf16 dZ of up to
+ * 32,768 tokens). */
 size_t rl_workspace_size(int64_t max_rows, int64_t V, int64_t D);
 
 /* Zero the workspace's status word. Call once after allocating a workspace,
@@ -242,11 +243,14 @@ rl_status rl_policy_loss_fwd_bwd(const void* logits, rl_dtype dtype, int64_t row
  *                 (overwritten; zero rows for tokens that are not trained on)
  *   d_weight      float [V x D]: d loss / d W is ADDED to it
  *   ws, ws_bytes  workspace of at least rl_workspace_size(T, V, D) bytes; it holds,
- *                 among others, the gradient of the logits for one chunk of 4,096
- *                 tokens (bf16), consumed by the dH and dW products of that chunk
- * Tokens are processed in chunks of 4,096: per chunk, a tensor-core pass forms the
- * softmax statistics, a second pass recomputes the logits and forms their gradient,
- * and two GEMMs (cuBLASLt) produce dH and accumulate dW.
+ *                 among others, the gradient of the logits (bf16) for a group of up
+ *                 to 32,768 tokens, consumed by the dH and dW products
+ * Tokens are processed in chunks of 4,096: per chunk, one tensor-core pass forms the
+ * logits tile by tile, folds them into softmax partials and keeps exp(z - tile max)
+ * in bf16 with the tile maxima; a per-token merge evaluates the objective; an in-place
+ * rescale turns the kept values into the logits' gradient; a GEMM (cuBLASLt) gives the
+ * chunk's dH. After the last chunk of each group of up to 32,768 tokens, one GEMM
+ * (cuBLASLt) adds the group's dW.
  */
 rl_status rl_fused_head_loss_fwd_bwd(const void* hidden, const void* weight, int64_t T, int64_t D, int64_t V,
                                      const int32_t* token_ids, const uint8_t* mask, const int32_t* token_traj,

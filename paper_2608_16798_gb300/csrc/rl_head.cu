@@ -14,7 +14,10 @@
 //   3. head_dz_kernel       rescales the stored e in place into
 //      dZ = c [g (delta_a - p) + alpha p (log p + H)], p = e exp(m_j - lse) (HBM-bound: the
 //      logits are formed once, not twice).
-//   4. dH = dZ W and dW += dZ^T H, two plain GEMMs through cuBLASLt.
+//   4. dH = dZ W for the chunk, through cuBLASLt. The chunks of a group (up to 32,768 tokens)
+//      keep their dZ side by side in the workspace, and after the group's last chunk one
+//      cuBLASLt GEMM adds dZ^T H over the whole group into dW: the fp32 dW (V x D x 4 bytes)
+//      is read and written once per group rather than once per chunk.
 // The forward-only call runs head_kernel<STATS> (no stores) and head_logp_merge_kernel.
 // The objective (Sec. 2.3.2, Sec. 3.2.4) is the same as for rl_policy_loss_fwd_bwd; here
 // pi_theta's logits come from the hidden states times the vocabulary projection.
@@ -48,6 +51,11 @@ constexpr size_t kSmem = NS * STAGE_BYTES + 1024;
 #define RL_HEAD_CHUNK 4096
 #endif
 constexpr int64_t kChunk = RL_HEAD_CHUNK;  // tokens per chunk (tuning knob, compile time)
+#ifndef RL_HEAD_GROUP
+#define RL_HEAD_GROUP 32768
+#endif
+// tokens whose dZ the workspace holds at once: dW += dZ^T H runs once per group (tuning knob)
+constexpr int64_t kGroup = RL_HEAD_GROUP;
 constexpr size_t kLtWorkspace = 32u << 20;
 
 enum Mode { STATS = 0, STATS_P = 1 };
@@ -501,7 +509,7 @@ static rl_status make_map(CUtensorMap* m, const void* base, int64_t inner, int64
 }
 
 struct Layout {
-  int64_t Tc, n_nt, n_vb, ldz;
+  int64_t Tc, G, n_nt, n_vb, ldz;  // G chunks per group
   size_t off_partials, off_rc, off_tmax, off_dz, off_lt, total;
 };
 
@@ -510,6 +518,8 @@ static size_t al256(size_t x) { return (x + 255) & ~size_t(255); }
 static Layout layout(int64_t max_rows, int64_t V) {
   Layout L;
   L.Tc = std::max<int64_t>(1, std::min<int64_t>(max_rows, kChunk));
+  const int64_t chunks = (std::max<int64_t>(max_rows, 1) + L.Tc - 1) / L.Tc;
+  L.G = std::max<int64_t>(1, std::min<int64_t>(chunks, kGroup / L.Tc));
   const int64_t n_nt = (V + BN - 1) / BN;
   L.n_nt = n_nt;
   L.n_vb = (n_nt + VB_TILES - 1) / VB_TILES;
@@ -523,7 +533,7 @@ static Layout layout(int64_t max_rows, int64_t V) {
   L.off_tmax = off;
   off += al(static_cast<size_t>(L.Tc * n_nt) * sizeof(float));
   L.off_dz = off;
-  off += al(static_cast<size_t>(L.Tc * L.ldz) * 2);
+  off += al(static_cast<size_t>(L.G * L.Tc * L.ldz) * 2);
   L.off_lt = off;
   off += kLtWorkspace;
   L.total = off;
@@ -666,7 +676,7 @@ extern "C" rl_status rl_fused_head_loss_fwd_bwd(
   float4* partials = reinterpret_cast<float4*>(wsb + L.off_partials);
   RowCoef* rcs = reinterpret_cast<RowCoef*>(wsb + L.off_rc);
   float* tmax = reinterpret_cast<float*>(wsb + L.off_tmax);
-  uint16_t* dz = reinterpret_cast<uint16_t*>(wsb + L.off_dz);
+  uint16_t* dz_base = reinterpret_cast<uint16_t*>(wsb + L.off_dz);
   void* lt_ws = wsb + L.off_lt;
   cublasLtHandle_t lt = nullptr;
   rl_status st = lt_handle(&lt);
@@ -678,8 +688,11 @@ extern "C" rl_status rl_fused_head_loss_fwd_bwd(
   st = make_map(&mw, weight, D, V, BN);
   if (st != RL_OK) return st;
   const int n_nt = static_cast<int>((V + BN - 1) / BN);
+  const int64_t group_rows = L.G * L.Tc;
   for (int64_t t0 = 0; t0 < T; t0 += L.Tc) {
     const int Tc = static_cast<int>(std::min<int64_t>(L.Tc, T - t0));
+    const int64_t g0 = t0 - t0 % group_rows;  // first token of this chunk's group
+    uint16_t* dz = dz_base + (t0 - g0) * L.ldz;
     const uint16_t* h0 = static_cast<const uint16_t*>(hidden) + t0 * D;
     CUtensorMap mh;
     st = make_map(&mh, h0, D, Tc, BM);
@@ -749,9 +762,14 @@ extern "C" rl_status rl_fused_head_loss_fwd_bwd(
     st = lt_matmul(lt, false, false, D, Tc, V, weight, D, dz, L.ldz, dh, D,
                    d_hidden_dtype == RL_BF16 ? CUDA_R_16BF : CUDA_R_32F, 0.f, lt_ws, kLtWorkspace, s);
     if (st != RL_OK) return st;
-    // dW += dZ^T H  (column-major: dW^T [D x V] += H^T [D x Tc] (dZ^T)^T [Tc x V])
-    st = lt_matmul(lt, false, true, D, V, Tc, h0, D, dz, L.ldz, d_weight, D, CUDA_R_32F, 1.f, lt_ws, kLtWorkspace, s);
-    if (st != RL_OK) return st;
+    // at the group's last chunk: dW += dZ^T H over the group's tokens
+    // (column-major: dW^T [D x V] += H^T [D x n] (dZ^T)^T [n x V])
+    const int64_t g1 = std::min<int64_t>(g0 + group_rows, T);
+    if (t0 + Tc == g1) {
+      st = lt_matmul(lt, false, true, D, V, g1 - g0, static_cast<const uint16_t*>(hidden) + g0 * D, D, dz_base,
+                     L.ldz, d_weight, D, CUDA_R_32F, 1.f, lt_ws, kLtWorkspace, s);
+      if (st != RL_OK) return st;
+    }
   }
   return launch_reduce_loss(row_loss, T, loss_accum, s);
 }
