@@ -248,9 +248,9 @@ rl_status rl_policy_loss_fwd_bwd(const void* logits, rl_dtype dtype, int64_t row
  * Tokens are processed in chunks of 4,096: per chunk, one tensor-core pass forms the
  * logits tile by tile, folds them into softmax partials and keeps exp(z - tile max)
  * in bf16 with the tile maxima; a per-token merge evaluates the objective; an in-place
- * rescale turns the kept values into the logits' gradient; a GEMM (cuBLASLt) gives the
- * chunk's dH. After the last chunk of each group of up to 32,768 tokens, one GEMM
- * (cuBLASLt) adds the group's dW.
+ * rescale turns the kept values into the logits' gradient. After the last chunk of
+ * each group of up to 32,768 tokens, two GEMMs (cuBLASLt) give the group's dH and add
+ * its dW.
  */
 rl_status rl_fused_head_loss_fwd_bwd(const void* hidden, const void* weight, int64_t T, int64_t D, int64_t V,
                                      const int32_t* token_ids, const uint8_t* mask, const int32_t* token_traj,

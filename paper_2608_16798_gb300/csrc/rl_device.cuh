@@ -125,6 +125,10 @@ __device__ __forceinline__ bool mbar_wait_cluster_bounded(uint64_t* bar, uint32_
 __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" :: "r"(smem_addr(bar)) : "memory");
 }
+// Arrive (release, cluster scope) on an mbarrier of a CTA of this cluster (address from map_to_rank).
+__device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" :: "r"(cluster_addr) : "memory");
+}
 
 // 16-byte store into shared memory of a CTA of this cluster (address from map_to_rank),
 // signalling `remote_bar` (same CTA) with complete_tx of 16 bytes. No ordering of other

@@ -2,9 +2,10 @@
 // and the output projection, with the logits Z = H W^T never written to memory.
 //
 // For each chunk of tokens:
-//   1. head_kernel<STATS_P> tcgen05 GEMM tiles Z[128 x 256] = H W^T (TMA-fed shared-memory
-//      stages, fp32 accumulators in TMEM, two accumulators so the epilogue of one tile
-//      overlaps the MMAs of the next). The epilogue reads each tile twice from TMEM: first
+//   1. head_kernel<STATS_P> tcgen05 GEMM tiles Z[256 x 256] = H W^T on CTA pairs (2-CTA
+//      clusters, cta_group::2 MMAs; TMA-fed shared-memory stages, fp32 accumulators in TMEM,
+//      two accumulators so the epilogue of one tile overlaps the MMAs of the next; each CTA
+//      holds 128 of the tile's tokens). The epilogue reads each tile twice from TMEM: first
 //      its row maximum m_j, then e = exp(z - m_j), which it stores (bf16) in the chunk's
 //      dZ buffer, with m_j per token and tile, and folds into per-row online-softmax
 //      partials for its vocabulary block.
@@ -14,10 +15,11 @@
 //   3. head_dz_kernel       rescales the stored e in place into
 //      dZ = c [g (delta_a - p) + alpha p (log p + H)], p = e exp(m_j - lse) (HBM-bound: the
 //      logits are formed once, not twice).
-//   4. dH = dZ W for the chunk, through cuBLASLt. The chunks of a group (up to 32,768 tokens)
-//      keep their dZ side by side in the workspace, and after the group's last chunk one
-//      cuBLASLt GEMM adds dZ^T H over the whole group into dW: the fp32 dW (V x D x 4 bytes)
-//      is read and written once per group rather than once per chunk.
+// The chunks of a group (up to 32,768 tokens) keep their dZ side by side in the workspace;
+// after the group's last chunk:
+//   4. dH = dZ W and dW += dZ^T H over the whole group, two plain GEMMs through cuBLASLt: the
+//      fp32 dW (V x D x 4 bytes) is read and written once per group rather than once per
+//      chunk, and the dH product has eight times the output tiles of a chunk's.
 // The forward-only call runs head_kernel<STATS> (no stores) and head_logp_merge_kernel.
 // The objective (Sec. 2.3.2, Sec. 3.2.4) is the same as for rl_policy_loss_fwd_bwd; here
 // pi_theta's logits come from the hidden states times the vocabulary projection.
@@ -47,6 +49,15 @@ constexpr int VB_TILES = RL_HEAD_VB_TILES;  // N tiles per work item (16: a voca
 constexpr uint32_t A_BYTES = BM * BK * 2, B_BYTES = BN * BK * 2, STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int kThreads = 192;      // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
 constexpr size_t kSmem = NS * STAGE_BYTES + 1024;
+// CTA-pair form: each CTA stages its 128 tokens and half of the 256 vocabulary rows
+constexpr int NS2 = 6;
+constexpr uint32_t STAGE2_BYTES = A_BYTES + B_BYTES / 2;
+constexpr size_t kSmem2 = NS2 * STAGE2_BYTES + 1024;
+#ifndef RL_HEAD_PAIR
+#define RL_HEAD_PAIR 1
+#endif
+constexpr bool kPair = RL_HEAD_PAIR != 0;
+constexpr uint32_t kWBoxRows = kPair ? BN / 2 : BN;  // rows of W per TMA box
 #ifndef RL_HEAD_CHUNK
 #define RL_HEAD_CHUNK 4096
 #endif
@@ -84,32 +95,51 @@ struct HeadArgs {
   int32_t* status;
 };
 
-template <int MODE>
+// Two forms share this kernel. PAIR = false: each CTA computes 128 x 256 tiles with
+// cta_group::1 MMAs from 48 KB stages (A 16 KB + B 32 KB, 4 stages). PAIR = true: a cluster of
+// two CTAs computes 256 x 256 tiles with cta_group::2 MMAs issued by the even CTA; each CTA
+// loads its own 128 tokens of H and its own 128 vocabulary rows of W (32 KB stages, 6 of them),
+// both CTAs' loads complete on the even CTA's barrier, the MMA's commits are multicast to both
+// CTAs, and each CTA's epilogue drains its own 128 TMEM lanes (all 256 columns) and tells the
+// even CTA's MMA thread when an accumulator is free. Per pair this halves the W operand each SM
+// fetches and stages per MMA.
+template <int MODE, bool PAIR>
 __global__ void __launch_bounds__(kThreads, 1) head_kernel(const __grid_constant__ CUtensorMap tmH,
                                                            const __grid_constant__ CUtensorMap tmW,
                                                            const HeadArgs p) {
+  constexpr int kNS = PAIR ? NS2 : NS;
+  constexpr uint32_t kStage = PAIR ? STAGE2_BYTES : STAGE_BYTES;
   extern __shared__ uint8_t smem_raw[];
-  __shared__ __align__(8) uint64_t full[NS], empty[NS], accf[2], acce[2];
+  __shared__ __align__(8) uint64_t full[kNS], empty[kNS], accf[2], acce[2];
   __shared__ uint32_t tbase;
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n_items = p.n_mt * p.n_vb;
+  const uint32_t rank = PAIR ? cluster_ctarank() : 0u;
+  const int unit = PAIR ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
+  const int n_units = PAIR ? static_cast<int>(gridDim.x >> 1) : static_cast<int>(gridDim.x);
+  constexpr int kMStep = PAIR ? 2 * BM : BM;  // tokens per work item
+  const int n_m = (p.Tc + kMStep - 1) / kMStep;
+  const int n_items = n_m * p.n_vb;
   const int nkb = p.D / BK;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < NS; ++s) {
+    for (int s = 0; s < kNS; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&accf[a], 1);
-      mbar_init(&acce[a], 4);
+      mbar_init(&acce[a], PAIR ? 8 : 4);
     }
     fence_mbar_init();
   }
-  if (warp == 1) tc::tmem_alloc(&tbase, 2 * BN);
+  if (warp == 1) {
+    if constexpr (PAIR) tc::tmem_alloc_pair(&tbase, 2 * BN);
+    else tc::tmem_alloc(&tbase, 2 * BN);
+  }
   tc::fence_before_sync();
-  __syncthreads();
+  if constexpr (PAIR) cluster_sync_all();
+  else __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = tbase;
 
@@ -118,60 +148,80 @@ __global__ void __launch_bounds__(kThreads, 1) head_kernel(const __grid_constant
     if (lane == 0) {
       uint32_t g = 0;
       bool ok = true;
-      for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
-        const int vb = item / p.n_mt, m0 = (item % p.n_mt) * BM;
+      for (int item = unit; item < n_items && ok; item += n_units) {
+        const int vb = item / n_m, m0 = (item % n_m) * kMStep + static_cast<int>(rank) * BM;
         const int nt1 = min((vb + 1) * VB_TILES, p.n_nt);
         for (int nt = vb * VB_TILES; nt < nt1 && ok; ++nt) {
           for (int kb = 0; kb < nkb; ++kb, ++g) {
-            const int s = g % NS;
-            const uint32_t use = g / NS;
+            const int s = g % kNS;
+            const uint32_t use = g / kNS;
             if (use > 0 && !mbar_wait_bounded(&empty[s], (use - 1) & 1)) {
               flag_status(p.status, RL_DEV_TIMEOUT);
               ok = false;
               break;
             }
-            uint8_t* st = sm + s * STAGE_BYTES;
-            mbar_arrive_expect_tx(&full[s], STAGE_BYTES);
-            tc::tma_load_2d(st, &tmH, kb * BK, m0, &full[s]);
-            tc::tma_load_2d(st + A_BYTES, &tmW, kb * BK, nt * BN, &full[s]);
+            uint8_t* st = sm + s * kStage;
+            if constexpr (PAIR) {
+              if (rank == 0) mbar_arrive_expect_tx(&full[s], 2 * kStage);  // both CTAs' bytes
+              const uint32_t bar = map_to_rank(smem_addr(&full[s]), 0);
+              tc::tma_load_2d_pair(st, &tmH, kb * BK, m0, bar);
+              tc::tma_load_2d_pair(st + A_BYTES, &tmW, kb * BK, nt * BN + static_cast<int>(rank) * (BN / 2), bar);
+            } else {
+              mbar_arrive_expect_tx(&full[s], kStage);
+              tc::tma_load_2d(st, &tmH, kb * BK, m0, &full[s]);
+              tc::tma_load_2d(st + A_BYTES, &tmW, kb * BK, nt * BN, &full[s]);
+            }
           }
         }
       }
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
-    if (lane == 0) {
-      constexpr uint32_t idesc = tc::idesc_bf16_f32(BM, BN);
+    if (lane == 0 && rank == 0) {
+      constexpr uint32_t idesc = tc::idesc_bf16_f32(kMStep, BN);
       uint32_t g = 0, t = 0;
       bool ok = true;
-      for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
-        const int vb = item / p.n_mt;
+      for (int item = unit; item < n_items && ok; item += n_units) {
+        const int vb = item / n_m;
         const int nt1 = min((vb + 1) * VB_TILES, p.n_nt);
         for (int nt = vb * VB_TILES; nt < nt1 && ok; ++nt, ++t) {
           const int acc = t & 1;
-          if (t >= 2 && !mbar_wait_bounded(&acce[acc], ((t >> 1) - 1) & 1)) {
-            flag_status(p.status, RL_DEV_TIMEOUT);
-            ok = false;
-            break;
+          if (t >= 2) {
+            const uint32_t par = ((t >> 1) - 1) & 1;
+            const bool got = PAIR ? mbar_wait_cluster_bounded(&acce[acc], par) : mbar_wait_bounded(&acce[acc], par);
+            if (!got) {
+              flag_status(p.status, RL_DEV_TIMEOUT);
+              ok = false;
+              break;
+            }
           }
           tc::fence_after_sync();
           const uint32_t d = tmem + acc * BN;
           for (int kb = 0; kb < nkb; ++kb, ++g) {
-            const int s = g % NS;
-            if (!mbar_wait_bounded(&full[s], (g / NS) & 1)) {
+            const int s = g % kNS;
+            if (!mbar_wait_bounded(&full[s], (g / kNS) & 1)) {
               flag_status(p.status, RL_DEV_TIMEOUT);
               ok = false;
               break;
             }
             tc::fence_after_sync();
-            const uint32_t a = smem_addr(sm + s * STAGE_BYTES), b = a + A_BYTES;
+            const uint32_t a = smem_addr(sm + s * kStage), b = a + A_BYTES;
 #pragma unroll
-            for (int k = 0; k < BK / 16; ++k)
-              tc::mma_bf16(d, tc::desc_kmajor_sw128(a + k * 32), tc::desc_kmajor_sw128(b + k * 32), idesc,
-                           (kb | k) != 0);
-            tc::mma_commit(&empty[s]);
+            for (int k = 0; k < BK / 16; ++k) {
+              if constexpr (PAIR)
+                tc::mma_bf16_pair(d, tc::desc_kmajor_sw128(a + k * 32), tc::desc_kmajor_sw128(b + k * 32), idesc,
+                                  (kb | k) != 0);
+              else
+                tc::mma_bf16(d, tc::desc_kmajor_sw128(a + k * 32), tc::desc_kmajor_sw128(b + k * 32), idesc,
+                             (kb | k) != 0);
+            }
+            if constexpr (PAIR) tc::mma_commit_pair(&empty[s], 0x3);
+            else tc::mma_commit(&empty[s]);
           }
-          if (ok) tc::mma_commit(&accf[acc]);
+          if (ok) {
+            if constexpr (PAIR) tc::mma_commit_pair(&accf[acc], 0x3);
+            else tc::mma_commit(&accf[acc]);
+          }
         }
       }
     }
@@ -182,8 +232,8 @@ __global__ void __launch_bounds__(kThreads, 1) head_kernel(const __grid_constant
     const float kNegInf = -__int_as_float(0x7f800000);
     uint32_t t = 0;
     bool ok = true;
-    for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
-      const int vb = item / p.n_mt, m0 = (item % p.n_mt) * BM;
+    for (int item = unit; item < n_items && ok; item += n_units) {
+      const int vb = item / n_m, m0 = (item % n_m) * kMStep + static_cast<int>(rank) * BM;
       const int r = m0 + rl;  // token within the chunk
       const bool row_ok = r < p.Tc;
       const int nt1 = min((vb + 1) * VB_TILES, p.n_nt);
@@ -259,7 +309,10 @@ __global__ void __launch_bounds__(kThreads, 1) head_kernel(const __grid_constant
         }
         tc::fence_before_sync();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&acce[acc]);
+        if (lane == 0) {
+          if (PAIR && rank != 0) mbar_arrive_remote(map_to_rank(smem_addr(&acce[acc]), 0));
+          else mbar_arrive(&acce[acc]);
+        }
         if (MODE == STATS_P && row_ok) p.tmax[static_cast<int64_t>(r) * p.n_nt + nt] = tm;
         ps = merge(ps, SoftmaxPartial{tm, s0 + s1, u0});
       }
@@ -267,10 +320,12 @@ __global__ void __launch_bounds__(kThreads, 1) head_kernel(const __grid_constant
     }
   }
   tc::fence_before_sync();
-  __syncthreads();
+  if constexpr (PAIR) cluster_sync_all();
+  else __syncthreads();
   if (warp == 1) {
     tc::fence_after_sync();
-    tc::tmem_dealloc(tmem, 2 * BN);
+    if constexpr (PAIR) tc::tmem_dealloc_pair(tmem, 2 * BN);
+    else tc::tmem_dealloc(tmem, 2 * BN);
   }
 }
 
@@ -592,26 +647,57 @@ static rl_status lt_handle(cublasLtHandle_t* out) {
 
 template <int MODE>
 static rl_status launch_head(const CUtensorMap& mh, const CUtensorMap& mw, const HeadArgs& a, cudaStream_t s) {
-  auto kern = head_kernel<MODE>;
+  auto kern = head_kernel<MODE, kPair>;
+  constexpr size_t smem = kPair ? kSmem2 : kSmem;
   int dev = 0, sms = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return cuda_error(e, "cudaDeviceGetAttribute");
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
   static std::mutex mu;
-  static std::map<std::pair<int, int>, bool> configured;
+  static std::map<std::pair<int, int>, int> resident;  // pairs resident at once (pair form)
+  int max_pairs = 0;
   {
     std::lock_guard<std::mutex> lock(mu);
     auto key = std::make_pair(dev, MODE);
-    if (!configured[key]) {
-      e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kSmem));
+    auto it = resident.find(key);
+    if (it == resident.end()) {
+      e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
       if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(head_kernel)");
-      configured[key] = true;
+      int n = sms;
+      if constexpr (kPair) {
+        cfg.gridDim = dim3(2);
+        e = cudaOccupancyMaxActiveClusters(&n, kern, &cfg);
+        if (e != cudaSuccess) return cuda_error(e, "cudaOccupancyMaxActiveClusters(head_kernel)");
+        if (n <= 0) return set_error(RL_ERR_UNSUPPORTED, "head_kernel: no CTA pair fits on the device");
+      }
+      it = resident.emplace(key, n).first;
     }
+    max_pairs = it->second;
   }
-  const int items = a.n_mt * a.n_vb;
-  kern<<<std::min(items, sms), kThreads, kSmem, s>>>(mh, mw, a);
-  e = cudaGetLastError();
-  if (e != cudaSuccess) return cuda_error(e, "head_kernel launch");
+  if constexpr (kPair) {
+    // persistent: one 2-CTA cluster per resident pair, work items of 256 tokens x one vocabulary block
+    const int items = (a.Tc + 2 * BM - 1) / (2 * BM) * a.n_vb;
+    const int pairs = std::max(1, std::min(items, max_pairs));
+    cfg.gridDim = dim3(2 * pairs);
+    e = cudaLaunchKernelEx(&cfg, kern, mh, mw, a);
+    if (e != cudaSuccess) return cuda_error(e, "cudaLaunchKernelEx(head_kernel)");
+  } else {
+    const int items = a.n_mt * a.n_vb;
+    kern<<<std::min(items, sms), kThreads, smem, s>>>(mh, mw, a);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_error(e, "head_kernel launch");
+  }
   return RL_OK;
 }
 
@@ -685,7 +771,7 @@ extern "C" rl_status rl_fused_head_loss_fwd_bwd(
   const bool ent = params->entropy_coef != 0.f || token_stats != nullptr;
 
   CUtensorMap mw;
-  st = make_map(&mw, weight, D, V, BN);
+  st = make_map(&mw, weight, D, V, kWBoxRows);
   if (st != RL_OK) return st;
   const int n_nt = static_cast<int>((V + BN - 1) / BN);
   const int64_t group_rows = L.G * L.Tc;
@@ -757,15 +843,15 @@ extern "C" rl_status rl_fused_head_loss_fwd_bwd(
     e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_error(e, "head_dz_kernel launch");
 
-    // dH[t0 : t0 + Tc] = dZ W    (column-major: dH^T [D x Tc] = W^T [D x V] dZ^T [V x Tc])
-    void* dh = static_cast<char*>(d_hidden) + t0 * D * (d_hidden_dtype == RL_BF16 ? 2 : 4);
-    st = lt_matmul(lt, false, false, D, Tc, V, weight, D, dz, L.ldz, dh, D,
-                   d_hidden_dtype == RL_BF16 ? CUDA_R_16BF : CUDA_R_32F, 0.f, lt_ws, kLtWorkspace, s);
-    if (st != RL_OK) return st;
-    // at the group's last chunk: dW += dZ^T H over the group's tokens
-    // (column-major: dW^T [D x V] += H^T [D x n] (dZ^T)^T [n x V])
+    // after the group's last chunk, the two products over the group's n = g1 - g0 tokens
     const int64_t g1 = std::min<int64_t>(g0 + group_rows, T);
     if (t0 + Tc == g1) {
+      // dH[g0 : g1] = dZ W    (column-major: dH^T [D x n] = W^T [D x V] dZ^T [V x n])
+      void* dh = static_cast<char*>(d_hidden) + g0 * D * (d_hidden_dtype == RL_BF16 ? 2 : 4);
+      st = lt_matmul(lt, false, false, D, g1 - g0, V, weight, D, dz_base, L.ldz, dh, D,
+                     d_hidden_dtype == RL_BF16 ? CUDA_R_16BF : CUDA_R_32F, 0.f, lt_ws, kLtWorkspace, s);
+      if (st != RL_OK) return st;
+      // dW += dZ^T H  (column-major: dW^T [D x V] += H^T [D x n] (dZ^T)^T [n x V])
       st = lt_matmul(lt, false, true, D, V, g1 - g0, static_cast<const uint16_t*>(hidden) + g0 * D, D, dz_base,
                      L.ldz, d_weight, D, CUDA_R_32F, 1.f, lt_ws, kLtWorkspace, s);
       if (st != RL_OK) return st;
@@ -801,7 +887,7 @@ extern "C" rl_status rl_fused_head_token_logprobs(const void* hidden, const void
   int32_t* status = reinterpret_cast<int32_t*>(wsb);
   float4* partials = reinterpret_cast<float4*>(wsb + kWsHeader);
   CUtensorMap mw;
-  rl_status st = make_map(&mw, weight, D, V, BN);
+  rl_status st = make_map(&mw, weight, D, V, kWBoxRows);
   if (st != RL_OK) return st;
   const int n_nt = static_cast<int>((V + BN - 1) / BN);
   for (int64_t t0 = 0; t0 < T; t0 += L.Tc) {

@@ -132,8 +132,8 @@ def test_fused_head_parity(R, T, D, V, agg, ent, tis):
 
 
 def test_fused_head_two_chunks_bf16_grad(R):
-    """More than 8,192 tokens: three chunks of 4,096 in one group (their dZ side by side, one dW
-    product); bf16 d_hidden."""
+    """More than 8,192 tokens: three chunks of 4,096 in one group (their dZ side by side, one dH
+    and one dW product); bf16 d_hidden."""
     c = make_head_case(8192 + 77, 128, 1100, seed=5, agg=2)
     out = run_head(R, c, dh_dtype=torch.bfloat16)
     compare_head(c, out, dh_bf16=True)
@@ -141,7 +141,7 @@ def test_fused_head_two_chunks_bf16_grad(R):
 
 def test_fused_head_two_groups(R):
     """More than 32,768 tokens: a full group of eight chunks and a ragged second group of two;
-    dW gets one product per group, the second added onto the first."""
+    one dH and one dW product per group, the second group's dW added onto the first's."""
     c = make_head_case(32768 + 4096 + 50, 64, 600, seed=11, agg=0, ent=True)
     out = run_head(R, c)
     compare_head(c, out)
