@@ -50,7 +50,10 @@ constexpr uint32_t A_BYTES = BM * BK * 2, B_BYTES = BN * BK * 2, STAGE_BYTES = A
 constexpr int kThreads = 192;      // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
 constexpr size_t kSmem = NS * STAGE_BYTES + 1024;
 // CTA-pair form: each CTA stages its 128 tokens and half of the 256 vocabulary rows
-constexpr int NS2 = 6;
+#ifndef RL_HEAD_NS2
+#define RL_HEAD_NS2 6
+#endif
+constexpr int NS2 = RL_HEAD_NS2;
 constexpr uint32_t STAGE2_BYTES = A_BYTES + B_BYTES / 2;
 constexpr size_t kSmem2 = NS2 * STAGE2_BYTES + 1024;
 #ifndef RL_HEAD_PAIR
