@@ -124,6 +124,8 @@ def compare_head(c, out, dh_bf16=False):
     (256, 128, 8292, 0, False, False),     # three vocabulary blocks
     (200, 192, 700, 2, True, False),       # entropy + k3 KL
     (130, 64, 513, 1, False, True),        # TIS, token-mean, smallest D
+    (100, 128, 777, 0, True, False),       # one CTA pair whose odd CTA's 128 tokens all lie past T
+    (5, 64, 300, 2, False, False),         # a handful of tokens
 ])
 def test_fused_head_parity(R, T, D, V, agg, ent, tis):
     c = make_head_case(T, D, V, seed=T + V, agg=agg, ent=ent, tis=tis)
@@ -198,6 +200,7 @@ def run_logprobs(R, c, want_entropy=True, ids=None):
     (300, 256, 1000),        # ragged M tile and vocabulary tile
     (256, 128, 8292),        # three vocabulary blocks, ragged last block
     (130, 64, 513),          # smallest D
+    (64, 64, 1000),          # the odd CTA of the only pair has no tokens
     (8192 + 77, 128, 1100),  # three chunks
 ])
 def test_fused_head_logprobs_parity(R, T, D, V):
