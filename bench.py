@@ -281,7 +281,49 @@ def time_other_workloads(torch, R, dev, peak, reps=10):
                      "achieved_gbs": gbs, "frac": gbs / peak, "reps": reps}
         del items
         t.cuda.empty_cache()
+    out["tiny"] = time_tiny(torch, R, dev)
     return out
+
+
+def time_tiny(torch, R, dev, reps=100):
+    """The tiny workload (one group of 8 trajectories x 64 tokens, V = 4,096 bf16): a whole step
+    (advantages + the loss over the 512 rows) is 8.4 MB of logits and gradient, resident in the
+    129 MB L2, so it is latency-bound and gets no HBM fraction. Timed as CUDA-graph replays (device
+    time) and as eager calls (with the host's launch overhead)."""
+    t = torch
+    w = W.WORKLOADS["tiny"]
+    lay = W.make_layout(w, 0)
+    d = lambda x: t.from_numpy(np.ascontiguousarray(x)).to(dev)  # noqa: E731
+    T = lay.n_tokens
+    logits = t.empty((T, w.vocab), dtype=t.bfloat16, device=dev)
+    W.logits_rows_torch(w, 0, 0, T, logits)
+    ids = W.sample_tokens_torch(logits, 0, 0, w)
+    params = R.make_params(W.CLIP_EPS_LOW, W.CLIP_EPS_HIGH, 0.0, 0, 0.0, 0.0, 1e-6, 0)
+    ws = R.new_workspace(T, w.vocab, device=dev)
+    logp, _, _ = R.rl_token_logprobs(logits, ids, ws)
+    old = d(W.old_logp_from(logp.cpu().numpy(), w, 0, 0))
+    go, rw, to, mask, valid = (d(lay.group_offsets), d(lay.rewards), d(lay.traj_offsets), d(lay.mask),
+                               d(lay.traj_valid))
+    adv, coef = t.empty(lay.n_traj, device=dev), t.empty(lay.n_traj, device=dev)
+    n_tok = t.empty(lay.n_traj, dtype=t.int32, device=dev)
+    tt = t.empty(T, dtype=t.int32, device=dev)
+    grad, loss = t.empty_like(logits), t.zeros(1, dtype=t.float64, device=dev)
+
+    def step():
+        R.rl_group_advantages(go, rw, to, mask, params, ws, traj_valid=valid, adv_out=adv, coef_out=coef,
+                              n_tok_out=n_tok, token_traj_out=tt)
+        R.rl_policy_loss_fwd_bwd(logits, ids, mask, tt, adv, coef, old, params, ws, loss, grad_out=grad)
+
+    ms_graph = _time_graph(torch, step, reps)
+    ms_eager = _time_calls(torch, step, 3, reps)
+    st, word = R.rl_query_status(ws)
+    if word != 0:
+        raise RuntimeError(f"device status word {word} after the tiny timing")
+    return {"rows_per_step": T, "vocab": w.vocab, "dtype": w.dtype, "l2_resident": True,
+            "bytes_per_step": int(((lay.mask.astype(np.int64) + 1) * w.vocab * 2).sum()),
+            "us_per_step_graph": ms_graph * 1e3, "us_per_step_eager": ms_eager * 1e3,
+            "tokens_per_s_graph": T / (ms_graph * 1e-3), "tokens_per_s_eager": T / (ms_eager * 1e-3),
+            "note": "advantages + loss over the whole batch; resident in L2, so latency-bound: no HBM fraction"}
 
 
 def time_ppo(torch, R, batch, dev, warmup=3, reps=20):
@@ -393,41 +435,55 @@ def time_tree(torch, R, dev, reps=3):
 
 class StagedPinned:
     """Host memory for the end-to-end leg: a HostStagingBuffer (one mapping with transparent huge
-    pages, registered with the CUDA runtime) whose units are qualified by timing a copy from each
-    to the device; units that copy far below the median are replaced before any timed work. On
-    the box, a few physical huge pages in some processes copy at 8-72 GB/s against 210 GB/s from
-    the rest. Falls back to torch's pinned allocator when the mapping or registration is refused."""
+    pages, registered with the CUDA runtime). Once filled, its units are qualified by timing a
+    copy from each to the device; units that copy far below the median are replaced and refilled
+    before any timed work. On the box, a few physical huge pages in some processes copy at 3-72
+    GB/s against 210 GB/s from the rest, and pages can turn slow when first written. Falls back to
+    torch's pinned allocator when the mapping or registration is refused."""
 
     def __init__(self, torch, rows, cols, dtype, dev):
         from paper_2608_16798_gb300.host_staging import HostStagingBuffer
 
-        self.buf, self.qualified = None, None
+        self.torch, self.dev, self.buf, self.qualified = torch, dev, None, None
         nbytes = rows * cols * torch.empty((), dtype=dtype).element_size()
         cr = torch.cuda.cudart()
         try:
             self.buf = HostStagingBuffer(nbytes, lambda a, n: cr.cudaHostRegister(a, n, 0) == cr.cudaError.success,
                                          lambda a: cr.cudaHostUnregister(a))
-            units = torch.frombuffer(self.buf.buffer(whole_units=True), dtype=torch.uint8)
-            scratch = torch.empty(self.buf.unit, dtype=torch.uint8, device=dev)
-            s = torch.cuda.Stream(dev)
-
-            def probe(off, n):
-                a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-                with torch.cuda.stream(s):
-                    a0.record(s)
-                    scratch[:n].copy_(units[off:off + n], non_blocking=True)
-                    a1.record(s)
-                a1.synchronize()
-                return n / a0.elapsed_time(a1) / 1e6
-
-            self.qualified = self.buf.qualify(probe)
-            del units, scratch
             self.tensor = torch.frombuffer(self.buf.buffer(), dtype=dtype).view(rows, cols)
             self.kind = "huge pages, registered, qualified"
         except Exception:
             self.close()
             self.tensor = torch.empty((rows, cols), dtype=dtype, pin_memory=True)
             self.kind = "torch pinned"
+
+    def qualify(self, source):
+        """After the fill: time a copy from each unit, replace slow units and refill them from
+        `source` (a device tensor whose bytes the buffer holds from its start)."""
+        if self.buf is None:
+            return
+        t = self.torch
+        units = t.frombuffer(self.buf.buffer(whole_units=True), dtype=t.uint8)
+        src = source.view(-1).view(t.uint8)
+        scratch = t.empty(self.buf.unit, dtype=t.uint8, device=self.dev)
+        s = t.cuda.Stream(self.dev)
+
+        def probe(off, n):
+            a0, a1 = t.cuda.Event(enable_timing=True), t.cuda.Event(enable_timing=True)
+            with t.cuda.stream(s):
+                a0.record(s)
+                scratch[:n].copy_(units[off:off + n], non_blocking=True)
+                a1.record(s)
+            a1.synchronize()
+            return n / a0.elapsed_time(a1) / 1e6
+
+        def refill(off, n):
+            n = max(0, min(n, self.buf.nbytes - off, src.numel() - off))
+            if n:
+                units[off:off + n].copy_(src[off:off + n])
+
+        self.qualified = self.buf.qualify(probe, refill)
+        t.cuda.synchronize(self.dev)
 
     def close(self):
         self.tensor = None
@@ -448,7 +504,7 @@ def host_mem_available() -> int:
     return 0
 
 
-def e2e_run(torch, R, batch, dev, steps, warmup, slots=4):
+def e2e_run(torch, R, batch, dev, steps, warmup, slots=4, repeats=3):
     """Same step through host buffers: every step copies its inputs from pinned host memory (the
     whole batch's logits, microbatch by microbatch, and the metadata) to the device and reads the
     step's loss back; the gradient stays in HBM (batch.grad), where a training step's backward
@@ -472,12 +528,15 @@ def e2e_run(torch, R, batch, dev, steps, warmup, slots=4):
         pinned = StagedPinned(t, batch.T, V, t.bfloat16, dev)
         for lo, hi in batch.mbs:
             pinned.tensor[lo:hi].copy_(batch.logits[lo:hi])
+        pinned.qualify(batch.logits)
         host_mb = [pinned.tensor[lo:hi] for lo, hi in batch.mbs]
     else:
         pinned = StagedPinned(t, 2 * mb, V, t.bfloat16, dev)
         for k in range(2):
             lo, hi = batch.mbs[k % len(batch.mbs)]
             pinned.tensor[k * mb:k * mb + hi - lo].copy_(batch.logits[lo:hi])
+        if len(batch.mbs) >= 2:  # the ring then holds the batch's first 2 x mb rows, byte for byte
+            pinned.qualify(batch.logits)
         host_mb = [pinned.tensor[(k % 2) * mb:(k % 2) * mb + hi - lo] for k, (lo, hi) in enumerate(batch.mbs)]
     src = list(range(len(batch.mbs)))
     host_kind = pinned.kind
@@ -526,33 +585,48 @@ def e2e_run(torch, R, batch, dev, steps, warmup, slots=4):
             read_done[s].record(comp)
         loss_host.copy_(loss, non_blocking=True)
 
-    # each microbatch's copy timed alone: the host source's bandwidth, which bounds the step
-    alone = []
-    for k, (lo, hi) in enumerate(batch.mbs):
-        a0, a1 = t.cuda.Event(enable_timing=True), t.cuda.Event(enable_timing=True)
-        with t.cuda.stream(copy_in):
-            a0.record(copy_in)
-            dev_logits[0][:hi - lo].copy_(host_mb[src[k]][:hi - lo], non_blocking=True)
-            a1.record(copy_in)
-        a1.synchronize()
-        alone.append((hi - lo) * V * 2 / a0.elapsed_time(a1) / 1e6)
-    t.cuda.synchronize(dev)
-    for _ in range(warmup):
-        one_step()
-    t.cuda.synchronize(dev)
-    e0, e1 = t.cuda.Event(enable_timing=True), t.cuda.Event(enable_timing=True)
-    e0.record(comp)
-    for _ in range(steps):
-        one_step()
-    e1.record(comp)
-    e1.synchronize()
-    t.cuda.synchronize(dev)
-    ms = e0.elapsed_time(e1)
+    def copies_alone():
+        # each microbatch's copy timed alone: the host source's bandwidth, which bounds the step
+        out = []
+        for k, (lo, hi) in enumerate(batch.mbs):
+            a0, a1 = t.cuda.Event(enable_timing=True), t.cuda.Event(enable_timing=True)
+            with t.cuda.stream(copy_in):
+                a0.record(copy_in)
+                dev_logits[0][:hi - lo].copy_(host_mb[src[k]][:hi - lo], non_blocking=True)
+                a1.record(copy_in)
+            a1.synchronize()
+            out.append((hi - lo) * V * 2 / a0.elapsed_time(a1) / 1e6)
+        return out
+
+    # repetitions of `steps` timed steps; before each, the staging buffer is qualified again (on
+    # the box, pages of a qualified buffer were seen to turn slow later in the same process)
+    runs = []
+    for rep in range(repeats):
+        if rep > 0:
+            pinned.qualify(batch.logits)
+        staging = pinned.qualified
+        alone = copies_alone()
+        t.cuda.synchronize(dev)
+        for _ in range(warmup):
+            one_step()
+        t.cuda.synchronize(dev)
+        e0, e1 = t.cuda.Event(enable_timing=True), t.cuda.Event(enable_timing=True)
+        e0.record(comp)
+        for _ in range(steps):
+            one_step()
+        e1.record(comp)
+        e1.synchronize()
+        t.cuda.synchronize(dev)
+        ms_run = e0.elapsed_time(e1)
+        runs.append({"ms": ms_run, "in_steps_gbs": h2d * steps / (ms_run * 1e-3) / 1e9,
+                     "alone_gbs_min": min(alone), "alone_gbs_median": statistics.median(alone),
+                     "staging_replaced": None if staging is None else staging["replaced"]})
     check = float(loss_host.item())
     del host_mb
     pinned.close()
-    copy_gbs = {"min": min(alone), "median": statistics.median(alone), "max": max(alone),
-                "in_steps": h2d * steps / (ms * 1e-3) / 1e9, "staging": pinned.qualified}
+    ms = statistics.median(r["ms"] for r in runs)
+    copy_gbs = {"in_steps_median": h2d * steps / (ms * 1e-3) / 1e9, "runs": runs,
+                "staging_unit_bytes": None if pinned.qualified is None else pinned.qualified["unit_bytes"]}
     return ms, h2d, d2h, check, ("whole batch" if whole else "ring of 2 microbatches") + ", " + host_kind, copy_gbs
 
 
@@ -1068,8 +1142,9 @@ def main():
     if not args.no_e2e:
         e_ms, h2d, d2h, e_loss, src, copy_gbs = e2e_run(torch, R, batch, dev, args.e2e_steps, 2)
         e2e = {"value": batch.T / (e_ms / 1e3 / args.e2e_steps) * world, "unit": UNIT, "h2d_bytes_per_step": h2d,
-               "d2h_bytes_per_step": d2h, "steps": args.e2e_steps, "loss": e_loss, "host_source": src,
-               "h2d_gbs": copy_gbs,
+               "d2h_bytes_per_step": d2h, "steps": args.e2e_steps, "repetitions": len(copy_gbs["runs"]),
+               "value_of": "median of the repetitions, each `steps` timed steps", "loss": e_loss,
+               "host_source": src, "h2d_gbs": copy_gbs,
                "note": "per step: metadata and every microbatch's logits from pinned host memory, loss read "
                        "back; the gradient stays in HBM for the model's backward"}
 

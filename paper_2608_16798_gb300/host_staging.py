@@ -5,13 +5,15 @@ registered with the CUDA runtime. Its units (a whole number of huge pages, at le
 ``min_unit`` bytes) can be qualified: a caller-supplied probe times a host-to-device copy
 from each unit, and units well below the median are moved out of the way (``mremap``; they
 stay allocated until ``close()`` so that the kernel cannot hand the same physical pages back)
-and replaced in place by fresh pages. The virtual addresses never change, so the whole buffer
-stays one registered range that a single copy can read from end to end.
+and replaced in place by fresh pages, which the caller refills. The virtual addresses never
+change, so the whole buffer stays one registered range that a single copy can read from end to
+end.
 
 On virtual machines, a few physical huge pages can be much slower sources of device reads
-than the rest (8-72 GB/s against 210 GB/s from the others, measured on GB300 hosts): which
-pages are slow changes from one process to the next and stays the same within it.
-Qualification costs one copy per unit and runs before any timed work.
+than the rest (3-72 GB/s against 210 GB/s from the others, measured on GB300 hosts): which
+pages are slow changes from one process to the next, stays the same within it once the data is
+written, and can change when the buffer is first written. Qualification costs one copy per unit
+and runs after the buffer is filled, before any timed work.
 
 The memory calls are made through libc with ctypes (Linux only); registration and the probe
 are injected, so the logic runs without a GPU.
@@ -150,9 +152,13 @@ class HostStagingBuffer:
     def n_units(self) -> int:
         return self.size // self.unit
 
-    def qualify(self, probe, slow_frac: float = 0.6, max_rounds: int = 4) -> dict:
+    def qualify(self, probe, refill=None, slow_frac: float = 0.6, max_rounds: int = 4) -> dict:
         """Time each unit with probe(offset, nbytes) -> GB/s; replace units below slow_frac x the
-        median and probe them again, at most max_rounds times. Returns a summary."""
+        median, call refill(offset, nbytes) for each replaced unit (its fresh pages read as zero),
+        and probe them again, at most max_rounds times. Returns a summary.
+
+        Qualify a buffer after writing its contents: on the hosts measured, pages that copied fast
+        while untouched could turn slow once the buffer was first written."""
         gbs = [float(probe(u * self.unit, self.unit)) for u in range(self.n_units)]
         ref = statistics.median(gbs)
         for _ in range(max_rounds):
@@ -162,6 +168,8 @@ class HostStagingBuffer:
             self.rounds += 1
             self._replace(slow)
             for u in slow:
+                if refill is not None:
+                    refill(u * self.unit, self.unit)
                 gbs[u] = float(probe(u * self.unit, self.unit))
         self.unit_gbs = gbs
         return self.summary()

@@ -44,29 +44,37 @@ def test_qualification_replaces_only_slow_units():
         for u in range(n):
             full[u * unit:(u + 1) * unit] = u + 1  # a pattern per unit
         stays_slow = {1: 1, 3: 2}  # unit -> number of probes that still read slow
-        probed = []
+        calls = []
 
         def probe(off, nbytes):
             assert nbytes == unit and off % unit == 0
             u = off // unit
-            probed.append(u)
+            calls.append(("probe", u))
             if stays_slow.get(u, 0):
                 stays_slow[u] -= 1
                 return 12.0
             return 210.0
 
-        s = b.qualify(probe)
-        assert probed == list(range(n)) + [1, 3, 3]
+        def refill(off, nbytes):
+            u = off // unit
+            fresh = _arr(b, whole=True)[off:off + nbytes]
+            assert not fresh.any(), "a replaced unit starts with fresh (zero) pages"
+            fresh[:] = 100 + u
+            calls.append(("refill", u))
+
+        s = b.qualify(probe, refill)
+        assert calls == [("probe", u) for u in range(n)] + [
+            ("refill", 1), ("probe", 1), ("refill", 3), ("probe", 3), ("refill", 3), ("probe", 3)]
         assert s["replaced"] == 3 and s["rounds"] == 2 and s["unit_gbs_min"] == 210.0
         assert b.addr == addr and events == ["reg", "unreg", "reg", "unreg", "reg"]
         full = _arr(b, whole=True)
-        for u in range(n):  # replaced units hold fresh (zero) pages, the others kept their data
-            want = 0 if u in (1, 3) else u + 1
+        for u in range(n):  # replaced units hold the refilled data, the others kept theirs
+            want = 100 + u if u in (1, 3) else u + 1
             assert (full[u * unit:(u + 1) * unit] == want).all(), u
         # the pages moved out are still mapped, with their data, outside the buffer
         assert len(b.quarantine) == 3
-        # (units 1 and 3 of the first round held their patterns; unit 3's second-round pages were fresh)
-        for (qa, qn), want in zip(b.quarantine, (2, 4, 0)):
+        # (units 1 and 3 held their patterns in the first round; unit 3 its refill in the second)
+        for (qa, qn), want in zip(b.quarantine, (2, 4, 103)):
             assert not (addr <= qa < addr + b.size) and qn == unit
             q = np.frombuffer((ctypes.c_uint8 * qn).from_address(qa), dtype=np.uint8)
             assert (q == want).all()
