@@ -166,7 +166,8 @@ rl_status rl_group_advantages(int32_t n_traj, int32_t n_groups, const int32_t* g
  *   lse_r = log sum_v exp(z_rv), logp_r = z_{r,a_r} - lse_r, H_r = -sum_v p_rv log p_rv.
  *
  *   logits       [rows x ld] of `dtype`; base 16-byte aligned
- *   rows, V, ld  rows >= 0, 1 <= V <= ld
+ *   rows, V, ld  rows >= 0, 1 <= V <= ld; V at most 819,200 (bf16) or 409,600 (fp32): a
+ *                row is spread over at most 16 CTAs of 100 KB (RL_ERR_UNSUPPORTED above)
  *   token_ids    int32 [rows]: a_r (out of range -> logp_r = NaN and RL_DEV_BAD_TOKEN)
  *   logp_out     float [rows]
  *   entropy_out  float [rows] or NULL (entropy work is skipped when NULL)
@@ -197,7 +198,8 @@ rl_status rl_token_logprobs(const void* logits, rl_dtype dtype, int64_t rows, in
  * loss term, statistics and gradient NaN (so the loss is NaN) and leaves the other rows alone.
  *
  *   logits        [rows x ld] of `dtype`, base 16-byte aligned
- *   rows, V, ld   rows >= 0, 1 <= V <= ld
+ *   rows, V, ld   rows >= 0, 1 <= V <= ld; V at most 819,200 (bf16) or 409,600 (fp32), as
+ *                 for rl_token_logprobs (RL_ERR_UNSUPPORTED above)
  *   token_ids     int32 [rows]
  *   mask          uint8 [rows]: M_t
  *   token_traj    int32 [rows]: trajectory of each row (index into adv / coef)

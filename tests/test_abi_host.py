@@ -95,6 +95,17 @@ def test_policy_loss_argument_checks(R):
     assert _loss(R, rows=0) == 0      # nothing to do: returns before any launch
 
 
+def test_largest_vocabulary_rows(R):
+    """A row is spread over at most 16 CTAs of 100 KB: up to 819,200 bf16 or 409,600 fp32 entries
+    pass the shape checks (these calls then stop at the NULL params, before any launch); one
+    more entry is unsupported."""
+    assert _loss(R, V=819_200, ld=819_200, params=None) == 1
+    assert _loss(R, V=819_201, ld=819_201, params=None) == 2
+    assert _loss(R, dt=R.RL_F32, V=409_600, ld=409_600, params=None) == 1
+    assert _loss(R, dt=R.RL_F32, V=409_601, ld=409_601, params=None) == 2
+    assert "16 x 100 KB" in R.rl_last_error_message()
+
+
 def test_token_logprobs_argument_checks(R):
     L = R.lib()
 

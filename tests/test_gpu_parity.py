@@ -131,7 +131,8 @@ def test_group_advantages_bad_offsets_flagged(R):
 @pytest.mark.parametrize("name,row0,rows,vocab,ld_pad", [
     ("tiny", 0, 512, None, 0), ("multiturn", 700, 48, None, 0), ("edge", 0, 1024, None, 0),
     ("multiturn", 0, 16, 1001, 0), ("tiny", 0, 40, 4097, 3), ("edge", 0, 64, 999, 5),
-    ("multiturn", 0, 8, 400_000, 0), ("tiny", 0, 7, 1, 0), ("tiny", 0, 9, 3, 8)])
+    ("multiturn", 0, 8, 400_000, 0), ("multiturn", 0, 6, 819_200, 0), ("edge", 0, 6, 409_600, 0),
+    ("tiny", 0, 7, 1, 0), ("tiny", 0, 9, 3, 8)])
 def test_token_logprobs_parity(R, name, row0, rows, vocab, ld_pad):
     case = make_case(name, seed=1, row0=row0, rows=rows, vocab=vocab)
     V = case.raw.shape[1]
@@ -177,7 +178,8 @@ def test_policy_loss_parity(R, name, row0, rows, agg, tis):
 
 @pytest.mark.parametrize("vocab,ld_pad,dtype_case", [
     (1001, 0, "multiturn"), (4097, 3, "tiny"), (999, 1, "edge"), (400_000, 0, "multiturn"), (3, 5, "tiny"),
-    (1, 0, "tiny"), (151_936, 16, "multiturn")])
+    (1, 0, "tiny"), (151_936, 16, "multiturn"),
+    (819_200, 0, "multiturn"), (409_600, 8, "edge")])  # the largest rows: 16 CTAs of 100 KB
 def test_policy_loss_ragged_shapes(R, vocab, ld_pad, dtype_case):
     case = make_case(dtype_case, seed=4, rows=24, vocab=vocab, loss_agg=2)
     out = run_loss(R, case, ld=vocab + ld_pad)
