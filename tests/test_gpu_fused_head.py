@@ -126,6 +126,8 @@ def compare_head(c, out, dh_bf16=False):
     (130, 64, 513, 1, False, True),        # TIS, token-mean, smallest D
     (100, 128, 777, 0, True, False),       # one CTA pair whose odd CTA's 128 tokens all lie past T
     (5, 64, 300, 2, False, False),         # a handful of tokens
+    (40, 64, 524_288, 2, False, False),    # the largest vocabulary (128 blocks of 4,096)
+    (8, 65_536, 256, 0, True, False),      # the largest hidden size (1,024 K slices per tile)
 ])
 def test_fused_head_parity(R, T, D, V, agg, ent, tis):
     c = make_head_case(T, D, V, seed=T + V, agg=agg, ent=ent, tis=tis)
