@@ -953,10 +953,10 @@ def profile_head(T):
     return 0 if word == 0 else 1
 
 
-def profile_case(rows):
-    """A small slice of the workload for profiler captures: the first `rows` packed tokens
-    (logits resident on the device), then three rl_policy_loss_fwd_bwd launches and three
-    rl_token_logprobs launches."""
+def profile_case(rows, workload="multiturn"):
+    """A small slice of a workload for profiler captures: the first `rows` packed tokens
+    (logits resident on the device), then three rl_policy_loss_fwd_bwd launches (with the
+    workload's entropy and KL terms) and three rl_token_logprobs launches."""
     import torch
 
     from paper_2608_16798_gb300 import build as B
@@ -965,31 +965,38 @@ def profile_case(rows):
     import paper_2608_16798_gb300.rl_loss as R
 
     dev = torch.device("cuda", 0)
-    w = WORKLOAD
+    w = W.WORKLOADS[workload]
     lay = W.make_layout(w, 0)
     rows = min(rows, lay.n_tokens)
-    logits = torch.empty((rows, w.vocab), dtype=torch.bfloat16, device=dev)
+    dt = torch.bfloat16 if w.dtype == "bf16" else torch.float32
+    logits = torch.empty((rows, w.vocab), dtype=dt, device=dev)
     W.logits_rows_torch(w, 0, 0, rows, logits)
     ids = W.sample_tokens_torch(logits, 0, 0, w)
     d = lambda x: torch.from_numpy(np.ascontiguousarray(x)).to(dev)  # noqa: E731
-    params = R.make_params()
+    params = R.make_params(W.CLIP_EPS_LOW, W.CLIP_EPS_HIGH, w.kl_coef, 3 if w.kl_coef else 0, w.entropy_coef,
+                           0.0, 1e-6, 0)
     ws = R.new_workspace(rows, w.vocab, device=dev)
     adv, coef, n_tok, tt = R.rl_group_advantages(d(lay.group_offsets), d(lay.rewards), d(lay.traj_offsets),
-                                                 d(lay.mask), params, ws)
+                                                 d(lay.mask), params, ws, traj_valid=d(lay.traj_valid))
     logp, _, _ = R.rl_token_logprobs(logits, ids, ws)
-    old = d(W.old_logp_from(logp.cpu().numpy(), w, 0))
+    lp = logp.cpu().numpy()
+    old = d(W.old_logp_from(lp, w, 0))
+    ref = d(W.ref_logp_from(lp, w, 0)) if w.ref_noise_std else None
     grad = torch.empty_like(logits)
     loss = torch.zeros(1, dtype=torch.float64, device=dev)
     mask = d(lay.mask[:rows])
     for _ in range(3):
-        R.rl_policy_loss_fwd_bwd(logits, ids, mask, tt[:rows], adv, coef, old, params, ws, loss, grad_out=grad)
+        R.rl_policy_loss_fwd_bwd(logits, ids, mask, tt[:rows], adv, coef, old, params, ws, loss, grad_out=grad,
+                                 ref_logp=ref)
     for _ in range(3):
         R.rl_token_logprobs(logits, ids, ws, logp_out=logp)
     st, word = R.rl_query_status(ws)
     m = lay.mask[:rows].astype(np.int64)
-    print(json.dumps({"profile_case_rows": rows, "trained_rows": int(m.sum()), "status": word,
-                      "algorithmic_bytes_fwd_bwd": int(((m + 1) * w.vocab * 2).sum()),
-                      "algorithmic_bytes_fwd": rows * w.vocab * 2}))
+    es = 2 if w.dtype == "bf16" else 4
+    trained = m * (coef.cpu().numpy()[tt[:rows].cpu().numpy()] != 0)
+    print(json.dumps({"profile_case_rows": rows, "workload": workload, "trained_rows": int(trained.sum()),
+                      "status": word, "algorithmic_bytes_fwd_bwd": int(((trained + 1) * w.vocab * es).sum()),
+                      "algorithmic_bytes_fwd": rows * w.vocab * es}))
     return 0 if word == 0 else 1
 
 
@@ -1047,6 +1054,8 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--profile-case", type=int, default=0, metavar="ROWS",
                     help="run a small slice of the workload for a profiler capture and exit")
+    ap.add_argument("--profile-workload", default="multiturn", choices=["tiny", "multiturn", "longhorizon", "edge"],
+                    help="workload of --profile-case (default: the benchmark's multiturn)")
     ap.add_argument("--profile-head", type=int, default=0, metavar="TOKENS",
                     help="run a small fused-head case for a profiler capture and exit")
     ap.add_argument("--profile-ppo", type=int, default=0, metavar="STEPS",
@@ -1057,7 +1066,7 @@ def main():
     ap.add_argument("--no-other", action="store_true", help="skip the long-horizon and edge workloads")
     args = ap.parse_args()
     if args.profile_case:
-        return profile_case(args.profile_case)
+        return profile_case(args.profile_case, args.profile_workload)
     if args.profile_head:
         return profile_head(args.profile_head)
     if args.profile_ppo:
