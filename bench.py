@@ -185,7 +185,8 @@ class DeviceBatch:
                 events[k][1].record()
 
     def launches_per_step(self):
-        return 2 + 2 * len(self.mbs)
+        # rl_group_advantages: 2 kernels; rl_policy_loss_fwd_bwd: 1 kernel per microbatch
+        return 2 + len(self.mbs)
 
 
 def time_logits_extras(torch, R, batch, dev, peak, reps=20):
@@ -1132,7 +1133,7 @@ def main():
     achieved = per_launch_bytes / (avg_launch_ms * 1e-3) / 1e9
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                 "traffic": profiled_traffic(), "peak_source": peak_kind,
-                "kernel": "rows_kernel<bf16> via rl_policy_loss_fwd_bwd (+ 1-CTA loss reduction)",
+                "kernel": "rows_kernel<bf16> via rl_policy_loss_fwd_bwd (one launch; its last cluster sums the loss)",
                 "algorithmic_bytes_per_launch": per_launch_bytes, "avg_launch_ms": avg_launch_ms,
                 "frac_of_nominal_8tbs": achieved / 8000.0}
     # per microbatch: median and best launch over the timed steps, and each one's GB/s

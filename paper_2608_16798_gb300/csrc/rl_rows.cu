@@ -21,9 +21,11 @@
 // trajectories with c_i = 0) are not read at all, only zero-filled.
 //
 // The kernels are persistent: the grid holds as many clusters as fit on the
-// GPU at once, and cluster j processes rows j, j + n_clusters, ... . Per-row
-// loss contributions go to the workspace and are summed in a fixed order by a
-// one-CTA kernel, so the loss is bit-reproducible.
+// GPU at once, and cluster j processes rows j, j + n_clusters, ... . Each
+// cluster adds its rows' loss contributions in row order and leaves one partial
+// in the workspace; the last cluster to finish (a counter in the workspace
+// header) sums the partials in a fixed order into the caller's total, so the
+// loss is bit-reproducible without a second launch.
 #include <algorithm>
 #include <cstdint>
 #include <map>
@@ -55,6 +57,8 @@ struct RowArgs {
   float tis_cap;           // <= 0 when TIS is off
   int32_t adv_per_row;     // adv holds one A_t per row (else one per trajectory)
   double* row_loss;
+  double* loss_accum;      // the caller's total (loss kernel: the last cluster adds into it)
+  uint32_t* done;          // finished-cluster count in the workspace header
   float* token_stats;
   float* logp_out;
   float* entropy_out;
@@ -727,7 +731,29 @@ __global__ void __launch_bounds__((NW + 1) * 32, 2) rows_kernel(const RowArgs p)
         if (lane == 0) mbar_arrive(&empty_bar[b]);
       }
     }
-    if (BWD && rank == 0 && warp == 0 && lane == 0) p.row_loss[cid] = cl_loss;  // cid < clusters <= rows
+    if (BWD && rank == 0 && warp == 0) {
+      // one partial per cluster (cid < clusters <= rows); the last cluster to finish adds all
+      // of them, in a fixed order, into the caller's total, so no second launch is needed
+      __syncwarp();
+      uint32_t last = 0;
+      if (lane == 0) {
+        p.row_loss[cid] = cl_loss;
+        __threadfence();
+        last = atomicAdd(p.done, 1u) == static_cast<uint32_t>(ncl - 1) ? 1u : 0u;
+        if (last) __threadfence();
+      }
+      __syncwarp();
+      last = __shfl_sync(0xffffffffu, last, 0);
+      if (last) {
+        double t = 0.0;
+        for (int64_t k = lane; k < ncl; k += 32) t += __ldcg(p.row_loss + k);
+        t = warp_sum(t);
+        if (lane == 0) {
+          *p.loss_accum += t;
+          *p.done = 0u;
+        }
+      }
+    }
   }
   __syncthreads();
   // no CTA leaves while a peer may still write into its mailbox
@@ -1006,7 +1032,7 @@ static rl_status launch_rows(const RowArgs& args, const Plan& plan, cudaStream_t
 constexpr int kHoldVecs = 11;
 
 // Launches the loss kernel; *n_clusters receives the number of clusters, each of which leaves
-// one loss partial at the head of the per-row loss area.
+// one loss partial at the head of the per-row loss area (the last one also adds them up).
 template <typename T>
 static rl_status dispatch_loss(bool ent, const RowArgs& args, const Plan& plan, cudaStream_t s, int64_t* n_clusters) {
   const bool hold = plan.slice * static_cast<int64_t>(sizeof(T)) / 16 <= int64_t(kHoldVecs) * kConsumerWarps * 32;
@@ -1155,6 +1181,8 @@ extern "C" rl_status rl_policy_loss_fwd_bwd(const void* logits, rl_dtype dtype, 
   a.adv_per_row = params->token_level_adv;
   double* row_loss = reinterpret_cast<double*>(static_cast<char*>(ws) + ws_row_loss_offset());
   a.row_loss = row_loss;
+  a.loss_accum = loss_accum;
+  a.done = reinterpret_cast<uint32_t*>(static_cast<char*>(ws) + kWsDoneOffset);
   a.token_stats = token_stats;
   a.status = reinterpret_cast<int32_t*>(ws);
   a.slice = plan.slice;
@@ -1165,6 +1193,5 @@ extern "C" rl_status rl_policy_loss_fwd_bwd(const void* logits, rl_dtype dtype, 
   int64_t n_clusters = 0;
   st = dtype == RL_BF16 ? dispatch_loss<uint16_t>(ent, a, plan, s, &n_clusters)
                         : dispatch_loss<float>(ent, a, plan, s, &n_clusters);
-  if (st != RL_OK) return st;
-  return launch_reduce_loss(row_loss, n_clusters, loss_accum, s);
+  return st;  // the kernel's last cluster has added the loss into loss_accum
 }
