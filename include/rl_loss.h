@@ -116,9 +116,10 @@ const char* rl_last_error_message(void);
  * 32,768 tokens). */
 size_t rl_workspace_size(int64_t max_rows, int64_t V, int64_t D);
 
-/* Zero the workspace's 256-byte header: the status word and the loss kernel's
- * finished-cluster counter (which each launch leaves at zero again). Call once
- * after allocating a workspace, and again to clear a reported device error. */
+/* Zero the workspace's 256-byte header: the status word and the finished-block
+ * counters of the policy and value losses (which each launch leaves at zero
+ * again). Call once after allocating a workspace, and again to clear a reported
+ * device error. */
 rl_status rl_workspace_init(void* ws, size_t ws_bytes, rl_stream_t stream);
 
 /* Synchronise `stream`, then read the device status word into

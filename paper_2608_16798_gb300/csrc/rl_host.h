@@ -22,6 +22,8 @@ inline size_t ws_row_loss_offset() { return kWsHeader; }
 // Header word counting the loss kernel's finished clusters (zeroed by rl_workspace_init; the
 // last cluster of each launch resets it).
 constexpr size_t kWsDoneOffset = 16;
+// The same for the value loss kernel's finished CTAs.
+constexpr size_t kWsValueDoneOffset = 20;
 
 rl_status set_error(rl_status st, const std::string& msg);
 rl_status cuda_error(cudaError_t e, const char* what);

@@ -15,8 +15,8 @@
 //                                         itself the suffix scan of the selection map
 //                                         x_t = M_t ? V_t : x_{t+1} (exact in fp32)
 //   value_loss_kernel  per token: c M (V - G)^2, added per CTA in a fixed order into one
-//                      partial per CTA, and dV = 2 c M (V - G); the fixed-order reduction
-//                      adds the partials into the caller's accumulator.
+//                      partial per CTA, and dV = 2 c M (V - G); the last CTA to finish adds
+//                      the partials, in a fixed order, into the caller's accumulator.
 //   rollout_adv_kernel A_t = R_i - V_t, G_t = R_i per token for tokens in any order (the
 //                      gamma = lambda = 1 form of Sec. 2.3.4, which also holds on the shared
 //                      prefixes of a rollout's prefix tree).
@@ -194,13 +194,17 @@ struct ValueArgs {
   const float* coef;
   float* d_values;
   double* row_loss;
+  double* loss_accum;
+  uint32_t* done;  // finished-CTA count in the workspace header
   int32_t* status;
 };
 
 // Each CTA adds its rows' terms in a fixed order (thread-strided, then warp and CTA) and leaves
-// one partial per CTA in row_loss[blockIdx.x]; the reduction then adds the partials in order.
+// one partial per CTA in row_loss[blockIdx.x]; the last CTA to finish (a counter in the
+// workspace header, which it resets) adds the partials in a fixed order into loss_accum.
 __global__ void __launch_bounds__(256) value_loss_kernel(const ValueArgs p) {
   __shared__ double part[8];
+  __shared__ uint32_t last;
   double acc = 0.0;
   for (int64_t t = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < p.rows;
        t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
@@ -222,6 +226,23 @@ __global__ void __launch_bounds__(256) value_loss_kernel(const ValueArgs p) {
     double t = 0.0;
     for (int w = 0; w < 8; ++w) t += part[w];
     p.row_loss[blockIdx.x] = t;
+    __threadfence();
+    last = atomicAdd(p.done, 1u) == gridDim.x - 1 ? 1u : 0u;
+    if (last) __threadfence();
+  }
+  __syncthreads();
+  if (last) {  // uniform across the CTA
+    double t = 0.0;
+    for (uint32_t k = threadIdx.x; k < gridDim.x; k += blockDim.x) t += __ldcg(p.row_loss + k);
+    t = warp_sum(t);
+    if ((threadIdx.x & 31) == 0) part[threadIdx.x >> 5] = t;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      double u = 0.0;
+      for (int w = 0; w < 8; ++w) u += part[w];
+      *p.loss_accum += u;
+      *p.done = 0u;
+    }
   }
 }
 
@@ -320,13 +341,15 @@ extern "C" rl_status rl_value_loss_fwd_bwd(int64_t rows, const float* values, co
   a.d_values = d_values;
   double* row_loss = reinterpret_cast<double*>(static_cast<char*>(ws) + ws_row_loss_offset());
   a.row_loss = row_loss;
+  a.loss_accum = loss_accum;
+  a.done = reinterpret_cast<uint32_t*>(static_cast<char*>(ws) + kWsValueDoneOffset);
   a.status = reinterpret_cast<int32_t*>(ws);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   const int blocks = ppo::grid_for(rows, 256, 152 * 16);  // <= rows: one partial per CTA fits
   ppo::value_loss_kernel<<<blocks, 256, 0, s>>>(a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_error(e, "value_loss_kernel launch");
-  return launch_reduce_loss(row_loss, blocks, loss_accum, s);
+  return RL_OK;  // the kernel's last CTA has added the loss into loss_accum
 }
 
 extern "C" rl_status rl_rollout_value_advantages(int64_t n_tokens, const int32_t* token_traj, const uint8_t* mask,
