@@ -122,6 +122,22 @@ size_t rl_workspace_size(int64_t max_rows, int64_t V, int64_t D);
  * device error. */
 rl_status rl_workspace_init(void* ws, size_t ws_bytes, rl_stream_t stream);
 
+/*
+ * Self-test of the failure path (no counterpart in the paper): one CTA waits, through the
+ * kernels' own bounded waits (the plain and the cluster-scope form), on an mbarrier that
+ * nothing arrives at. Each wait gives up after limit_ns nanoseconds of %globaltimer (the
+ * kernels use 2e9); the kernel then sets RL_DEV_TIMEOUT in the status word and returns, so
+ * rl_query_status reports RL_ERR_TIMEOUT and the context stays usable (rl_workspace_init
+ * clears the word). No fault, trap or unbounded wait is involved.
+ *
+ *   ws, ws_bytes  workspace (its status word is set), at least the 256-byte header
+ *   limit_ns      in [1e3, 2e9]
+ *   waited_ns     device uint64 (or NULL): receives the longest time the CTA spent waiting
+ *                 (max with its previous value)
+ */
+rl_status rl_selftest_bounded_wait(void* ws, size_t ws_bytes, int64_t limit_ns, uint64_t* waited_ns,
+                                   rl_stream_t stream);
+
 /* Synchronise `stream`, then read the device status word into
  * *device_status_out (0 = no error; else RL_DEV_* bits). Returns RL_OK,
  * RL_ERR_DEVICE_CHECK or RL_ERR_TIMEOUT. The word is not cleared. */

@@ -35,6 +35,7 @@ EXPORTS = {
     "rl_workspace_size": (_SZ, [_I64, _I64, _I64]),
     "rl_workspace_init": (_I32, [_P, _SZ, _P]),
     "rl_query_status": (_I32, [_P, _P, ctypes.POINTER(_I32)]),
+    "rl_selftest_bounded_wait": (_I32, [_P, _SZ, _I64, _P, _P]),
     "rl_group_advantages": (_I32, [_I32, _I32, _P, _P, _P, _I64, _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P]),
     "rl_token_logprobs": (_I32, [_P, _I32, _I64, _I64, _I64, _P, _P, _P, _P, _P, _SZ, _P]),
     "rl_policy_loss_fwd_bwd": (_I32, [_P, _I32, _I64, _I64, _I64, _P, _P, _P, _I32, _P, _P, _P, _P, _P, _P,
@@ -164,6 +165,15 @@ def rl_workspace_size(max_rows: int, V: int, D: int = 0) -> int:
 def rl_workspace_init(ws: torch.Tensor, stream=None):
     _need(ws, "ws", torch.uint8)
     _check("rl_workspace_init", lib().rl_workspace_init(_ptr(ws), ws.numel(), _stream(stream)))
+
+
+def rl_selftest_bounded_wait(ws: torch.Tensor, limit_ns: int, waited_ns: torch.Tensor | None = None, stream=None):
+    """Run one bounded wait that runs out (the failure path of every kernel wait); afterwards
+    rl_query_status reports RL_ERR_TIMEOUT. waited_ns: optional int64 [1] on the device."""
+    _need(ws, "ws", torch.uint8)
+    _opt(waited_ns, "waited_ns", torch.int64, 1, device=ws.device)
+    _check("rl_selftest_bounded_wait",
+           lib().rl_selftest_bounded_wait(_ptr(ws), ws.numel(), int(limit_ns), _ptr(waited_ns), _stream(stream)))
 
 
 def new_workspace(max_rows: int, V: int, D: int = 0, device=None, stream=None) -> torch.Tensor:

@@ -145,6 +145,16 @@ def test_group_advantages_argument_checks(R):
     assert call(n=0) == 0
 
 
+def test_selftest_bounded_wait_argument_checks(R):
+    L = R.lib()
+    assert L.rl_selftest_bounded_wait(None, 1 << 20, 1_000_000, None, None) == 1
+    assert L.rl_selftest_bounded_wait(FAKE, 100, 1_000_000, None, None) == 4
+    assert L.rl_selftest_bounded_wait(FAKE + 8, 1 << 20, 1_000_000, None, None) == 3
+    assert L.rl_selftest_bounded_wait(FAKE, 1 << 20, 999, None, None) == 1
+    assert L.rl_selftest_bounded_wait(FAKE, 1 << 20, 2_000_000_001, None, None) == 1
+    assert "limit_ns" in R.rl_last_error_message()
+
+
 def test_status_and_init_argument_checks(R):
     L = R.lib()
     assert L.rl_workspace_init(None, 1024, None) == 1
