@@ -483,7 +483,18 @@ class StagedPinned:
             if n:
                 units[off:off + n].copy_(src[off:off + n])
 
-        self.qualified = self.buf.qualify(probe, refill)
+        try:
+            self.qualified = self.buf.qualify(probe, refill)
+        except OSError as exc:
+            self.qualified = {"error": str(exc), "replaced": self.buf.replaced, "unit_bytes": self.buf.unit}
+            if self.buf.broken:  # never copy from a range with a hole: torch's pinned memory instead
+                rows, cols = self.tensor.shape
+                dtype = self.tensor.dtype
+                del units
+                self.close()
+                self.tensor = t.empty((rows, cols), dtype=dtype, pin_memory=True)
+                self.tensor.view(-1).copy_(source.view(-1)[:self.tensor.numel()])
+                self.kind = "torch pinned (a staging unit could not be replaced)"
         t.cuda.synchronize(self.dev)
 
     def close(self):
@@ -530,7 +541,9 @@ def e2e_run(torch, R, batch, dev, steps, warmup, slots=4, repeats=3):
         for lo, hi in batch.mbs:
             pinned.tensor[lo:hi].copy_(batch.logits[lo:hi])
         pinned.qualify(batch.logits)
-        host_mb = [pinned.tensor[lo:hi] for lo, hi in batch.mbs]
+
+        def make_host_views():
+            return [pinned.tensor[lo:hi] for lo, hi in batch.mbs]
     else:
         pinned = StagedPinned(t, 2 * mb, V, t.bfloat16, dev)
         for k in range(2):
@@ -538,9 +551,11 @@ def e2e_run(torch, R, batch, dev, steps, warmup, slots=4, repeats=3):
             pinned.tensor[k * mb:k * mb + hi - lo].copy_(batch.logits[lo:hi])
         if len(batch.mbs) >= 2:  # the ring then holds the batch's first 2 x mb rows, byte for byte
             pinned.qualify(batch.logits)
-        host_mb = [pinned.tensor[(k % 2) * mb:(k % 2) * mb + hi - lo] for k, (lo, hi) in enumerate(batch.mbs)]
+
+        def make_host_views():
+            return [pinned.tensor[(k % 2) * mb:(k % 2) * mb + hi - lo] for k, (lo, hi) in enumerate(batch.mbs)]
+    host_mb = make_host_views()
     src = list(range(len(batch.mbs)))
-    host_kind = pinned.kind
     meta_host = {n: getattr(batch, n).cpu().pin_memory() for n in
                  ("ids", "mask", "old", "rewards", "group_offsets", "traj_offsets", "valid")}
     meta_dev = {n: t.empty_like(getattr(batch, n)) for n in meta_host}
@@ -603,8 +618,9 @@ def e2e_run(torch, R, batch, dev, steps, warmup, slots=4, repeats=3):
     # the box, pages of a qualified buffer were seen to turn slow later in the same process)
     runs = []
     for rep in range(repeats):
-        if rep > 0:
+        if rep > 0 and (whole or len(batch.mbs) >= 2):
             pinned.qualify(batch.logits)
+            host_mb[:] = make_host_views()  # the buffer may have been replaced
         staging = pinned.qualified
         alone = copies_alone()
         t.cuda.synchronize(dev)
@@ -628,7 +644,7 @@ def e2e_run(torch, R, batch, dev, steps, warmup, slots=4, repeats=3):
     ms = statistics.median(r["ms"] for r in runs)
     copy_gbs = {"in_steps_median": h2d * steps / (ms * 1e-3) / 1e9, "runs": runs,
                 "staging_unit_bytes": None if pinned.qualified is None else pinned.qualified["unit_bytes"]}
-    return ms, h2d, d2h, check, ("whole batch" if whole else "ring of 2 microbatches") + ", " + host_kind, copy_gbs
+    return ms, h2d, d2h, check, ("whole batch" if whole else "ring of 2 microbatches") + ", " + pinned.kind, copy_gbs
 
 
 # ----------------------------------------------------------------------------- oracle (CPU) legs

@@ -93,6 +93,7 @@ class HostStagingBuffer:
         self.rounds = 0
         self.unit_gbs: list[float] = []
         self.registered = False
+        self.broken = False  # set if a failed replacement left part of the range unmapped
         # reserve size + one huge page, keep the aligned part
         raw = _check_map(lib.mmap(None, self.size + self.hp, _PROT_RW, mmap.MAP_PRIVATE | mmap.MAP_ANONYMOUS, -1, 0),
                          "mmap")
@@ -127,25 +128,37 @@ class HostStagingBuffer:
             self.registered = False
 
     def _replace(self, units):
-        """Move the given units out of the way (kept allocated) and map fresh pages in place."""
+        """Move the given units out of the way (kept allocated) and map fresh pages in place.
+        The buffer is registered again even when a step fails (the error is then raised)."""
         lib = _lib()
         self._unpin()
-        for u in units:
-            off = u * self.unit
-            # a same-size mremap without a destination is a no-op: reserve one and move there
-            dest = _check_map(lib.mmap(None, self.unit, 0, mmap.MAP_PRIVATE | mmap.MAP_ANONYMOUS, -1, 0), "mmap")
-            moved = lib.mremap(self.addr + off, self.unit, self.unit, _MREMAP_MAYMOVE | _MREMAP_FIXED, dest)
-            if moved is None or moved == _MAP_FAILED:
-                lib.munmap(dest, self.unit)
-                _check_map(moved, "mremap")
-            self.quarantine.append((moved, self.unit))
-            got = _check_map(lib.mmap(self.addr + off, self.unit, _PROT_RW,
-                                      mmap.MAP_PRIVATE | mmap.MAP_ANONYMOUS | _MAP_FIXED, -1, 0), "mmap fixed")
-            if got != self.addr + off:
-                raise OSError("mmap with MAP_FIXED returned another address")
-            self._prepare(off, self.unit)
-            self.replaced += 1
-        self._pin()
+        try:
+            for u in units:
+                off = u * self.unit
+                # a same-size mremap without a destination is a no-op: reserve one and move there
+                dest = _check_map(lib.mmap(None, self.unit, 0, mmap.MAP_PRIVATE | mmap.MAP_ANONYMOUS, -1, 0),
+                                  "mmap")
+                moved = lib.mremap(self.addr + off, self.unit, self.unit, _MREMAP_MAYMOVE | _MREMAP_FIXED, dest)
+                if moved is None or moved == _MAP_FAILED:
+                    err = ctypes.get_errno()
+                    lib.munmap(dest, self.unit)
+                    raise OSError(err, f"mremap: {os.strerror(err)}")
+                # the unit's range is unmapped now: map fresh pages there, or put the old ones back
+                got = lib.mmap(self.addr + off, self.unit, _PROT_RW,
+                               mmap.MAP_PRIVATE | mmap.MAP_ANONYMOUS | _MAP_FIXED, -1, 0)
+                if got != self.addr + off:
+                    err = ctypes.get_errno()
+                    back = lib.mremap(moved, self.unit, self.unit, _MREMAP_MAYMOVE | _MREMAP_FIXED, self.addr + off)
+                    if back != self.addr + off:
+                        self.broken = True  # a hole in the buffer: it must not be used any more
+                        self.quarantine.append((moved, self.unit))
+                    raise OSError(err, f"mmap fixed: {os.strerror(err)}")
+                self.quarantine.append((moved, self.unit))
+                self._prepare(off, self.unit)
+                self.replaced += 1
+        finally:
+            if not self.broken:
+                self._pin()
 
     # -- qualification --------------------------------------------------------------------------
     @property
@@ -183,8 +196,8 @@ class HostStagingBuffer:
     def buffer(self, whole_units: bool = False):
         """A ctypes array (it supports the buffer protocol) over the first nbytes, or over every
         unit with whole_units. It is valid until close()."""
-        if self.addr is None:
-            raise ValueError("the buffer is closed")
+        if self.addr is None or self.broken:
+            raise ValueError("the buffer is closed" if self.addr is None else "the buffer has a hole")
         return (ctypes.c_uint8 * (self.size if whole_units else self.nbytes)).from_address(self.addr)
 
     def close(self):
@@ -192,7 +205,7 @@ class HostStagingBuffer:
             return
         lib = _lib()
         self._unpin()
-        lib.munmap(self.addr, self.size)
+        lib.munmap(self.addr, self.size)  # unmapping a range with a hole in it is fine
         for a, n in self.quarantine:
             lib.munmap(a, n)
         self.quarantine = []

@@ -97,3 +97,35 @@ def test_refused_registration_raises_and_rejects_bad_size():
         HostStagingBuffer(0)
     with pytest.raises(RuntimeError):
         HostStagingBuffer(1 << 20, lambda a, n: False, lambda a: None)
+
+
+def test_failed_replacement_registers_again(monkeypatch):
+    """A replacement whose fresh mapping is refused puts the old pages back, registers the
+    buffer again and raises; the data and the addresses are unchanged."""
+    import paper_2608_16798_gb300.host_staging as HS
+
+    events = []
+    b = HostStagingBuffer(3 * (4 << 20), lambda a, n: events.append("reg") or True,
+                          lambda a: events.append("unreg"), min_unit=4 << 20)
+    try:
+        full = _arr(b, whole=True)
+        full[:] = 9
+        lib = HS._lib()
+        real_mmap = lib.mmap
+
+        class Refusing:  # refuses MAP_FIXED requests, passes the others through
+            def __call__(self, addr, length, prot, flags, fd, off):
+                if flags & HS._MAP_FIXED:
+                    ctypes.set_errno(12)
+                    return HS._MAP_FAILED
+                return real_mmap(addr, length, prot, flags, fd, off)
+
+        monkeypatch.setattr(lib, "mmap", Refusing())
+        with pytest.raises(OSError):
+            b.qualify(lambda off, n: 1.0 if off // b.unit == 1 else 200.0)
+        monkeypatch.setattr(lib, "mmap", real_mmap)
+        assert not b.broken and b.registered and events[-1] == "reg"
+        assert (_arr(b, whole=True) == 9).all()  # the old pages are back in place
+        assert b.quarantine == []
+    finally:
+        b.close()
