@@ -22,7 +22,9 @@
  *     prefix, and the advantages and counts of their tokens in any order
  *     (Sec. 3.2.1-3.2.3);
  *   - sequence-level importance weights (Sec. 3.2.4) and batch summaries of the
- *     per-token statistics (entropy, clip fraction; Sec. 4).
+ *     per-token statistics (entropy, clip fraction; Sec. 4);
+ *   - a self-test of the failure path that every bounded device wait shares
+ *     (rl_selftest_bounded_wait).
  *
  * Conventions shared by every entry point:
  *   - Array arguments are DEVICE pointers owned by the caller (the one
