@@ -243,6 +243,9 @@ def test_policy_loss_bad_ids_flagged_and_zeroed(R):
     assert np.all(gg[[3, 5]] == 0.0) and np.any(gg[0] != 0.0)
     R.rl_workspace_init(ws)
     assert R.rl_query_status(ws)[1] == 0
+    # the same workspace (its finished-cluster counter included) serves a clean call next
+    clean = make_case("tiny", seed=9, rows=32)
+    compare(clean, run_loss(R, clean, ws=ws), "clean call after the flagged one")
 
 
 def test_end_to_end_advantages_then_loss(R):
