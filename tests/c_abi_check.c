@@ -4,7 +4,8 @@
  * uniform logits (all 0) give logp = -ln V for every token; with old_logp = logp the ratio
  * is 1, nothing is clipped, and the loss is -sum_i c_i L_i A_i, which is 0 for complete
  * groups under RL_AGG_SEQ_MEAN_TOKEN_MEAN; every trained gradient row is
- * -c_i A_i (onehot_a - 1/V). Exit status 0 on success. */
+ * -c_i A_i (onehot_a - 1/V); the fused head, the masked GAE and the value loss are checked
+ * against closed forms too (gpu_checks_more). Exit status 0 on success. */
 #include <math.h>
 #include <stdint.h>
 #include <stdio.h>
@@ -145,9 +146,174 @@ static int gpu_checks(void) {
   return fails;
 }
 
+/* The fused head with all hidden states 0 (so every logits row is 0: uniform), the masked GAE at
+ * gamma = lambda = 1 in the skip reading, and the value loss, each against its closed form:
+ *   fused head: loss as above; dW = dZ^T H = 0 exactly; trained dH rows -c_i A_i (W[a] - mean_v W[v]);
+ *   GAE: A_t = R_i - V_t and G_t = R_i on trainable tokens (Sec. 2.3.4), 0 on masked ones;
+ *   value loss: sum_t c M (V_t - G_t)^2 and dV_t = 2 c M (V_t - G_t). */
+static uint16_t bf16_bits(float x) { /* exact for the small multiples of 1/256 used here */
+  uint32_t u;
+  memcpy(&u, &x, 4);
+  return (uint16_t)(u >> 16);
+}
+
+static int gpu_checks_more(void) {
+  enum { G = 2, PER = 4, N = G * PER, LEN = 24, T = N * LEN, V = 1000, D = 64 };
+  const int32_t go[G + 1] = {0, PER, 2 * PER};
+  float rewards[N];
+  int64_t offs[N + 1];
+  uint8_t mask[T];
+  int32_t ids[T];
+  float old[T], values[T];
+  for (int i = 0; i < N; ++i) rewards[i] = (float)((i * 7) % 3);
+  for (int i = 0; i <= N; ++i) offs[i] = (int64_t)i * LEN;
+  for (int t = 0; t < T; ++t) {
+    mask[t] = (uint8_t)((t % 5) != 0);
+    ids[t] = (t * 37) % V;
+    old[t] = (float)(-log((double)V));
+    values[t] = (float)((t * 13) % 29) / 32.0f;
+  }
+  uint16_t* w = (uint16_t*)malloc((size_t)V * D * 2);
+  float* wf = (float*)malloc((size_t)V * D * 4);
+  for (int v = 0; v < V; ++v)
+    for (int d = 0; d < D; ++d) {
+      wf[v * D + d] = (float)((v * 31 + d * 17) % 97 - 48) / 256.0f;
+      w[v * D + d] = bf16_bits(wf[v * D + d]);
+    }
+  rl_loss_params p;
+  memset(&p, 0, sizeof p);
+  p.clip_eps_low = 0.2f;
+  p.clip_eps_high = 0.28f;
+  p.adv_eps = 1e-6f;
+  p.loss_agg = RL_AGG_SEQ_MEAN_TOKEN_MEAN;
+
+  void *d_go, *d_rw, *d_offs, *d_mask, *d_ids, *d_old, *d_adv, *d_coef, *d_ntok, *d_tt, *d_h, *d_w, *d_dh, *d_dw,
+      *d_loss, *d_ws, *d_val, *d_gadv, *d_ret, *d_dv, *d_vloss;
+  const size_t ws_bytes = rl_workspace_size(T, V, D);
+  int bad = 0;
+  bad |= cudaMalloc(&d_go, sizeof go) | cudaMalloc(&d_rw, sizeof rewards) | cudaMalloc(&d_offs, sizeof offs);
+  bad |= cudaMalloc(&d_mask, sizeof mask) | cudaMalloc(&d_ids, sizeof ids) | cudaMalloc(&d_old, sizeof old);
+  bad |= cudaMalloc(&d_adv, N * 4) | cudaMalloc(&d_coef, N * 4) | cudaMalloc(&d_ntok, N * 4) | cudaMalloc(&d_tt, T * 4);
+  bad |= cudaMalloc(&d_h, (size_t)T * D * 2) | cudaMalloc(&d_w, (size_t)V * D * 2);
+  bad |= cudaMalloc(&d_dh, (size_t)T * D * 4) | cudaMalloc(&d_dw, (size_t)V * D * 4);
+  bad |= cudaMalloc(&d_loss, 8) | cudaMalloc(&d_ws, ws_bytes) | cudaMalloc(&d_val, T * 4);
+  bad |= cudaMalloc(&d_gadv, T * 4) | cudaMalloc(&d_ret, T * 4) | cudaMalloc(&d_dv, T * 4) | cudaMalloc(&d_vloss, 8);
+  if (bad) {
+    fprintf(stderr, "FAIL: cudaMalloc\n");
+    return 1;
+  }
+  cudaMemcpy(d_go, go, sizeof go, H2D);
+  cudaMemcpy(d_rw, rewards, sizeof rewards, H2D);
+  cudaMemcpy(d_offs, offs, sizeof offs, H2D);
+  cudaMemcpy(d_mask, mask, sizeof mask, H2D);
+  cudaMemcpy(d_ids, ids, sizeof ids, H2D);
+  cudaMemcpy(d_old, old, sizeof old, H2D);
+  cudaMemcpy(d_w, w, (size_t)V * D * 2, H2D);
+  cudaMemcpy(d_val, values, sizeof values, H2D);
+  cudaMemset(d_h, 0, (size_t)T * D * 2); /* zero hidden states: uniform logits */
+  cudaMemset(d_dw, 0, (size_t)V * D * 4);
+  cudaMemset(d_loss, 0, 8);
+  cudaMemset(d_vloss, 0, 8);
+  CHECK(rl_workspace_init(d_ws, ws_bytes, NULL) == RL_OK, "workspace init");
+  CHECK(rl_group_advantages(N, G, d_go, d_rw, NULL, T, d_offs, d_mask, &p, d_adv, d_coef, d_ntok, d_tt, d_ws,
+                            ws_bytes, NULL) == RL_OK,
+        "rl_group_advantages: %s", rl_last_error_message());
+  CHECK(rl_fused_head_loss_fwd_bwd(d_h, d_w, T, D, V, d_ids, d_mask, d_tt, N, d_adv, d_coef, d_old, NULL, NULL, &p,
+                                   d_dh, RL_F32, d_dw, d_loss, NULL, d_ws, ws_bytes, NULL) == RL_OK,
+        "rl_fused_head_loss_fwd_bwd: %s", rl_last_error_message());
+  CHECK(rl_masked_gae(N, d_offs, T, d_mask, d_val, NULL, d_rw, 1.0f, 1.0f, 1, d_gadv, d_ret, d_ws, ws_bytes,
+                      NULL) == RL_OK,
+        "rl_masked_gae: %s", rl_last_error_message());
+  CHECK(rl_value_loss_fwd_bwd(T, d_val, d_ret, d_mask, d_tt, N, d_coef, d_dv, d_vloss, d_ws, ws_bytes, NULL) == RL_OK,
+        "rl_value_loss_fwd_bwd: %s", rl_last_error_message());
+  int32_t word = -1;
+  CHECK(rl_query_status(d_ws, NULL, &word) == RL_OK && word == 0, "device status %d", word);
+
+  float adv[N], coef[N], gadv[T], ret[T], dv[T];
+  int32_t ntok[N];
+  double loss = 0.0, vloss = 0.0;
+  float* dh = (float*)malloc((size_t)T * D * 4);
+  float* dw = (float*)malloc((size_t)V * D * 4);
+  cudaMemcpy(adv, d_adv, sizeof adv, D2H);
+  cudaMemcpy(coef, d_coef, sizeof coef, D2H);
+  cudaMemcpy(ntok, d_ntok, sizeof ntok, D2H);
+  cudaMemcpy(&loss, d_loss, 8, D2H);
+  cudaMemcpy(&vloss, d_vloss, 8, D2H);
+  cudaMemcpy(dh, d_dh, (size_t)T * D * 4, D2H);
+  cudaMemcpy(dw, d_dw, (size_t)V * D * 4, D2H);
+  cudaMemcpy(gadv, d_gadv, sizeof gadv, D2H);
+  cudaMemcpy(ret, d_ret, sizeof ret, D2H);
+  cudaMemcpy(dv, d_dv, sizeof dv, D2H);
+
+  /* fused head */
+  double expect = 0.0, scale = 0.0;
+  for (int i = 0; i < N; ++i) {
+    expect -= (double)coef[i] * ntok[i] * adv[i];
+    scale += fabs((double)coef[i] * ntok[i] * adv[i]);
+  }
+  CHECK(fabs(loss - expect) <= 1e-5 * scale + 1e-12, "fused head loss %.9g, closed form %.9g", loss, expect);
+  int dw_nonzero = 0;
+  for (size_t k = 0; k < (size_t)V * D; ++k) dw_nonzero += dw[k] != 0.0f;
+  CHECK(dw_nonzero == 0, "dW must be exactly 0 with zero hidden states (%d nonzero)", dw_nonzero);
+  double wmean[D], wabs = 0.0;
+  for (int d = 0; d < D; ++d) {
+    double m = 0.0;
+    for (int v = 0; v < V; ++v) m += wf[v * D + d];
+    wmean[d] = m / V;
+  }
+  for (size_t k = 0; k < (size_t)V * D; ++k) wabs += fabs(wf[k]);
+  wabs /= (double)V * D;
+  for (int t = 0; t < T; ++t) {
+    const int i = t / LEN;
+    const double g = mask[t] ? -(double)coef[i] * adv[i] : 0.0;
+    for (int d = 0; d < D; ++d) {
+      const double ref = g * (wf[ids[t] * D + d] - wmean[d]);
+      /* dZ passes through two bf16 roundings (2^-8 each, relative) */
+      const double tol = fabs(g) * (fabs(wf[ids[t] * D + d]) + wabs) * (1.0 / 64.0) + 1e-12;
+      if (fabs(dh[t * D + d] - ref) > tol) {
+        fprintf(stderr, "FAIL: dH[%d][%d] = %.9g, closed form %.9g (tol %.3g)\n", t, d, dh[t * D + d], ref, tol);
+        ++fails;
+        t = T;
+        break;
+      }
+    }
+  }
+  /* GAE and value loss */
+  double vexpect = 0.0, vscale = 0.0;
+  for (int t = 0; t < T; ++t) {
+    const int i = t / LEN;
+    const double a_ref = mask[t] ? (double)rewards[i] - values[t] : 0.0;
+    const double g_ref = mask[t] ? (double)rewards[i] : 0.0;
+    if (fabs(gadv[t] - a_ref) > 1e-5 * (1.0 + fabs(a_ref)) || fabs(ret[t] - g_ref) > 1e-5 * (1.0 + fabs(g_ref))) {
+      fprintf(stderr, "FAIL: GAE at %d: A %.9g (closed form %.9g), G %.9g (closed form %.9g)\n", t, gadv[t], a_ref,
+              ret[t], g_ref);
+      ++fails;
+      break;
+    }
+    const double c = mask[t] ? coef[i] : 0.0, d = (double)values[t] - ret[t];
+    vexpect += c * d * d;
+    vscale += fabs(c * d * d);
+    if (fabs(dv[t] - 2.0 * c * d) > 1e-6 * (fabs(2.0 * c * d) + 1e-6)) {
+      fprintf(stderr, "FAIL: dV[%d] = %.9g, closed form %.9g\n", t, dv[t], 2.0 * c * d);
+      ++fails;
+      break;
+    }
+  }
+  CHECK(fabs(vloss - vexpect) <= 1e-6 * vscale + 1e-12, "value loss %.9g, closed form %.9g", vloss, vexpect);
+
+  free(dh);
+  free(dw);
+  free(w);
+  free(wf);
+  void* all[] = {d_go, d_rw, d_offs, d_mask, d_ids, d_old, d_adv, d_coef, d_ntok, d_tt, d_h, d_w, d_dh, d_dw,
+                 d_loss, d_ws, d_val, d_gadv, d_ret, d_dv, d_vloss};
+  for (size_t k = 0; k < sizeof all / sizeof all[0]; ++k) cudaFree(all[k]);
+  return fails;
+}
+
 int main(int argc, char** argv) {
   int f = host_checks();
-  if (argc > 1 && strcmp(argv[1], "gpu") == 0) f += gpu_checks();
+  if (argc > 1 && strcmp(argv[1], "gpu") == 0) f += gpu_checks() + gpu_checks_more();
   if (f == 0) printf("c_abi_check ok\n");
   return f == 0 ? 0 : 1;
 }
