@@ -1,5 +1,6 @@
 /* A plain C caller of the library (no Python, no torch): it includes only rl_loss.h and
- * links librl_loss.so. Argument "host" runs the host-side checks; argument "gpu" also runs
+ * links librl_loss.so. Argument "host" runs the host-side checks (argument checks and the host
+ * prefix-tree builder on a worked example); argument "gpu" also runs
  * the advantages and the policy loss on a small batch whose result has a closed form:
  * uniform logits (all 0) give logp = -ln V for every token; with old_logp = logp the ratio
  * is 1, nothing is clipped, and the loss is -sum_i c_i L_i A_i, which is 0 for complete
@@ -55,6 +56,48 @@ static int host_checks(void) {
                                lacc, NULL, fake, 100, NULL) == RL_ERR_WORKSPACE_TOO_SMALL,
         "small workspace");
   CHECK(strstr(rl_last_error_message(), "rl_policy_loss_fwd_bwd") != NULL, "error message");
+  return fails;
+}
+
+/* The host prefix-tree builder on a worked example: prompt [1 2 3]; call 0 answers [10 11];
+ * call 1 sees the tool output [20 21] after it and answers [30]; call 2 retries the first turn
+ * (input [1 2 3]) with [12]. Call 0 and the retry form one segment; its longest leaf (call 1)
+ * is kept, so the packed stream is [1 2 3 10 11 20 21 30] with mask 0 0 0 1 1 0 0 1, each token's
+ * parent the previous position, 2 leaves in the tree and 1 kept. */
+static int tree_checks(void) {
+  const int64_t po[2] = {0, 3};
+  const int32_t pt[3] = {1, 2, 3};
+  const int32_t co[2] = {0, 3};
+  const int64_t xo[4] = {0, 3, 10, 13};
+  const int32_t xt[13] = {1, 2, 3, 1, 2, 3, 10, 11, 20, 21, 1, 2, 3};
+  const int64_t yo[4] = {0, 2, 3, 4};
+  const int32_t yt[4] = {10, 11, 30, 12};
+  int64_t n = -1, ro[2], lo[2], parent[8], leaf_end[3];
+  int32_t tokens[8], depth[8], owner[8], node_call[8], leaf_call[3];
+  uint8_t mask[8];
+  rl_tree_stats st;
+  /* size query */
+  CHECK(rl_prefix_tree_build_batch(1, po, pt, co, xo, xt, yo, yt, NULL, 0, 1, 0, NULL, NULL, NULL, NULL, NULL, NULL,
+                                   NULL, NULL, NULL, NULL, NULL, &n) == RL_ERR_WORKSPACE_TOO_SMALL && n == 8,
+        "tree size query: n = %lld", (long long)n);
+  CHECK(rl_prefix_tree_build_batch(1, po, pt, co, xo, xt, yo, yt, NULL, 0, 1, 8, tokens, mask, parent, depth, owner,
+                                   node_call, leaf_call, leaf_end, lo, &st, ro, &n) == RL_OK,
+        "rl_prefix_tree_build_batch: %s", rl_last_error_message());
+  const int32_t want_tok[8] = {1, 2, 3, 10, 11, 20, 21, 30};
+  const uint8_t want_mask[8] = {0, 0, 0, 1, 1, 0, 0, 1};
+  const int32_t want_call[8] = {-1, -1, -1, 0, 0, 1, 1, 1};
+  for (int t = 0; t < 8; ++t) {
+    CHECK(tokens[t] == want_tok[t] && mask[t] == want_mask[t], "tree token %d: %d/%d", t, tokens[t], mask[t]);
+    CHECK(parent[t] == t - 1 && depth[t] == t && owner[t] == 0 && node_call[t] == want_call[t],
+          "tree links of token %d: parent %lld depth %d owner %d call %d", t, (long long)parent[t], depth[t],
+          owner[t], node_call[t]);
+  }
+  CHECK(st.valid == 1 && st.n_leaves == 2 && st.n_kept_leaves == 1 && st.n_unplaced == 0 && st.n_tokens == 8 &&
+            st.n_trainable == 3,
+        "tree stats: valid %d leaves %d kept %d unplaced %d tokens %lld trainable %lld", st.valid, st.n_leaves,
+        st.n_kept_leaves, st.n_unplaced, (long long)st.n_tokens, (long long)st.n_trainable);
+  CHECK(lo[0] == 0 && lo[1] == 1 && leaf_call[0] == 1 && leaf_end[0] == 7 && ro[0] == 0 && ro[1] == 8,
+        "tree leaves: call %d end %lld", leaf_call[0], (long long)leaf_end[0]);
   return fails;
 }
 
@@ -313,6 +356,7 @@ static int gpu_checks_more(void) {
 
 int main(int argc, char** argv) {
   int f = host_checks();
+  f += tree_checks();
   if (argc > 1 && strcmp(argv[1], "gpu") == 0) f += gpu_checks() + gpu_checks_more();
   if (f == 0) printf("c_abi_check ok\n");
   return f == 0 ? 0 : 1;
