@@ -650,4 +650,45 @@ def pin_fused_head_logprobs_vs_library(O):
     _close([logp[3], H[3]], [-math.log(40), math.log(40)], what="zero hidden row")
 
 
+def pin_gradients_autograd(O):
+    """The analytic d loss / d logits against autograd of a separate float64 PyTorch statement of
+    the objective (clipped surrogate with both branches present, k3 KL, entropy, TIS as a constant
+    weight, coefficient-weighted sum), to float64 rounding."""
+    import torch
+
+    rng = np.random.default_rng(41)
+    rows, V, n = 40, 29, 5
+    z = rng.normal(0.0, 2.0, (rows, V))
+    ids = rng.integers(0, V, rows)
+    zt = torch.tensor(z, requires_grad=True)
+    logp_all = torch.log_softmax(zt, dim=1)
+    logp0 = logp_all.detach().numpy()[np.arange(rows), ids]
+    delta = rng.uniform(-0.6, 0.6, rows)
+    delta = np.where(np.abs(delta - np.log(0.8)) < 2e-4, delta + 5e-4, delta)
+    delta = np.where(np.abs(delta - np.log(1.28)) < 2e-4, delta + 5e-4, delta)
+    old, ref = logp0 - delta, logp0 + rng.normal(0.0, 0.3, rows)
+    roll = old + rng.normal(0.0, 0.4, rows)
+    tt = rng.integers(0, n, rows)
+    mask = (rng.random(rows) < 0.8).astype(np.uint8)
+    adv, coef = rng.normal(0.0, 1.0, n), rng.uniform(0.05, 1.0, n)
+    prm = O.LossParams(kl_coef=0.05, kl_estimator=3, entropy_coef=0.03, tis_cap=1.5)
+    loss, grad, stats, _ = O.policy_loss_fwd_bwd(z, "f64", ids, mask, tt, adv, coef, old, prm, ref, roll)
+    if not 0 < stats[mask != 0, O.STAT_CLIPPED].sum() < (mask != 0).sum():
+        raise AssertionError("the case must hold clipped and unclipped tokens")
+    T = lambda x: torch.tensor(x, dtype=torch.float64)  # noqa: E731
+    logp = logp_all.gather(1, torch.tensor(ids)[:, None])[:, 0]
+    p = logp_all.exp()
+    H = -(p * logp_all).sum(dim=1)
+    A, c = T(adv)[torch.tensor(tt)], T(coef)[torch.tensor(tt)] * T(mask)
+    rho = torch.exp(logp - T(old))
+    surr = torch.minimum(rho * A, torch.clamp(rho, 0.8, 1.28) * A)
+    w = torch.clamp(torch.exp(T(old) - T(roll)), max=1.5)
+    d = T(ref) - logp
+    ell = -w * surr + 0.05 * (torch.exp(d) - d - 1.0) - 0.03 * H
+    (c * ell).sum().backward()
+    g = zt.grad.numpy()
+    _close([loss], [float((c * ell).sum().detach())], rtol=1e-12, atol=1e-12, what="loss vs autograd")
+    _close(grad, g, rtol=0.0, atol=1e-11 * float(np.abs(g).max()), what="gradient vs autograd")
+
+
 ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_")]
