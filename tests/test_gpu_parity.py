@@ -186,6 +186,19 @@ def test_policy_loss_ragged_shapes(R, vocab, ld_pad, dtype_case):
     compare(case, out, f"V={vocab} ld=V+{ld_pad}")
 
 
+@pytest.mark.parametrize("name,row0,rows", [("tiny", 0, 1), ("multiturn", 100, 1), ("edge", 3, 2), ("multiturn", 0, 3)])
+def test_policy_loss_fewest_rows(R, name, row0, rows):
+    """One to three rows: a single cluster (or as many as rows), whose last one sums the loss."""
+    case = make_case(name, seed=12, row0=row0, rows=rows, loss_agg=2)
+    out = run_loss(R, case)
+    compare(case, out, f"{name}[{row0}:+{rows}]")
+    lp, H, lse = R.rl_token_logprobs(logits_to_dev(case), to_dev(case.ids), R.new_workspace(rows, case.raw.shape[1]),
+                                     want_entropy=True, want_lse=True)
+    lp_ref, H_ref, _ = O.token_logprobs(case.raw, case.w.dtype, case.ids)
+    assert np.all(np.abs(lp.cpu().numpy() - lp_ref) <= 1e-5 + 2.0 ** -22 * np.abs(lp_ref))
+    assert np.all(np.abs(H.cpu().numpy() - H_ref) <= 5e-5 + 2e-5 * np.abs(H_ref))
+
+
 def test_policy_loss_in_place_and_deterministic(R):
     case = make_case("multiturn", seed=5, row0=300, rows=64, loss_agg=2)
     a = run_loss(R, case)
