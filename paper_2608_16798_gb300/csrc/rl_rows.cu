@@ -768,12 +768,15 @@ __global__ void __launch_bounds__((NW + 1) * 32, 2) rows_kernel(const RowArgs p)
 // shared-memory stages (bulk copies, full / empty mbarriers); consumer warps fold
 // each chunk into per-thread online-softmax partials and, at the end of a row,
 // merge them (one named barrier among the consumers per row).
-#ifndef RL_FWD_STAGES
-#define RL_FWD_STAGES 6
-#endif
-#ifndef RL_FWD_CHUNK_KB
-#define RL_FWD_CHUNK_KB 16
-#endif
+// Stages and chunk size per form, chosen by a sweep on the benchmark batch (bf16, V = 151,936):
+// without the entropy 3 x 16 KB (3 CTAs per SM, bound by registers) ran in 6.54 ms per batch
+// against 6.80 with 6 x 16 KB (2 CTAs per SM, bound by shared memory); with the entropy
+// 4 x 12 KB ran in 7.19 against 7.27 ms (3 x 16 KB: 7.55).
+template <bool ENT>
+struct FwdCfg {
+  static constexpr int kStages = ENT ? 4 : 3;
+  static constexpr int kChunkKB = ENT ? 12 : 16;
+};
 
 struct StreamArgs {
   const void* logits;
@@ -797,7 +800,7 @@ struct ChunkInfo {
 template <typename T, int NW, bool ENT>
 __global__ void __launch_bounds__((NW + 1) * 32, 2) stream_logprobs_kernel(const StreamArgs p) {
   constexpr int EPV = Vec<T>::N;
-  constexpr int NS = RL_FWD_STAGES;
+  constexpr int NS = FwdCfg<ENT>::kStages;
   constexpr int NC = NW * 32;
   extern __shared__ __align__(128) unsigned char smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[NS], empty_bar[NS];
@@ -876,7 +879,7 @@ __global__ void __launch_bounds__((NW + 1) * 32, 2) stream_logprobs_kernel(const
       const T* buf = buf_base + st * p.buf_elems;
       const int cv = ci.count / EPV;
       {
-        constexpr int KV = (RL_FWD_CHUNK_KB * 1024 / 16 + NC - 1) / NC;  // vectors per thread per chunk
+        constexpr int KV = (FwdCfg<ENT>::kChunkKB * 1024 / 16 + NC - 1) / NC;  // vectors per thread per chunk
         uint4 x[KV];
         const uint32_t pad = Vec<T>::kPadWord;
         auto reload = [&](int k) {
@@ -1045,9 +1048,11 @@ static rl_status dispatch_loss(bool ent, const RowArgs& args, const Plan& plan, 
 constexpr int kFwdWarps = 8;
 
 template <typename T, bool ENT>
-static rl_status launch_stream(const StreamArgs& args, cudaStream_t s) {
+static rl_status launch_stream(StreamArgs args, cudaStream_t s) {
   auto kern = stream_logprobs_kernel<T, kFwdWarps, ENT>;
-  const size_t smem = static_cast<size_t>(RL_FWD_STAGES) * args.buf_elems * sizeof(T);
+  args.chunk = static_cast<int64_t>(FwdCfg<ENT>::kChunkKB) * 1024 / static_cast<int64_t>(sizeof(T));
+  args.buf_elems = args.chunk;  // chunk bytes are a multiple of 128
+  const size_t smem = static_cast<size_t>(FwdCfg<ENT>::kStages) * args.buf_elems * sizeof(T);
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return cuda_error(e, "cudaGetDevice");
@@ -1121,9 +1126,7 @@ extern "C" rl_status rl_token_logprobs(const void* logits, rl_dtype dtype, int64
   a.entropy_out = entropy_out;
   a.lse_out = lse_out;
   a.status = reinterpret_cast<int32_t*>(ws);
-  a.chunk = static_cast<int64_t>(RL_FWD_CHUNK_KB) * 1024 / es;
-  a.buf_elems = a.chunk;  // chunk bytes are a multiple of 128
-  a.tma = ((ld * es) % 16) == 0;
+  a.tma = ((ld * es) % 16) == 0;  // chunk and buf_elems are set per form by launch_stream
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (dtype == RL_BF16)
     return entropy_out ? launch_stream<uint16_t, true>(a, s) : launch_stream<uint16_t, false>(a, s);
