@@ -189,7 +189,10 @@ __device__ __forceinline__ void raise_max(SoftmaxPartial& ps, float vm) {
 #endif
 
 constexpr int kMaxCluster = 16;
-constexpr int kZeroBytes = 2048;  // zero-filled shared region, source of the masked rows' bulk stores
+#ifndef RL_ZERO_BYTES
+#define RL_ZERO_BYTES 8192
+#endif
+constexpr int kZeroBytes = RL_ZERO_BYTES;  // zero-filled shared region, source of the masked rows' bulk stores
 
 // Per-row inputs, staged in shared memory by the producer warp.
 struct RowMeta {
