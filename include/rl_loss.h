@@ -113,10 +113,21 @@ const char* rl_last_error_message(void);
 /* Workspace bytes needed by calls on at most `max_rows` logits rows of
  * vocabulary V (D = hidden size of the fused head, 0 if unused). The
  * workspace holds the device status word and per-row loss contributions; with
- * D > 0 it also holds the fused head's buffers (about
- * min(max_rows, 32768) * V * 2 bytes plus 32 MiB: the bf16 dZ of up to
- * 32,768 tokens). */
+ * D > 0 it also holds the fused head's buffers, the largest being the bf16
+ * gradient of the logits of ONE chunk of min(max_rows, 4096) tokens
+ * (min(max_rows, 4096) * ceil(V / 8) * 8 * 2 bytes: 1.24 GB at V = 151,936),
+ * plus min(max_rows, 4096) * D * 4 bytes of fp32 d_hidden. This is the
+ * smallest workspace of rl_fused_head_loss_fwd_bwd. */
 size_t rl_workspace_size(int64_t max_rows, int64_t V, int64_t D);
+
+/* Workspace bytes with which rl_fused_head_loss_fwd_bwd on up to T tokens keeps the
+ * bf16 logits gradient of up to group_tokens tokens at once (rounded up to whole
+ * chunks of 4,096 tokens; group_tokens <= 4096 gives rl_workspace_size(T, V, D)).
+ * The fused head then runs its dH and dW products once per group instead of once
+ * per chunk, which reads and writes the fp32 d_weight fewer times, at the cost of
+ * ceil(V / 8) * 8 * 2 bytes per token of the group. Any workspace size between the
+ * two works: the group is as many whole chunks as the workspace holds. */
+size_t rl_fused_head_workspace_size(int64_t T, int64_t V, int64_t D, int64_t group_tokens);
 
 /* Zero the workspace's 256-byte header: the status word and the finished-block
  * counters of the policy and value losses (which each launch leaves at zero
@@ -265,14 +276,16 @@ rl_status rl_policy_loss_fwd_bwd(const void* logits, rl_dtype dtype, int64_t row
  *                 (overwritten; zero rows for tokens that are not trained on)
  *   d_weight      float [V x D]: d loss / d W is ADDED to it
  *   ws, ws_bytes  workspace of at least rl_workspace_size(T, V, D) bytes; it holds,
- *                 among others, the gradient of the logits (bf16) for a group of up
- *                 to 32,768 tokens, consumed by the dH and dW products
+ *                 among others, the gradient of the logits (bf16) of one chunk of
+ *                 4,096 tokens, or of a group of several chunks when ws_bytes allows
+ *                 (rl_fused_head_workspace_size), consumed by the dH and dW products
  * Tokens are processed in chunks of 4,096: per chunk, one tensor-core pass forms the
  * logits tile by tile, folds them into softmax partials and keeps exp(z - tile max)
  * in bf16 with the tile maxima; a per-token merge evaluates the objective; an in-place
  * rescale turns the kept values into the logits' gradient. After the last chunk of
- * each group of up to 32,768 tokens, two GEMMs (cuBLASLt) give the group's dH and add
- * its dW.
+ * each group (each chunk, with the smallest workspace), two tensor-core products give
+ * the group's dH and add its dW (fp32, one addition per element and group, in chunk
+ * order: deterministic). The logits of all T tokens are never held at once.
  */
 rl_status rl_fused_head_loss_fwd_bwd(const void* hidden, const void* weight, int64_t T, int64_t D, int64_t V,
                                      const int32_t* token_ids, const uint8_t* mask, const int32_t* token_traj,

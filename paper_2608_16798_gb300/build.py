@@ -73,7 +73,7 @@ def build(verbose: bool = False, force: bool = False, extra_flags=()) -> str:
         objs = list(ex.map(compile_one, sources()))
     tmp = LIB + ".tmp"
     cuda_lib = os.path.join(os.path.dirname(os.path.dirname(os.path.realpath(cc))), "lib64")
-    cmd = [cc, *ARCH, "-shared", "-o", tmp, *objs, "-cudart", "static", "-L", cuda_lib, "-lcublasLt",
+    cmd = [cc, *ARCH, "-shared", "-o", tmp, *objs, "-cudart", "static", "-L", cuda_lib,
            "-lpthread", "-Xlinker", f"-rpath={cuda_lib}"]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:

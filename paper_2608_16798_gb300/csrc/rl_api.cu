@@ -58,6 +58,12 @@ size_t rl_workspace_size(int64_t max_rows, int64_t V, int64_t D) {
   return rl::kWsHeader + rows_bytes;
 }
 
+size_t rl_fused_head_workspace_size(int64_t T, int64_t V, int64_t D, int64_t group_tokens) {
+  if (T < 0) T = 0;
+  if (V < 1 || D < 1) return rl_workspace_size(T, V, D);
+  return rl::head_workspace_bytes_grouped(T, V, D, group_tokens);
+}
+
 rl_status rl_workspace_init(void* ws, size_t ws_bytes, rl_stream_t stream) {
   rl::clear_error();
   if (!ws) return rl::set_error(RL_ERR_INVALID_ARG, "rl_workspace_init: ws is NULL");

@@ -15,15 +15,16 @@
 //   3. head_dz_kernel       rescales the stored e in place into
 //      dZ = c [g (delta_a - p) + alpha p (log p + H)], p = e exp(m_j - lse) (HBM-bound: the
 //      logits are formed once, not twice).
-// The chunks of a group (up to 32,768 tokens) keep their dZ side by side in the workspace;
-// after the group's last chunk:
-//   4. dH = dZ W and dW += dZ^T H over the whole group, two plain GEMMs through cuBLASLt: the
-//      fp32 dW (V x D x 4 bytes) is read and written once per group rather than once per
-//      chunk, and the dH product has eight times the output tiles of a chunk's.
+// The dZ of one chunk (4,096 tokens x V in bf16) is the only logits-sized buffer; a caller
+// that passes more workspace lets a group of several chunks keep their dZ side by side.
+// After the group's last chunk (every chunk, with the smallest workspace):
+//   4. dH = dZ W and dW += dZ^T H over the group: head_grad_kernel (rl_head_grad.cu), the
+//      same CTA-pair tcgen05 machinery with the operands in their row-major layouts (dZ
+//      K-major for dH, MN-major for dW; W and H MN-major); dW is added in fp32 by TMA
+//      reduce-add, once per group.
 // The forward-only call runs head_kernel<STATS> (no stores) and head_logp_merge_kernel.
 // The objective (Sec. 2.3.2, Sec. 3.2.4) is the same as for rl_policy_loss_fwd_bwd; here
 // pi_theta's logits come from the hidden states times the vocabulary projection.
-#include <cublasLt.h>
 #include <cuda.h>
 
 #include <algorithm>
@@ -34,6 +35,7 @@
 #include "rl_device.cuh"
 #include "rl_host.h"
 #include "rl_tc.cuh"
+#include "rl_tmap.h"
 
 namespace rl {
 namespace head {
@@ -65,12 +67,6 @@ constexpr uint32_t kWBoxRows = kPair ? BN / 2 : BN;  // rows of W per TMA box
 #define RL_HEAD_CHUNK 4096
 #endif
 constexpr int64_t kChunk = RL_HEAD_CHUNK;  // tokens per chunk (tuning knob, compile time)
-#ifndef RL_HEAD_GROUP
-#define RL_HEAD_GROUP 32768
-#endif
-// tokens whose dZ the workspace holds at once: dW += dZ^T H runs once per group (tuning knob)
-constexpr int64_t kGroup = RL_HEAD_GROUP;
-constexpr size_t kLtWorkspace = 32u << 20;
 
 enum Mode { STATS = 0, STATS_P = 1 };
 
@@ -530,54 +526,26 @@ __global__ void __launch_bounds__(256) head_logp_merge_kernel(const LogpMergeArg
 
 // ------------------------------------------------------------------ host side
 
-typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
-                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
-                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-static rl_status encoder(EncodeTiledFn* out) {
-  static std::mutex mu;
-  static EncodeTiledFn fn = nullptr;
-  std::lock_guard<std::mutex> lock(mu);
-  if (!fn) {
-    cudaDriverEntryPointQueryResult q;
-    void* f = nullptr;
-    cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q);
-    if (e != cudaSuccess || !f || q != cudaDriverEntryPointSuccess)
-      return set_error(RL_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
-    fn = reinterpret_cast<EncodeTiledFn>(f);
-  }
-  *out = fn;
-  return RL_OK;
-}
-
 // bf16 matrix [rows x inner] (row stride inner), tiles of box_rows x 64 with the 128-byte swizzle.
 static rl_status make_map(CUtensorMap* m, const void* base, int64_t inner, int64_t rows, uint32_t box_rows) {
-  EncodeTiledFn enc = nullptr;
-  rl_status st = encoder(&enc);
-  if (st != RL_OK) return st;
-  cuuint64_t dims[2] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(rows)};
-  cuuint64_t strides[1] = {static_cast<cuuint64_t>(inner) * 2};
-  cuuint32_t box[2] = {64, box_rows};
-  cuuint32_t es[2] = {1, 1};
-  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
-                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  if (r != CUDA_SUCCESS) return set_error(RL_ERR_CUDA, "cuTensorMapEncodeTiled failed");
-  return RL_OK;
+  return tmap_2d(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, base, inner, rows, inner * 2, 64, box_rows,
+                 CU_TENSOR_MAP_SWIZZLE_128B);
 }
 
 struct Layout {
   int64_t Tc, G, n_nt, n_vb, ldz;  // G chunks per group
-  size_t off_partials, off_rc, off_tmax, off_dz, off_lt, total;
+  size_t off_partials, off_rc, off_tmax, off_dh32, off_dz, total;
 };
 
 static size_t al256(size_t x) { return (x + 255) & ~size_t(255); }
 
-static Layout layout(int64_t max_rows, int64_t V) {
+// Workspace of the loss call for up to max_rows tokens. Its smallest form (ws_bytes = 0)
+// keeps the dZ of one chunk; every further Tc x ldz x 2 bytes the caller passes keep one more
+// chunk's dZ, so that the two products run once per group of G chunks.
+static Layout layout(int64_t max_rows, int64_t V, int64_t D, size_t ws_bytes = 0, int64_t want_G = 0) {
   Layout L;
   L.Tc = std::max<int64_t>(1, std::min<int64_t>(max_rows, kChunk));
   const int64_t chunks = (std::max<int64_t>(max_rows, 1) + L.Tc - 1) / L.Tc;
-  L.G = std::max<int64_t>(1, std::min<int64_t>(chunks, kGroup / L.Tc));
   const int64_t n_nt = (V + BN - 1) / BN;
   L.n_nt = n_nt;
   L.n_vb = (n_nt + VB_TILES - 1) / VB_TILES;
@@ -590,62 +558,26 @@ static Layout layout(int64_t max_rows, int64_t V) {
   off += al(static_cast<size_t>(L.Tc) * sizeof(RowCoef));
   L.off_tmax = off;
   off += al(static_cast<size_t>(L.Tc * n_nt) * sizeof(float));
+  L.off_dh32 = off;  // fp32 dH of one chunk: the two halves of a split contraction add here
+  off += al(static_cast<size_t>(L.Tc * std::max<int64_t>(D, 0)) * sizeof(float));
   L.off_dz = off;
-  off += al(static_cast<size_t>(L.G * L.Tc * L.ldz) * 2);
-  L.off_lt = off;
-  off += kLtWorkspace;
+  const size_t chunk_dz = static_cast<size_t>(L.Tc * L.ldz) * 2;
+  int64_t G = std::max<int64_t>(want_G, 1);
+  if (ws_bytes > off + chunk_dz) G = static_cast<int64_t>((ws_bytes - off) / chunk_dz);
+  L.G = std::max<int64_t>(1, std::min<int64_t>(G, chunks));
+  off += al(static_cast<size_t>(L.G) * chunk_dz);
   L.total = off;
   return L;
 }
 
-// C (col-major m x n) = op(A) op(B) + beta C with bf16 A, B and fp32 accumulation.
-static rl_status lt_matmul(cublasLtHandle_t lt, bool ta, bool tb, int64_t m, int64_t n, int64_t k, const void* A,
-                           int64_t lda, const void* B, int64_t ldb, void* C, int64_t ldc, cudaDataType_t ctype,
-                           float beta, void* ws, size_t ws_bytes, cudaStream_t s) {
-  cublasLtMatmulDesc_t op = nullptr;
-  cublasLtMatrixLayout_t la = nullptr, lb = nullptr, lc = nullptr;
-  cublasLtMatmulPreference_t pref = nullptr;
-  rl_status st = RL_OK;
-  const float alpha = 1.f;
-  cublasOperation_t opa = ta ? CUBLAS_OP_T : CUBLAS_OP_N, opb = tb ? CUBLAS_OP_T : CUBLAS_OP_N;
-  cublasLtMatmulHeuristicResult_t heur = {};
-  int found = 0;
-  auto fail = [&](const char* what) { st = set_error(RL_ERR_CUDA, std::string("cuBLASLt: ") + what); };
-  if (cublasLtMatmulDescCreate(&op, CUBLAS_COMPUTE_32F, CUDA_R_32F) != CUBLAS_STATUS_SUCCESS) { fail("desc"); goto done; }
-  cublasLtMatmulDescSetAttribute(op, CUBLASLT_MATMUL_DESC_TRANSA, &opa, sizeof(opa));
-  cublasLtMatmulDescSetAttribute(op, CUBLASLT_MATMUL_DESC_TRANSB, &opb, sizeof(opb));
-  if (cublasLtMatrixLayoutCreate(&la, CUDA_R_16BF, ta ? k : m, ta ? m : k, lda) != CUBLAS_STATUS_SUCCESS ||
-      cublasLtMatrixLayoutCreate(&lb, CUDA_R_16BF, tb ? n : k, tb ? k : n, ldb) != CUBLAS_STATUS_SUCCESS ||
-      cublasLtMatrixLayoutCreate(&lc, ctype, m, n, ldc) != CUBLAS_STATUS_SUCCESS) {
-    fail("layout");
-    goto done;
+// dH rows in fp32 -> bf16 (round to nearest even), 8 elements per thread and step.
+__global__ void __launch_bounds__(256) f32_to_bf16_kernel(const float4* __restrict__ src, uint4* __restrict__ dst,
+                                                          int64_t n8) {
+  for (int64_t k = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; k < n8;
+       k += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const float4 a = src[2 * k], b = src[2 * k + 1];
+    dst[k] = make_uint4(pack_bf16x2(a.x, a.y), pack_bf16x2(a.z, a.w), pack_bf16x2(b.x, b.y), pack_bf16x2(b.z, b.w));
   }
-  if (cublasLtMatmulPreferenceCreate(&pref) != CUBLAS_STATUS_SUCCESS) { fail("preference"); goto done; }
-  cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MAX_WORKSPACE_BYTES, &ws_bytes, sizeof(ws_bytes));
-  if (cublasLtMatmulAlgoGetHeuristic(lt, op, la, lb, lc, lc, pref, 1, &heur, &found) != CUBLAS_STATUS_SUCCESS ||
-      found == 0) {
-    fail("no algorithm");
-    goto done;
-  }
-  if (cublasLtMatmul(lt, op, &alpha, A, la, B, lb, &beta, C, lc, C, lc, &heur.algo, ws, ws_bytes, s) !=
-      CUBLAS_STATUS_SUCCESS)
-    fail("matmul");
-done:
-  if (pref) cublasLtMatmulPreferenceDestroy(pref);
-  if (lc) cublasLtMatrixLayoutDestroy(lc);
-  if (lb) cublasLtMatrixLayoutDestroy(lb);
-  if (la) cublasLtMatrixLayoutDestroy(la);
-  if (op) cublasLtMatmulDescDestroy(op);
-  return st;
-}
-
-static rl_status lt_handle(cublasLtHandle_t* out) {
-  static std::mutex mu;
-  static cublasLtHandle_t h = nullptr;
-  std::lock_guard<std::mutex> lock(mu);
-  if (!h && cublasLtCreate(&h) != CUBLAS_STATUS_SUCCESS) return set_error(RL_ERR_CUDA, "cublasLtCreate failed");
-  *out = h;
-  return RL_OK;
 }
 
 template <int MODE>
@@ -707,8 +639,12 @@ static rl_status launch_head(const CUtensorMap& mh, const CUtensorMap& mw, const
 }  // namespace head
 
 size_t head_workspace_bytes(int64_t max_rows, int64_t V, int64_t D) {
-  (void)D;
-  return head::layout(max_rows, V).total;
+  return head::layout(max_rows, V, D).total;
+}
+
+size_t head_workspace_bytes_grouped(int64_t max_rows, int64_t V, int64_t D, int64_t group_tokens) {
+  const int64_t g = (std::max<int64_t>(group_tokens, 1) + head::kChunk - 1) / head::kChunk;
+  return head::layout(max_rows, V, D, 0, g).total;
 }
 
 // The forward-only call needs the status word and one chunk's partials, which sit at the
@@ -719,7 +655,7 @@ size_t head_workspace_bytes(int64_t max_rows, int64_t V, int64_t D) {
 // 3,072 and 6,144 are within 2%, 8,192 takes 26.7 ms (73.1), and 32,768 takes 31.5 ms: the
 // hidden states (256 MB) then evict W's tiles from the 129 MB L2.
 static size_t head_logp_workspace_bytes(int64_t T, int64_t V) {
-  const head::Layout L = head::layout(T, V);
+  const head::Layout L = head::layout(T, V, 0);
   return kWsHeader + head::al256(static_cast<size_t>(L.n_vb * L.Tc) * sizeof(float4));
 }
 
@@ -758,18 +694,16 @@ extern "C" rl_status rl_fused_head_loss_fwd_bwd(
                      "rl_fused_head_loss_fwd_bwd: hidden, weight, d_hidden, d_weight and ws must be 16-byte aligned");
 
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  const Layout L = layout(T, V);
+  const Layout L = layout(T, V, D, ws_bytes);
   char* wsb = static_cast<char*>(ws);
   int32_t* status = reinterpret_cast<int32_t*>(wsb);
   double* row_loss = reinterpret_cast<double*>(wsb + ws_row_loss_offset());
   float4* partials = reinterpret_cast<float4*>(wsb + L.off_partials);
   RowCoef* rcs = reinterpret_cast<RowCoef*>(wsb + L.off_rc);
   float* tmax = reinterpret_cast<float*>(wsb + L.off_tmax);
+  float* dh32 = reinterpret_cast<float*>(wsb + L.off_dh32);
   uint16_t* dz_base = reinterpret_cast<uint16_t*>(wsb + L.off_dz);
-  void* lt_ws = wsb + L.off_lt;
-  cublasLtHandle_t lt = nullptr;
-  rl_status st = lt_handle(&lt);
-  if (st != RL_OK) return st;
+  rl_status st = RL_OK;
   const bool kl_on = params->kl_estimator == 3 && params->kl_coef != 0.f && ref_logp != nullptr;
   const bool ent = params->entropy_coef != 0.f || token_stats != nullptr;
 
@@ -849,14 +783,31 @@ extern "C" rl_status rl_fused_head_loss_fwd_bwd(
     // after the group's last chunk, the two products over the group's n = g1 - g0 tokens
     const int64_t g1 = std::min<int64_t>(g0 + group_rows, T);
     if (t0 + Tc == g1) {
-      // dH[g0 : g1] = dZ W    (column-major: dH^T [D x n] = W^T [D x V] dZ^T [V x n])
-      void* dh = static_cast<char*>(d_hidden) + g0 * D * (d_hidden_dtype == RL_BF16 ? 2 : 4);
-      st = lt_matmul(lt, false, false, D, g1 - g0, V, weight, D, dz_base, L.ldz, dh, D,
-                     d_hidden_dtype == RL_BF16 ? CUDA_R_16BF : CUDA_R_32F, 0.f, lt_ws, kLtWorkspace, s);
-      if (st != RL_OK) return st;
-      // dW += dZ^T H  (column-major: dW^T [D x V] += H^T [D x n] (dZ^T)^T [n x V])
-      st = lt_matmul(lt, false, true, D, V, g1 - g0, static_cast<const uint16_t*>(hidden) + g0 * D, D, dz_base,
-                     L.ldz, d_weight, D, CUDA_R_32F, 1.f, lt_ws, kLtWorkspace, s);
+      const int64_t n = g1 - g0;
+      const bool bf16_out = d_hidden_dtype == RL_BF16;
+      void* dh = static_cast<char*>(d_hidden) + g0 * D * (bf16_out ? 2 : 4);
+      // dH[g0 : g1] = dZ W; a split contraction adds its two halves onto zeros in fp32 (the
+      // caller's fp32 rows, or the workspace's one-chunk buffer before rounding to bf16)
+      const int split = (bf16_out && n > L.Tc) ? 1 : head_grad_dh_split(n, V, D);
+      if (split == 2) {
+        float* acc = bf16_out ? dh32 : static_cast<float*>(dh);
+        e = cudaMemsetAsync(acc, 0, static_cast<size_t>(n * D) * sizeof(float), s);
+        if (e != cudaSuccess) return cuda_error(e, "cudaMemsetAsync(d_hidden)");
+        st = head_grad_dh(dz_base, L.ldz, n, V, weight, D, acc, 0, 2, status, s);
+        if (st != RL_OK) return st;
+        if (bf16_out) {
+          const int64_t n8 = n * D / 8;
+          f32_to_bf16_kernel<<<static_cast<int>(std::min<int64_t>((n8 + 255) / 256, 148 * 8)), 256, 0, s>>>(
+              reinterpret_cast<const float4*>(dh32), static_cast<uint4*>(dh), n8);
+          e = cudaGetLastError();
+          if (e != cudaSuccess) return cuda_error(e, "f32_to_bf16_kernel launch");
+        }
+      } else {
+        st = head_grad_dh(dz_base, L.ldz, n, V, weight, D, dh, bf16_out ? 2 : 1, 1, status, s);
+        if (st != RL_OK) return st;
+      }
+      // dW += dZ^T H[g0 : g1]
+      st = head_grad_dw(dz_base, L.ldz, n, V, static_cast<const uint16_t*>(hidden) + g0 * D, D, d_weight, status, s);
       if (st != RL_OK) return st;
     }
   }
@@ -885,7 +836,7 @@ extern "C" rl_status rl_fused_head_token_logprobs(const void* hidden, const void
     return set_error(RL_ERR_ALIGNMENT, "rl_fused_head_token_logprobs: hidden, weight and ws must be 16-byte aligned");
 
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  const Layout L = layout(T, V);
+  const Layout L = layout(T, V, 0);
   char* wsb = static_cast<char*>(ws);
   int32_t* status = reinterpret_cast<int32_t*>(wsb);
   float4* partials = reinterpret_cast<float4*>(wsb + kWsHeader);

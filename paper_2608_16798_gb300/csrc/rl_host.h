@@ -31,8 +31,23 @@ void clear_error();
 
 // Fixed-order sum of `rows` loss contributions into *loss_accum (rl_stats.cu).
 rl_status launch_reduce_loss(const double* row_loss, int64_t rows, double* loss_accum, cudaStream_t s);
-// Workspace of the fused LM head for up to max_rows tokens (rl_head.cu).
+// Smallest workspace of the fused LM head for up to max_rows tokens (rl_head.cu).
 size_t head_workspace_bytes(int64_t max_rows, int64_t V, int64_t D);
+// The same, keeping the dZ of up to group_tokens tokens (whole chunks) at once.
+size_t head_workspace_bytes_grouped(int64_t max_rows, int64_t V, int64_t D, int64_t group_tokens);
+
+// Backward products of the fused LM head on the tensor cores (rl_head_grad.cu). dz is the
+// bf16 gradient of the logits of n tokens ([n x V], rows ldz elements apart).
+// out_kind: 0 = add into fp32 (TMA reduce-add), 1 = store fp32, 2 = store bf16.
+// dH[n x D] = dZ W; with ksplit = 2 the contraction over V is cut in two halves that are
+// both added (out_kind 0) into a zeroed fp32 destination.
+rl_status head_grad_dh(const uint16_t* dz, int64_t ldz, int64_t n, int64_t V, const void* weight, int64_t D,
+                       void* out, int out_kind, int ksplit, int32_t* status, cudaStream_t s);
+// dW[V x D] += dZ^T H[n x D] (fp32, one addition per element).
+rl_status head_grad_dw(const uint16_t* dz, int64_t ldz, int64_t n, int64_t V, const void* hidden, int64_t D,
+                       float* d_weight, int32_t* status, cudaStream_t s);
+// 2 if splitting dH's contraction in two balances the CTA pairs' work better, else 1.
+int head_grad_dh_split(int64_t n, int64_t V, int64_t D);
 
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 

@@ -34,6 +34,7 @@ EXPORTS = {
     "rl_last_error_message": (ctypes.c_char_p, []),
     "rl_workspace_size": (_SZ, [_I64, _I64, _I64]),
     "rl_workspace_init": (_I32, [_P, _SZ, _P]),
+    "rl_fused_head_workspace_size": (_SZ, [_I64, _I64, _I64, _I64]),
     "rl_query_status": (_I32, [_P, _P, ctypes.POINTER(_I32)]),
     "rl_selftest_bounded_wait": (_I32, [_P, _SZ, _I64, _P, _P]),
     "rl_group_advantages": (_I32, [_I32, _I32, _P, _P, _P, _I64, _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P]),
@@ -162,6 +163,10 @@ def rl_workspace_size(max_rows: int, V: int, D: int = 0) -> int:
     return int(lib().rl_workspace_size(max_rows, V, D))
 
 
+def rl_fused_head_workspace_size(T: int, V: int, D: int, group_tokens: int) -> int:
+    return int(lib().rl_fused_head_workspace_size(T, V, D, group_tokens))
+
+
 def rl_workspace_init(ws: torch.Tensor, stream=None):
     _need(ws, "ws", torch.uint8)
     _check("rl_workspace_init", lib().rl_workspace_init(_ptr(ws), ws.numel(), _stream(stream)))
@@ -176,9 +181,12 @@ def rl_selftest_bounded_wait(ws: torch.Tensor, limit_ns: int, waited_ns: torch.T
            lib().rl_selftest_bounded_wait(_ptr(ws), ws.numel(), int(limit_ns), _ptr(waited_ns), _stream(stream)))
 
 
-def new_workspace(max_rows: int, V: int, D: int = 0, device=None, stream=None) -> torch.Tensor:
-    """Allocate (with torch) and initialise a workspace for calls of up to max_rows rows."""
-    ws = torch.empty(rl_workspace_size(max_rows, V, D), dtype=torch.uint8, device=device or "cuda")
+def new_workspace(max_rows: int, V: int, D: int = 0, device=None, stream=None, group_tokens: int = 0) -> torch.Tensor:
+    """Allocate (with torch) and initialise a workspace for calls of up to max_rows rows
+    (with group_tokens > 0: the fused head's grouped workspace, rl_fused_head_workspace_size)."""
+    nbytes = rl_fused_head_workspace_size(max_rows, V, D, group_tokens) if group_tokens > 0 and D > 0 \
+        else rl_workspace_size(max_rows, V, D)
+    ws = torch.empty(nbytes, dtype=torch.uint8, device=device or "cuda")
     rl_workspace_init(ws, stream)
     return ws
 

@@ -55,6 +55,25 @@ def test_version_and_workspace_size(R):
     assert R.rl_workspace_size(3, 10) == 256 + 256
 
 
+def test_fused_head_workspace_is_one_chunk_of_logits_gradient(R):
+    """The smallest fused-head workspace holds the bf16 logits gradient of one 4,096-token
+    chunk, not of all T tokens: at 32,768 x 151,936 x 4,096 it stays near 1.24 GB (plus the
+    per-token and per-tile buffers) while the logits of all tokens would take 9.96 GB. Each
+    further chunk of a grouped workspace costs exactly one chunk's bf16 gradient."""
+    T, V, D = 32768, 151936, 4096
+    chunk_dz = 4096 * V * 2  # V is a multiple of 8
+    minimum = R.rl_workspace_size(T, V, D)
+    assert chunk_dz <= minimum < chunk_dz + 200 * 2**20
+    assert minimum < T * V * 2 / 7
+    assert R.rl_fused_head_workspace_size(T, V, D, 0) == minimum
+    assert R.rl_fused_head_workspace_size(T, V, D, 4096) == minimum
+    assert R.rl_fused_head_workspace_size(T, V, D, 4097) == minimum + chunk_dz
+    assert R.rl_fused_head_workspace_size(T, V, D, T) == minimum + 7 * chunk_dz
+    # a group never exceeds the call's chunks
+    assert R.rl_fused_head_workspace_size(T, V, D, 10 * T) == minimum + 7 * chunk_dz
+    assert R.rl_fused_head_workspace_size(100, 1000, 64, 10**6) == R.rl_workspace_size(100, 1000, 64)
+
+
 FAKE = 0x10000  # never dereferenced: every call below fails validation first
 PARAMS = None
 

@@ -69,9 +69,9 @@ def make_head_case(T, D, V, seed=0, masked=0.3, agg=0, ent=False, tis=False, wst
                 coef32=coef.astype(np.float32), old=old, ref=ref, roll=roll, P=P, T=T, D=D, V=V)
 
 
-def run_head(R, c, dh_dtype=torch.float32):
+def run_head(R, c, dh_dtype=torch.float32, group_tokens=0):
     T, D, V = c["T"], c["D"], c["V"]
-    ws = R.new_workspace(T, V, D)
+    ws = R.new_workspace(T, V, D, group_tokens=group_tokens)
     loss = torch.zeros(1, dtype=torch.float64, device="cuda")
     dW = torch.zeros((V, D), dtype=torch.float32, device="cuda")
     st = torch.zeros(T * 5, dtype=torch.float32, device="cuda")
@@ -135,20 +135,40 @@ def test_fused_head_parity(R, T, D, V, agg, ent, tis):
     compare_head(c, out)
 
 
-def test_fused_head_two_chunks_bf16_grad(R):
-    """More than 8,192 tokens: three chunks of 4,096 in one group (their dZ side by side, one dH
-    and one dW product); bf16 d_hidden."""
+@pytest.mark.parametrize("group_tokens", [0, 3 * 4096])
+def test_fused_head_three_chunks_bf16_grad(R, group_tokens):
+    """More than 8,192 tokens, bf16 d_hidden. With the smallest workspace each chunk of 4,096 is
+    its own group: dH's contraction over V is split in two halves added in fp32 in the
+    workspace, then rounded to bf16, and dW is added three times. With room for three chunks
+    the group holds them all: dH is stored directly in bf16 and dW is added once."""
     c = make_head_case(8192 + 77, 128, 1100, seed=5, agg=2)
-    out = run_head(R, c, dh_dtype=torch.bfloat16)
+    out = run_head(R, c, dh_dtype=torch.bfloat16, group_tokens=group_tokens)
     compare_head(c, out, dh_bf16=True)
 
 
-def test_fused_head_two_groups(R):
-    """More than 32,768 tokens: a full group of eight chunks and a ragged second group of two;
-    one dH and one dW product per group, the second group's dW added onto the first's."""
+@pytest.mark.parametrize("group_tokens", [0, 32768])
+def test_fused_head_ten_chunks(R, group_tokens):
+    """More than 32,768 tokens: ten chunks, each its own group (the smallest workspace: dW
+    added ten times), or a full group of eight and a ragged second group of two (dH stored in
+    fp32 over 32,768 tokens, the second group's dW added onto the first's)."""
     c = make_head_case(32768 + 4096 + 50, 64, 600, seed=11, agg=0, ent=True)
-    out = run_head(R, c)
+    out = run_head(R, c, group_tokens=group_tokens)
     compare_head(c, out)
+
+
+def test_fused_head_deterministic_and_workspace_independent(R):
+    """Two calls give the same bits (dH's split halves and dW's per-chunk additions land in a
+    fixed order); the smallest and a grouped workspace give the same loss and statistics bit
+    for bit (the products group their sums differently, so those are held to the oracle)."""
+    c = make_head_case(4096 + 300, 128, 2000, seed=8, agg=0)
+    a = run_head(R, c)
+    b = run_head(R, c)
+    g = run_head(R, c, group_tokens=8192)
+    for k in ("loss", "dH", "dW", "stats"):
+        assert np.array_equal(a[k], b[k]), k
+    for k in ("loss", "stats"):
+        assert np.array_equal(a[k], g[k]), k
+    compare_head(c, g)
 
 
 def test_fused_head_matches_logits_path(R):
