@@ -483,11 +483,14 @@ rl_status rl_fused_head_token_logprobs(const void* hidden, const void* weight, i
  *                  `stream`
  *
  * The first call on a device looks up the array's device address (once per
- * device, with that device current); make that first call before any stream
- * capture. Every call shares the one array, and each call clears the part that
- * must start at zero (the status word); calls that overlap on the GPU (for
- * example on two streams at once) race on it and must be serialised by the
- * caller.
+ * device, with that device current) and the library keeps it for the life of
+ * the process; make that first call before any stream capture, and make no call
+ * after a cudaDeviceReset of that device (the kept address would be stale).
+ * Every call shares the one array. Each call first clears the array's 256-byte
+ * header (the status word and the loss kernel's finished-cluster counter), so a
+ * call is not affected by what an earlier call left there; calls that overlap on
+ * the GPU (for example on two streams at once) race on the array, give wrong
+ * losses, and must be serialised by the caller.
  */
 rl_status rl_policy_loss_fwd_bwd_noalloc(const void* logits, rl_dtype dtype, int64_t rows, int64_t V,
                                          int64_t ld, const int32_t* token_ids, const uint8_t* mask,

@@ -24,7 +24,9 @@ constexpr int64_t kNoAllocMaxRows = 131072;
 // device address.
 static __device__ __align__(256) unsigned char g_noalloc_ws[kWsHeader + kNoAllocMaxRows * sizeof(double)];
 
-// Device address of g_noalloc_ws on the current device, looked up once per device.
+// Device address of g_noalloc_ws on the current device, looked up once per device (the first
+// call on a device) and kept for the life of the process: a cudaDeviceReset, which destroys the
+// context that holds the array, makes the kept address stale.
 static rl_status noalloc_workspace(void** out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -60,9 +62,10 @@ extern "C" rl_status rl_policy_loss_fwd_bwd_noalloc(
   rl_status st = noalloc_workspace(&ws);
   if (st != RL_OK) return st;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  // the status word is the only part that must start at zero: every row's loss slot
-  // is written by the kernel before the reduction reads it
-  cudaError_t e = cudaMemsetAsync(ws, 0, sizeof(int32_t), s);
+  // The 256-byte header must start at zero: it holds the status word and the loss kernel's
+  // finished-cluster counter, which a call that overlapped another one (or did not run to
+  // its end) can leave non-zero; the per-cluster loss slots are written before they are read.
+  cudaError_t e = cudaMemsetAsync(ws, 0, kWsHeader, s);
   if (e != cudaSuccess) return cuda_error(e, "rl_policy_loss_fwd_bwd_noalloc: cudaMemsetAsync");
   st = rl_policy_loss_fwd_bwd(logits, dtype, rows, V, ld, token_ids, mask, token_traj, n_traj, adv, coef, old_logp,
                               ref_logp, rollout_logp, params, grad_out, loss_accum, token_stats, ws,
