@@ -115,9 +115,8 @@ const char* rl_last_error_message(void);
  * workspace holds the device status word and per-row loss contributions; with
  * D > 0 it also holds the fused head's buffers, the largest being the bf16
  * gradient of the logits of ONE chunk of min(max_rows, 4096) tokens
- * (min(max_rows, 4096) * ceil(V / 8) * 8 * 2 bytes: 1.24 GB at V = 151,936),
- * plus min(max_rows, 4096) * D * 4 bytes of fp32 d_hidden. This is the
- * smallest workspace of rl_fused_head_loss_fwd_bwd. */
+ * (min(max_rows, 4096) * ceil(V / 8) * 8 * 2 bytes: 1.24 GB at V = 151,936).
+ * This is the smallest workspace of rl_fused_head_loss_fwd_bwd. */
 size_t rl_workspace_size(int64_t max_rows, int64_t V, int64_t D);
 
 /* Workspace bytes with which rl_fused_head_loss_fwd_bwd on up to T tokens keeps the

@@ -18,10 +18,11 @@
 // The dZ of one chunk (4,096 tokens x V in bf16) is the only logits-sized buffer; a caller
 // that passes more workspace lets a group of several chunks keep their dZ side by side.
 // After the group's last chunk (every chunk, with the smallest workspace):
-//   4. dH = dZ W and dW += dZ^T H over the group: head_grad_kernel (rl_head_grad.cu), the
-//      same CTA-pair tcgen05 machinery with the operands in their row-major layouts (dZ
-//      K-major for dH, MN-major for dW; W and H MN-major); dW is added in fp32 by TMA
-//      reduce-add, once per group.
+//   4. dH = dZ W and dW += dZ^T H over the group in one persistent launch of
+//      head_grad_kernel (rl_head_grad.cu): CTA-pair tcgen05 MMAs on 256 x 512 tiles with the
+//      operands in their row-major layouts (dZ K-major for dH, MN-major for dW; W and H
+//      MN-major), dH tiles first and dW tiles after them, handed out by a work counter; dH is
+//      stored, dW added in fp32 by TMA reduce-add, once per group.
 // The forward-only call runs head_kernel<STATS> (no stores) and head_logp_merge_kernel.
 // The objective (Sec. 2.3.2, Sec. 3.2.4) is the same as for rl_policy_loss_fwd_bwd; here
 // pi_theta's logits come from the hidden states times the vocabulary projection.
@@ -534,7 +535,7 @@ static rl_status make_map(CUtensorMap* m, const void* base, int64_t inner, int64
 
 struct Layout {
   int64_t Tc, G, n_nt, n_vb, ldz;  // G chunks per group
-  size_t off_partials, off_rc, off_tmax, off_dh32, off_dz, total;
+  size_t off_partials, off_rc, off_tmax, off_dz, total;
 };
 
 static size_t al256(size_t x) { return (x + 255) & ~size_t(255); }
@@ -542,7 +543,7 @@ static size_t al256(size_t x) { return (x + 255) & ~size_t(255); }
 // Workspace of the loss call for up to max_rows tokens. Its smallest form (ws_bytes = 0)
 // keeps the dZ of one chunk; every further Tc x ldz x 2 bytes the caller passes keep one more
 // chunk's dZ, so that the two products run once per group of G chunks.
-static Layout layout(int64_t max_rows, int64_t V, int64_t D, size_t ws_bytes = 0, int64_t want_G = 0) {
+static Layout layout(int64_t max_rows, int64_t V, size_t ws_bytes = 0, int64_t want_G = 0) {
   Layout L;
   L.Tc = std::max<int64_t>(1, std::min<int64_t>(max_rows, kChunk));
   const int64_t chunks = (std::max<int64_t>(max_rows, 1) + L.Tc - 1) / L.Tc;
@@ -558,8 +559,6 @@ static Layout layout(int64_t max_rows, int64_t V, int64_t D, size_t ws_bytes = 0
   off += al(static_cast<size_t>(L.Tc) * sizeof(RowCoef));
   L.off_tmax = off;
   off += al(static_cast<size_t>(L.Tc * n_nt) * sizeof(float));
-  L.off_dh32 = off;  // fp32 dH of one chunk: the two halves of a split contraction add here
-  off += al(static_cast<size_t>(L.Tc * std::max<int64_t>(D, 0)) * sizeof(float));
   L.off_dz = off;
   const size_t chunk_dz = static_cast<size_t>(L.Tc * L.ldz) * 2;
   int64_t G = std::max<int64_t>(want_G, 1);
@@ -568,16 +567,6 @@ static Layout layout(int64_t max_rows, int64_t V, int64_t D, size_t ws_bytes = 0
   off += al(static_cast<size_t>(L.G) * chunk_dz);
   L.total = off;
   return L;
-}
-
-// dH rows in fp32 -> bf16 (round to nearest even), 8 elements per thread and step.
-__global__ void __launch_bounds__(256) f32_to_bf16_kernel(const float4* __restrict__ src, uint4* __restrict__ dst,
-                                                          int64_t n8) {
-  for (int64_t k = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; k < n8;
-       k += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const float4 a = src[2 * k], b = src[2 * k + 1];
-    dst[k] = make_uint4(pack_bf16x2(a.x, a.y), pack_bf16x2(a.z, a.w), pack_bf16x2(b.x, b.y), pack_bf16x2(b.z, b.w));
-  }
 }
 
 template <int MODE>
@@ -639,12 +628,14 @@ static rl_status launch_head(const CUtensorMap& mh, const CUtensorMap& mw, const
 }  // namespace head
 
 size_t head_workspace_bytes(int64_t max_rows, int64_t V, int64_t D) {
-  return head::layout(max_rows, V, D).total;
+  (void)D;
+  return head::layout(max_rows, V).total;
 }
 
 size_t head_workspace_bytes_grouped(int64_t max_rows, int64_t V, int64_t D, int64_t group_tokens) {
   const int64_t g = (std::max<int64_t>(group_tokens, 1) + head::kChunk - 1) / head::kChunk;
-  return head::layout(max_rows, V, D, 0, g).total;
+  (void)D;
+  return head::layout(max_rows, V, 0, g).total;
 }
 
 // The forward-only call needs the status word and one chunk's partials, which sit at the
@@ -655,7 +646,7 @@ size_t head_workspace_bytes_grouped(int64_t max_rows, int64_t V, int64_t D, int6
 // 3,072 and 6,144 are within 2%, 8,192 takes 26.7 ms (73.1), and 32,768 takes 31.5 ms: the
 // hidden states (256 MB) then evict W's tiles from the 129 MB L2.
 static size_t head_logp_workspace_bytes(int64_t T, int64_t V) {
-  const head::Layout L = head::layout(T, V, 0);
+  const head::Layout L = head::layout(T, V);
   return kWsHeader + head::al256(static_cast<size_t>(L.n_vb * L.Tc) * sizeof(float4));
 }
 
@@ -694,14 +685,13 @@ extern "C" rl_status rl_fused_head_loss_fwd_bwd(
                      "rl_fused_head_loss_fwd_bwd: hidden, weight, d_hidden, d_weight and ws must be 16-byte aligned");
 
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  const Layout L = layout(T, V, D, ws_bytes);
+  const Layout L = layout(T, V, ws_bytes);
   char* wsb = static_cast<char*>(ws);
   int32_t* status = reinterpret_cast<int32_t*>(wsb);
   double* row_loss = reinterpret_cast<double*>(wsb + ws_row_loss_offset());
   float4* partials = reinterpret_cast<float4*>(wsb + L.off_partials);
   RowCoef* rcs = reinterpret_cast<RowCoef*>(wsb + L.off_rc);
   float* tmax = reinterpret_cast<float*>(wsb + L.off_tmax);
-  float* dh32 = reinterpret_cast<float*>(wsb + L.off_dh32);
   uint16_t* dz_base = reinterpret_cast<uint16_t*>(wsb + L.off_dz);
   rl_status st = RL_OK;
   const bool kl_on = params->kl_estimator == 3 && params->kl_coef != 0.f && ref_logp != nullptr;
@@ -784,30 +774,9 @@ extern "C" rl_status rl_fused_head_loss_fwd_bwd(
     const int64_t g1 = std::min<int64_t>(g0 + group_rows, T);
     if (t0 + Tc == g1) {
       const int64_t n = g1 - g0;
-      const bool bf16_out = d_hidden_dtype == RL_BF16;
-      void* dh = static_cast<char*>(d_hidden) + g0 * D * (bf16_out ? 2 : 4);
-      // dH[g0 : g1] = dZ W; a split contraction adds its two halves onto zeros in fp32 (the
-      // caller's fp32 rows, or the workspace's one-chunk buffer before rounding to bf16)
-      const int split = (bf16_out && n > L.Tc) ? 1 : head_grad_dh_split(n, V, D);
-      if (split == 2) {
-        float* acc = bf16_out ? dh32 : static_cast<float*>(dh);
-        e = cudaMemsetAsync(acc, 0, static_cast<size_t>(n * D) * sizeof(float), s);
-        if (e != cudaSuccess) return cuda_error(e, "cudaMemsetAsync(d_hidden)");
-        st = head_grad_dh(dz_base, L.ldz, n, V, weight, D, acc, 0, 2, status, s);
-        if (st != RL_OK) return st;
-        if (bf16_out) {
-          const int64_t n8 = n * D / 8;
-          f32_to_bf16_kernel<<<static_cast<int>(std::min<int64_t>((n8 + 255) / 256, 148 * 8)), 256, 0, s>>>(
-              reinterpret_cast<const float4*>(dh32), static_cast<uint4*>(dh), n8);
-          e = cudaGetLastError();
-          if (e != cudaSuccess) return cuda_error(e, "f32_to_bf16_kernel launch");
-        }
-      } else {
-        st = head_grad_dh(dz_base, L.ldz, n, V, weight, D, dh, bf16_out ? 2 : 1, 1, status, s);
-        if (st != RL_OK) return st;
-      }
-      // dW += dZ^T H[g0 : g1]
-      st = head_grad_dw(dz_base, L.ldz, n, V, static_cast<const uint16_t*>(hidden) + g0 * D, D, d_weight, status, s);
+      void* dh = static_cast<char*>(d_hidden) + g0 * D * (d_hidden_dtype == RL_BF16 ? 2 : 4);
+      st = head_grad(dz_base, L.ldz, n, V, weight, static_cast<const uint16_t*>(hidden) + g0 * D, D, dh,
+                     d_hidden_dtype, d_weight, reinterpret_cast<uint32_t*>(wsb + kWsHeadCounterOffset), status, s);
       if (st != RL_OK) return st;
     }
   }
@@ -836,7 +805,7 @@ extern "C" rl_status rl_fused_head_token_logprobs(const void* hidden, const void
     return set_error(RL_ERR_ALIGNMENT, "rl_fused_head_token_logprobs: hidden, weight and ws must be 16-byte aligned");
 
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  const Layout L = layout(T, V, 0);
+  const Layout L = layout(T, V);
   char* wsb = static_cast<char*>(ws);
   int32_t* status = reinterpret_cast<int32_t*>(wsb);
   float4* partials = reinterpret_cast<float4*>(wsb + kWsHeader);

@@ -24,6 +24,8 @@ inline size_t ws_row_loss_offset() { return kWsHeader; }
 constexpr size_t kWsDoneOffset = 16;
 // The same for the value loss kernel's finished CTAs.
 constexpr size_t kWsValueDoneOffset = 20;
+// Work-item counter of the fused head's backward products (zeroed before each launch).
+constexpr size_t kWsHeadCounterOffset = 24;
 
 rl_status set_error(rl_status st, const std::string& msg);
 rl_status cuda_error(cudaError_t e, const char* what);
@@ -36,18 +38,13 @@ size_t head_workspace_bytes(int64_t max_rows, int64_t V, int64_t D);
 // The same, keeping the dZ of up to group_tokens tokens (whole chunks) at once.
 size_t head_workspace_bytes_grouped(int64_t max_rows, int64_t V, int64_t D, int64_t group_tokens);
 
-// Backward products of the fused LM head on the tensor cores (rl_head_grad.cu). dz is the
-// bf16 gradient of the logits of n tokens ([n x V], rows ldz elements apart).
-// out_kind: 0 = add into fp32 (TMA reduce-add), 1 = store fp32, 2 = store bf16.
-// dH[n x D] = dZ W; with ksplit = 2 the contraction over V is cut in two halves that are
-// both added (out_kind 0) into a zeroed fp32 destination.
-rl_status head_grad_dh(const uint16_t* dz, int64_t ldz, int64_t n, int64_t V, const void* weight, int64_t D,
-                       void* out, int out_kind, int ksplit, int32_t* status, cudaStream_t s);
-// dW[V x D] += dZ^T H[n x D] (fp32, one addition per element).
-rl_status head_grad_dw(const uint16_t* dz, int64_t ldz, int64_t n, int64_t V, const void* hidden, int64_t D,
-                       float* d_weight, int32_t* status, cudaStream_t s);
-// 2 if splitting dH's contraction in two balances the CTA pairs' work better, else 1.
-int head_grad_dh_split(int64_t n, int64_t V, int64_t D);
+// Backward products of the fused LM head on the tensor cores (rl_head_grad.cu), one launch:
+// d_hidden[n x D] = dZ W (stored, bf16 or fp32) and d_weight[V x D] += dZ^T H[n x D] (fp32),
+// with dz the bf16 gradient of the logits of the n tokens ([n x V], rows ldz elements apart).
+// counter: a workspace word for the work-item counter (zeroed here, on the stream).
+rl_status head_grad(const uint16_t* dz, int64_t ldz, int64_t n, int64_t V, const void* weight, const void* hidden,
+                    int64_t D, void* d_hidden, rl_dtype dh_dtype, float* d_weight, uint32_t* counter,
+                    int32_t* status, cudaStream_t s);
 
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
