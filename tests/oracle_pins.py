@@ -561,6 +561,28 @@ def pin_logprobs_vs_library(O):
     _close(H, -(np.exp(ls) * ls).sum(axis=1), rtol=1e-10, what="entropy")
 
 
+def pin_decode_logits_vs_library(O):
+    """decode_logits of bf16 bit patterns equals torch's own bfloat16 -> float64 conversion on
+    every class of pattern: zeros of both signs, subnormals, normals, the largest finite values,
+    +-inf and NaNs, and a random sample of all 65,536 patterns."""
+    import torch
+
+    special = np.array([0x0000, 0x8000, 0x0001, 0x8001, 0x007F, 0x807F, 0x0080, 0x8080, 0x3F80, 0xBF80,
+                        0x7F7F, 0xFF7F, 0x7F80, 0xFF80, 0x7FC0, 0xFFC0, 0x7F81, 0xFFFF], dtype=np.uint16)
+    rng = np.random.default_rng(31)
+    bits = np.concatenate([special, rng.integers(0, 1 << 16, size=4096, dtype=np.uint32).astype(np.uint16)])
+    got = O.decode_logits(bits, "bf16")
+    ref = torch.from_numpy(bits.view(np.int16).copy()).view(torch.bfloat16).double().numpy()
+    assert got.dtype == np.float64 and got.shape == ref.shape
+    nan = np.isnan(ref)
+    assert np.array_equal(np.isnan(got), nan), "NaN patterns"
+    assert np.array_equal(got[~nan], ref[~nan]), "decoded values"
+    assert np.array_equal(np.signbit(got[~nan]), np.signbit(ref[~nan])), "signs (of zeros too)"
+    assert got[2] == 2.0 ** -133 and got[4] == (1 - 2.0 ** -7) * 2.0 ** -126 and got[6] == 2.0 ** -126, "subnormals"
+    f32 = rng.normal(0, 100, size=64).astype(np.float32)
+    _close(O.decode_logits(f32, "f32"), torch.from_numpy(f32).double().numpy(), rtol=0, atol=0, what="f32 decode")
+
+
 # ---------------------------------------------------------------------------
 # C: fused head
 # ---------------------------------------------------------------------------

@@ -72,6 +72,9 @@ MUTANTS = {
     "summary counts masked tokens": ("act = (np.asarray(mask) != 0) & (c != 0)", "act = c != 0"),
     "summary sums the wrong column": ("math.fsum(st[act, STAT_ENTROPY])", "math.fsum(st[act, STAT_LOGP])"),
     "head logprobs chunk offset": ("Z = Hm[r0:r0 + chunk] @ Wm.T", "Z = Hm[r0 + 1:r0 + 1 + chunk] @ Wm.T"),
+    "bf16 decode shifted by 15": ("<< np.uint32(16)", "<< np.uint32(15)"),
+    "bf16 decoded as fp16": ("return bits.view(np.float32).astype(np.float64)",
+                             "return np.asarray(raw, dtype=np.uint16).view(np.float16).astype(np.float64)"),
 }
 
 
