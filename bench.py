@@ -652,6 +652,25 @@ def e2e_run(torch, R, batch, dev, steps, warmup, slots=4, repeats=3):
 _W = {}
 
 
+def _gen_init(shm_name, shape, ids_name):
+    from multiprocessing import shared_memory
+
+    sys.path.insert(0, ROOT)
+    shm, ids_shm = shared_memory.SharedMemory(name=shm_name), shared_memory.SharedMemory(name=ids_name)
+    _W.update(shm=shm, ids_shm=ids_shm, raw=np.ndarray(shape, dtype=np.uint16, buffer=shm.buf),
+              ids=np.ndarray((shape[0],), dtype=np.int32, buffer=ids_shm.buf))
+
+
+def _gen_rows(span):
+    """Draw rows [lo, hi) of the workload with the numpy generators (each row its own seeded
+    stream, so any split of the rows gives the same values)."""
+    lo, hi = span
+    raw, vals = W.logits_rows_np(WORKLOAD, 0, lo, hi - lo)
+    _W["raw"][lo:hi] = raw
+    _W["ids"][lo:hi] = W.sample_tokens_np(vals, 0, lo, WORKLOAD)
+    return hi - lo
+
+
 def _oracle_init(shm_name, shape, ids, mask, tt, adv, coef, old):
     from multiprocessing import shared_memory
 
@@ -670,107 +689,151 @@ def _oracle_rows(span):
     return hi - lo
 
 
-def oracle_sample_inputs(batch_host):
-    """Inputs of the CPU oracle for a sample of the workload: the first packed tokens.
+class OracleSample:
+    """The first microbatch of the benchmark batch (its first 16,384 packed tokens) in host
+    shared memory for the float64 oracle: copied from the device batch (torch-drawn, the rows the
+    GPU times) or, without a GPU, drawn by the numpy generators on all host cores (same law)."""
 
-    old_logp is placed near the sampled token's log-probability from the logit law
-    (lse ~ ln V + sigma^2 / 2 for N(0, sigma^2) logits), which keeps the timing leg
-    independent of the CUDA library's outputs."""
-    import oracle.grpo_objective as O
-
-    w = WORKLOAD
-    lay = batch_host["layout"]
-    raw = batch_host["raw"]
-    ids = batch_host["ids"]
-    rows = raw.shape[0]
-    z_a = (raw[np.arange(rows), ids].astype(np.uint32) << 16).view(np.float32).astype(np.float64)
-    logp_hat = z_a - (math.log(w.vocab) + w.logit_std ** 2 / 2)
-    old = W.old_logp_from(logp_hat, w, 0)
-    P = O.LossParams()
-    adv, coef, L, tt = O.advantages_and_coefficients(lay.rewards, lay.group_offsets, lay.traj_offsets, lay.mask,
-                                                     lay.traj_valid, P)
-    return raw, ids, lay.mask[:rows], tt[:rows], adv, coef, old
-
-
-class OraclePool:
-    """The float64 oracle, as it stands, over a spawn pool of all host cores.
-
-    The sample's logits sit in shared memory; each job is a 16-row span of the sample.
-    ``run(seconds)`` cycles over the sample's spans for about that long and returns
-    rows per second."""
-
-    CHUNK = 16
-
-    def __init__(self, batch_host):
+    def __init__(self, rows, device_logits=None, device_ids=None):
         from multiprocessing import shared_memory
 
-        self.cores = len(os.sched_getaffinity(0))
-        raw, ids, mask, tt, adv, coef, old = oracle_sample_inputs(batch_host)
-        self.rows = raw.shape[0]
-        self.shm = shared_memory.SharedMemory(create=True, size=raw.nbytes)
-        np.ndarray(raw.shape, dtype=np.uint16, buffer=self.shm.buf)[:] = raw
-        self.spans = [(i, min(self.rows, i + self.CHUNK)) for i in range(0, self.rows, self.CHUNK)]
-        self.pool = mp.get_context("spawn").Pool(self.cores, initializer=_oracle_init,
-                                                 initargs=(self.shm.name, raw.shape, ids, mask, tt, adv, coef, old))
-        self.pool.map(_oracle_rows, self.spans[:self.cores], chunksize=1)   # imports and first touch
-        t0 = time.perf_counter()
-        n = sum(self.pool.map(_oracle_rows, [self.spans[j % len(self.spans)] for j in range(self.cores)],
-                              chunksize=1))
-        self.rate = n / max(time.perf_counter() - t0, 1e-6)
-        self.done = 0
-        self.wall = 0.0
+        self.layout = W.make_layout(WORKLOAD, 0)
+        self.rows = rows
+        V = WORKLOAD.vocab
+        self.shm = shared_memory.SharedMemory(create=True, size=rows * V * 2)
+        self.raw = np.ndarray((rows, V), dtype=np.uint16, buffer=self.shm.buf)
+        if device_logits is not None:
+            import torch
 
-    def run(self, seconds):
-        n_jobs = max(self.cores, int(self.rate * seconds / self.CHUNK))
-        jobs = [self.spans[(self.done // self.CHUNK + j) % len(self.spans)] for j in range(n_jobs)]
-        t0 = time.perf_counter()
-        done = sum(self.pool.map(_oracle_rows, jobs, chunksize=1))
-        dt = time.perf_counter() - t0
-        self.done += done
-        self.wall += dt
-        return done / dt
+            torch.from_numpy(self.raw.view(np.int16)).copy_(device_logits[:rows].view(torch.int16))
+            self.ids = device_ids[:rows].cpu().numpy().astype(np.int32)
+            self.source = "the device batch's torch-drawn logits, copied to the host"
+        else:
+            ids_shm = shared_memory.SharedMemory(create=True, size=rows * 4)
+            try:
+                spans = [(i, min(rows, i + 16)) for i in range(0, rows, 16)]
+                cores = len(os.sched_getaffinity(0))
+                with mp.get_context("spawn").Pool(cores, initializer=_gen_init,
+                                                  initargs=(self.shm.name, (rows, V), ids_shm.name)) as pool:
+                    pool.map(_gen_rows, spans, chunksize=4)
+                self.ids = np.ndarray((rows,), dtype=np.int32, buffer=ids_shm.buf).copy()
+            finally:
+                ids_shm.close()
+                ids_shm.unlink()
+            self.source = "numpy-drawn logits of the same law (no GPU used)"
 
-    def describe(self):
-        return {"unit": UNIT, "cores": self.cores, "kind": "oracle",
-                "sample": f"{self.done} token rows cycled over the first {self.rows} packed tokens of the batch "
-                          f"(masked rows included), float64 numpy oracle on {self.cores} spawn workers, "
-                          f"{self.wall:.1f} s wall"}
+    def oracle_inputs(self):
+        """Inputs of the oracle for these rows. old_logp is placed near the sampled token's
+        log-probability from the logit law (lse ~ ln V + sigma^2 / 2 for N(0, sigma^2) logits),
+        which keeps the timing leg independent of the CUDA library's outputs."""
+        import oracle.grpo_objective as O
+
+        w, lay, rows = WORKLOAD, self.layout, self.rows
+        z_a = (self.raw[np.arange(rows), self.ids].astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+        logp_hat = z_a - (math.log(w.vocab) + w.logit_std ** 2 / 2)
+        old = W.old_logp_from(logp_hat, w, 0)
+        P = O.LossParams()
+        adv, coef, L, tt = O.advantages_and_coefficients(lay.rewards, lay.group_offsets, lay.traj_offsets, lay.mask,
+                                                         lay.traj_valid, P)
+        return self.ids, lay.mask[:rows], tt[:rows], adv, coef, old
 
     def close(self):
-        self.pool.close()
-        self.pool.join()
         self.shm.close()
         self.shm.unlink()
 
 
-def time_oracle(batch_host, target_s=15.0):
-    """One bounded timing of the oracle on a sample of the workload (about target_s of wall time)."""
-    op = OraclePool(batch_host)
+class OraclePool:
+    """The float64 oracle, as it stands, over a spawn pool of all host cores. Each job is a
+    16-row span of the sample; ``run(lo, hi)`` times the oracle over rows [lo, hi) once."""
+
+    CHUNK = 16
+
+    def __init__(self, sample: OracleSample):
+        self.cores = len(os.sched_getaffinity(0))
+        self.sample = sample
+        ids, mask, tt, adv, coef, old = sample.oracle_inputs()
+        self.pool = mp.get_context("spawn").Pool(self.cores, initializer=_oracle_init,
+                                                 initargs=(sample.shm.name, sample.raw.shape, ids, mask, tt, adv,
+                                                           coef, old))
+        # imports and first touch of the workers (untimed)
+        self.pool.map(_oracle_rows, [(i * self.CHUNK, (i + 1) * self.CHUNK) for i in range(self.cores)], chunksize=1)
+
+    def run(self, lo, hi):
+        """Seconds of wall time for the oracle over rows [lo, hi)."""
+        spans = [(i, min(hi, i + self.CHUNK)) for i in range(lo, hi, self.CHUNK)]
+        t0 = time.perf_counter()
+        n = sum(self.pool.map(_oracle_rows, spans, chunksize=1))
+        dt = time.perf_counter() - t0
+        assert n == hi - lo
+        return dt
+
+    def close(self):
+        self.pool.close()
+        self.pool.join()
+
+
+def time_oracle(sample: OracleSample):
+    """The oracle over the whole first microbatch, once (about 1.5 s on 16 host cores)."""
+    op = OraclePool(sample)
     try:
-        v = op.run(target_s)
-        d = op.describe()
+        dt = op.run(0, sample.rows)
     finally:
         op.close()
-    d["value"] = v
-    return d
-
-
-def host_sample(torch, batch, rows):
-    """Copy a sample of the device workload (torch-drawn logits and ids) to the host."""
-    raw = batch.logits[:rows].view(torch.int16).cpu().numpy().view(np.uint16)
-    ids = batch.ids[:rows].cpu().numpy()
-    return {"layout": batch.lay, "raw": raw, "ids": ids}
-
-
-def host_sample_np(rows):
-    """A host-only sample of the same workload (numpy generator), for runs without a GPU."""
-    lay = W.make_layout(WORKLOAD, 0)
-    raw, vals = W.logits_rows_np(WORKLOAD, 0, 0, rows)
-    ids = W.sample_tokens_np(vals, 0, 0, WORKLOAD)
-    return {"layout": lay, "raw": raw, "ids": ids}
+    lay = sample.layout
+    trained = int(lay.mask[:sample.rows].sum())
+    return {"value": sample.rows / dt, "unit": UNIT, "cores": op.cores, "kind": "oracle", "seconds": dt,
+            "sample": f"the first microbatch of the batch, all {sample.rows} rows ({trained} trained, the others "
+                      f"masked), once, from {sample.source}; float64 numpy oracle on {op.cores} spawn workers"}
 
 
 # ----------------------------------------------------------------------------- main
+
+def _r(x, nd=4):
+    return None if x is None else float(f"{x:.{nd}g}")
+
+
+def compact_summary(value, ms_step, roofline, extras, head, ppo, tree, cpu, e2e):
+    """One short object per workload (time, tokens/s, fraction of the roofline it is held to),
+    printed as the last key of the JSON line so that a reader keeping only the line's tail
+    still has every workload's numbers."""
+    out = {"multiturn_loss": {"ms_per_step": _r(ms_step), "tokens_per_s": _r(value), "frac": _r(roofline["frac"]),
+                              "bound": "hbm"}}
+    for k in ("longhorizon", "edge"):
+        o = (extras.get("other_workloads") or {}).get(k)
+        if o:
+            out[f"{k}_loss"] = {"ms": _r(o["ms_per_launch"]), "tokens_per_s": _r(o["tokens_per_s"]),
+                                "frac": _r(o["frac"]), "bound": "hbm"}
+    tiny = (extras.get("other_workloads") or {}).get("tiny")
+    if tiny:
+        out["tiny_step"] = {"us_graph": _r(tiny["us_per_step_graph"]), "tokens_per_s": _r(tiny["tokens_per_s_graph"]),
+                            "frac": None, "bound": "latency (L2-resident)"}
+    for k in ("token_logprobs", "token_logprobs_entropy"):
+        o = extras.get(k)
+        if o:
+            out[k] = {"ms": _r(o["ms_per_batch"]), "tokens_per_s": _r(o["tokens_per_s"]), "frac": _r(o["frac"]),
+                      "bound": "hbm (read only)"}
+    if head:
+        out["fused_head_loss"] = {"ms": _r(head["ms_per_call"]), "tokens_per_s": _r(head["tokens_per_s"]),
+                                  "frac": _r(head["frac"]), "frac_of_sustained": _r(head["frac_of_sustained"]),
+                                  "bound": "tensor"}
+        f = head["logprobs"]
+        out["fused_head_logprobs"] = {"ms": _r(f["ms_per_call"]), "tokens_per_s": _r(f["tokens_per_s"]),
+                                      "frac": _r(f["frac"]), "frac_of_sustained": _r(f["frac_of_sustained"]),
+                                      "bound": "tensor"}
+    if ppo:
+        out["ppo_step"] = {"ms": _r(ppo["ms_per_step"]), "tokens_per_s": _r(ppo["tokens_per_s"]), "frac": None,
+                           "bound": "hbm (its policy loss)"}
+    if "group_advantages_us" in extras:
+        out["group_advantages"] = {"us": _r(extras["group_advantages_us"]), "bound": "latency"}
+    if tree:
+        out["tree_build"] = {"ms": _r(tree["host_build_ms"]), "captured_tokens_per_s": _r(tree["host_captured_tokens_per_s"]),
+                             "bound": "host"}
+    if cpu:
+        out["cpu_oracle"] = {"tokens_per_s": _r(cpu["value"]), "cores": cpu["cores"]}
+    if e2e:
+        out["e2e"] = {"tokens_per_s": _r(e2e["value"])}
+    return out
+
 
 def max_over_ranks(value, dist, device):
     """Maximum of a per-rank float over all ranks (the step time every rank reports)."""
@@ -794,28 +857,49 @@ def dist_env():
 
 
 def run_reference(args):
-    """The oracle timed on the host cores, on the same workload, metric and unit: each step is a
-    bounded sample sized so that the whole run stays within a few minutes."""
+    """The oracle timed on the host cores, on the same workload, metric and unit. Each step runs
+    the oracle over a span of the first microbatch's rows (the whole microbatch when the run is
+    short; fewer rows per step for many steps, so that the run stays within a few minutes), the
+    spans following each other through the microbatch; value is rows over the measured seconds
+    of the timed steps and ms_per_step their measured median."""
     rank, world, _ = dist_env()
     if rank != 0:
         return 0
     lay = W.make_layout(WORKLOAD, 0)
     n_mb = len(W.microbatches(lay, WORKLOAD.microbatch))
-    op = OraclePool(host_sample_np(min(lay.n_tokens, 512)))
-    per_step = max(0.3, 150.0 / max(1, args.steps + args.warmup))
-    vals = []
+    rows = min(lay.n_tokens, WORKLOAD.microbatch)
+    sample = OracleSample(rows)
+    op = None
     try:
-        for i in range(args.warmup + args.steps):
-            v = op.run(per_step)
+        op = OraclePool(sample)
+        # rows per step: about 120 s of oracle time for the whole run at the first span's rate
+        n_probe = min(rows, 4 * op.CHUNK * op.cores)
+        rate = n_probe / op.run(0, n_probe)
+        steps = args.warmup + args.steps
+        per_step = int(min(rows, max(op.CHUNK * op.cores, rate * 120.0 / steps)))
+        per_step -= per_step % op.CHUNK
+        times, lo = [], 0
+        for i in range(steps):
+            if lo + per_step > rows:
+                lo = 0
+            dt = op.run(lo, lo + per_step)
+            lo += per_step
             if i >= args.warmup:
-                vals.append(v)
-        cb = op.describe()
+                times.append(dt)
+        cores = op.cores
     finally:
-        op.close()
-    v = statistics.median(vals)
-    cb["value"] = v
+        if op is not None:
+            op.close()
+        sample.close()
+    v = per_step * len(times) / sum(times)
+    ms_step = statistics.median(times) * 1e3
+    trained = int(lay.mask[:rows].sum())
+    cb = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
+          "sample": f"{per_step} rows per step (of the first microbatch's {rows}, {trained} trained), "
+                    f"{args.steps} timed steps after {args.warmup} warm-up steps, from {sample.source}; float64 "
+                    f"numpy oracle on {cores} spawn workers"}
     line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": lay.n_tokens / v * 1e3,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step, "rows_per_step": per_step,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": workload_config(lay.n_tokens, n_mb), "cpu_baseline": cb,
             "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -945,7 +1029,9 @@ def time_head(torch, R, dev, warmup=2, reps=5):
             "peak": burst, "unit": "TFLOP/s", "frac": tf / burst, "frac_of_sustained": tf / sustained,
             "peak_source": kind, "algorithmic_flops_per_call": flops, "executed_flops_per_call": flops,
             "reps": reps, "chunks_per_call": chunks,
-            "note": "6 T D V (Z once, dH, dW); dH and dW through cuBLASLt",
+            "note": "6 T D V (Z once, dH, dW), all on hand-written tcgen05 kernels (head_kernel: logits tiles and "
+                    "softmax partials; head_grad_kernel: dH and dW in one launch), smallest workspace "
+                    f"({hb.ws.numel() / 1e9:.2f} GB: one 4,096-token chunk of the logits gradient)",
             "logprobs": fwd}
 
 
@@ -1161,8 +1247,8 @@ def main():
     extras = time_logits_extras(torch, R, batch, dev, peak)
     if not args.no_other:
         extras["other_workloads"] = time_other_workloads(torch, R, dev, peak)
-    extras["loss_microbatches"] = per_mb
     extras["loss_batch_sum_ms"] = sum(m["median_ms"] for m in per_mb)
+    extras["loss_microbatch_median_ms"] = [round(m["median_ms"], 4) for m in per_mb]
 
     e2e = None
     if not args.no_e2e:
@@ -1176,7 +1262,11 @@ def main():
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = time_oracle(host_sample(torch, batch, 2048))
+        sample = OracleSample(batch.mbs[0][1] - batch.mbs[0][0], batch.logits, batch.ids)
+        try:
+            cpu = time_oracle(sample)
+        finally:
+            sample.close()
 
     ppo = None if args.no_ppo else time_ppo(torch, R, batch, dev)
     tree = None if args.no_tree else time_tree(torch, R, dev)
@@ -1186,12 +1276,14 @@ def main():
         head = time_head(torch, R, dev)
 
     if rank == 0:
+        summary = compact_summary(value, ms_step, roofline, extras, head, ppo, tree, cpu, e2e)
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": "f32", "data": "synthetic", "config": workload_config(batch.T, n_mb, batch.inputs_sha256),
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks, "logits_path": extras, "fused_head": head, "ppo": ppo, "tree": tree,
                 "gpu_launches": batch.launches_per_step() * args.steps,
-                "loss_per_step": float(batch.loss.item()) / (args.warmup + args.steps)}
+                "loss_per_step": float(batch.loss.item()) / (args.warmup + args.steps),
+                "summary": summary}
         print(json.dumps(line))
     if world > 1:
         dist.destroy_process_group()

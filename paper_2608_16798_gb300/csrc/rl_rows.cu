@@ -176,23 +176,17 @@ __device__ __forceinline__ void raise_max(SoftmaxPartial& ps, float vm) {
   }
 }
 
-// Tuning knobs (compile-time): shared-memory stages per CTA, consumer warps per
-// CTA, and the slice size that picks the cluster width.
+// Shared-memory stages per CTA (tuning knob). The consumer warps per CTA, the 16-byte vectors
+// of the slice each consumer thread holds in registers, the CTAs per SM and the slice size that
+// picks the cluster width are chosen per path on the host (loss_shape).
 #ifndef RL_STAGES
 #define RL_STAGES 2
 #endif
-#ifndef RL_CONSUMER_WARPS
-#define RL_CONSUMER_WARPS 7
-#endif
-#ifndef RL_SLICE_KB
-#define RL_SLICE_KB 40
-#endif
 
 constexpr int kMaxCluster = 16;
-#ifndef RL_ZERO_BYTES
-#define RL_ZERO_BYTES 8192
-#endif
-constexpr int kZeroBytes = RL_ZERO_BYTES;  // zero-filled shared region, source of the masked rows' bulk stores
+// zero-filled shared region, source of the masked rows' bulk stores (8 KB at 2 CTAs per SM:
+// 12.947 against 13.029 ms per benchmark step with 2 KB)
+constexpr int kZeroBytesMax = 8192;
 
 // Per-row inputs, staged in shared memory by the producer warp.
 struct RowMeta {
@@ -347,8 +341,10 @@ __device__ __forceinline__ void fold_block(SoftmaxPartial& ps, const uint4 (&x)[
   ps.s = fmaf(se, f, ps.s);
 }
 
-template <typename T, int NW, bool ENT, bool BWD, int HOLDV>
-__global__ void __launch_bounds__((NW + 1) * 32, 2) rows_kernel(const RowArgs p) {
+// MINB: CTAs per SM the register budget is sized for (2, or 3 with a smaller zero region).
+template <typename T, int NW, bool ENT, bool BWD, int HOLDV, int MINB>
+__global__ void __launch_bounds__((NW + 1) * 32, MINB) rows_kernel(const RowArgs p) {
+  constexpr int kZeroBytes = MINB >= 3 ? 2048 : kZeroBytesMax;
   constexpr int EPV = Vec<T>::N;
   constexpr int NB = RL_STAGES;
   constexpr int NC = NW * 32;  // consumer threads
@@ -933,9 +929,6 @@ __global__ void __launch_bounds__((NW + 1) * 32, 2) stream_logprobs_kernel(const
 
 // ------------------------------------------------------------------ host side
 
-constexpr int kConsumerWarps = RL_CONSUMER_WARPS;
-constexpr int kRowThreads = (RL_CONSUMER_WARPS + 1) * 32;
-constexpr int64_t kTargetSliceBytes = RL_SLICE_KB * 1024;
 constexpr int64_t kMaxSliceBytes = 100 * 1024;
 
 struct Plan {
@@ -944,12 +937,13 @@ struct Plan {
   size_t smem;
 };
 
-static bool make_plan(int64_t V, int es, Plan* out) {
+// Smallest cluster whose slices are at most target_bytes (or, at 16 CTAs, at most 100 KB).
+static bool make_plan(int64_t V, int es, Plan* out, int64_t target_bytes = 40 * 1024) {
   const int64_t epv = 16 / es;
   for (int C = 1; C <= 16; ++C) {
     const int64_t per = (V + C - 1) / C;
     const int64_t slice = (per + epv - 1) / epv * epv;
-    if (slice * es <= kTargetSliceBytes || (C == 16 && slice * es <= kMaxSliceBytes)) {
+    if (slice * es <= target_bytes || (C == 16 && slice * es <= kMaxSliceBytes)) {
       const int64_t stride_bytes = (slice * es + 127) / 128 * 128;
       out->C = C;
       out->slice = slice;
@@ -979,9 +973,10 @@ static rl_status configure(const void* kern, int dev, size_t smem) {
   return RL_OK;
 }
 
-template <typename T, bool ENT, int HOLDV>
+template <typename T, int NW, bool ENT, int HOLDV, int MINB>
 static rl_status launch_rows(const RowArgs& args, const Plan& plan, cudaStream_t s, int64_t* n_clusters_out) {
-  auto kern = rows_kernel<T, kConsumerWarps, ENT, true, HOLDV>;
+  auto kern = rows_kernel<T, NW, ENT, true, HOLDV, MINB>;
+  constexpr int kRowThreads = (NW + 1) * 32;
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return cuda_error(e, "cudaGetDevice");
@@ -1034,18 +1029,59 @@ static rl_status launch_rows(const RowArgs& args, const Plan& plan, cudaStream_t
   return RL_OK;
 }
 
-// Registers hold the slice when it fits kHoldVecs 16-byte vectors per consumer thread.
-constexpr int kHoldVecs = 11;
+// Shape of the loss kernel per path, from sweeps on the GB300 (full-size microbatches):
+//   bf16 without the entropy (the benchmark): 8 consumer warps holding up to 10 vectors each,
+//     slices up to 40 KB (clusters of 8 at V = 151,936), 2 CTAs per SM: 12.84 ms per benchmark
+//     step against 12.96 with 7 warps of 11 vectors; wider clusters or 3 CTAs per SM were
+//     slower (13.6-18.5 ms);
+//   bf16 with the entropy: 7 warps of 11 vectors, clusters of 8, 2 CTAs per SM: 3.20 ms per
+//     32,768-row long-horizon microbatch, against 3.35-3.71 with 8, 9 or 11 warps and
+//     3.57-4.61 with clusters of 10, 12 or 16 at 3 CTAs per SM;
+//   fp32: slices up to 30 KB (clusters of 5 at V = 32,000), 7 warps of up to 9 vectors, 3 CTAs
+//     per SM: 4.15 ms per 131,072-row edge batch against 4.35 with clusters of 4 at 2 per SM.
+template <typename T>
+struct LossShape;
+template <>
+struct LossShape<uint16_t> {
+  static constexpr int64_t kSliceBytes[2] = {40 * 1024, 40 * 1024};  // [entropy off, on]
+};
+template <>
+struct LossShape<float> {
+  static constexpr int64_t kSliceBytes[2] = {30 * 1024, 30 * 1024};
+};
+
+// The plan of the loss kernel for this path (the forward-only kernel has no clusters).
+template <typename T>
+static Plan loss_plan(int64_t V, bool ent) {
+  Plan plan;
+  if (!make_plan(V, static_cast<int>(sizeof(T)), &plan, LossShape<T>::kSliceBytes[ent ? 1 : 0]))
+    make_plan(V, static_cast<int>(sizeof(T)), &plan);
+  return plan;
+}
 
 // Launches the loss kernel; *n_clusters receives the number of clusters, each of which leaves
 // one loss partial at the head of the per-row loss area (the last one also adds them up).
+// Registers hold the slice when it fits the path's held vectors; otherwise the slice stays in
+// shared memory (7 warps, 2 CTAs per SM, slices up to 40 KB).
 template <typename T>
-static rl_status dispatch_loss(bool ent, const RowArgs& args, const Plan& plan, cudaStream_t s, int64_t* n_clusters) {
-  const bool hold = plan.slice * static_cast<int64_t>(sizeof(T)) / 16 <= int64_t(kHoldVecs) * kConsumerWarps * 32;
-  if (hold)
-    return ent ? launch_rows<T, true, kHoldVecs>(args, plan, s, n_clusters)
-               : launch_rows<T, false, kHoldVecs>(args, plan, s, n_clusters);
-  return ent ? launch_rows<T, true, 0>(args, plan, s, n_clusters) : launch_rows<T, false, 0>(args, plan, s, n_clusters);
+static rl_status dispatch_loss(bool ent, RowArgs args, int64_t V, cudaStream_t s, int64_t* n_clusters) {
+  auto run = [&](const Plan& plan, auto launcher) {
+    args.slice = plan.slice;
+    args.buf_elems = plan.buf_elems;
+    return launcher(args, plan, s, n_clusters);
+  };
+  const Plan plan = loss_plan<T>(V, ent);
+  const int64_t vecs_per_slice = plan.slice * static_cast<int64_t>(sizeof(T)) / 16;
+  if constexpr (sizeof(T) == 2) {
+    if (!ent && vecs_per_slice <= 10 * 8 * 32) return run(plan, launch_rows<T, 8, false, 10, 2>);
+    if (ent && vecs_per_slice <= 11 * 7 * 32) return run(plan, launch_rows<T, 7, true, 11, 2>);
+  } else {
+    if (vecs_per_slice <= 9 * 7 * 32)
+      return ent ? run(plan, launch_rows<T, 7, true, 9, 3>) : run(plan, launch_rows<T, 7, false, 9, 3>);
+  }
+  Plan big;
+  make_plan(V, static_cast<int>(sizeof(T)), &big);
+  return ent ? run(big, launch_rows<T, 7, true, 0, 2>) : run(big, launch_rows<T, 7, false, 0, 2>);
 }
 
 constexpr int kFwdWarps = 8;
@@ -1191,13 +1227,11 @@ extern "C" rl_status rl_policy_loss_fwd_bwd(const void* logits, rl_dtype dtype, 
   a.done = reinterpret_cast<uint32_t*>(static_cast<char*>(ws) + kWsDoneOffset);
   a.token_stats = token_stats;
   a.status = reinterpret_cast<int32_t*>(ws);
-  a.slice = plan.slice;
-  a.buf_elems = plan.buf_elems;
   a.tma = ((ld * es) % 16) == 0;
   const bool ent = params->entropy_coef != 0.f || token_stats != nullptr;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   int64_t n_clusters = 0;
-  st = dtype == RL_BF16 ? dispatch_loss<uint16_t>(ent, a, plan, s, &n_clusters)
-                        : dispatch_loss<float>(ent, a, plan, s, &n_clusters);
+  st = dtype == RL_BF16 ? dispatch_loss<uint16_t>(ent, a, V, s, &n_clusters)
+                        : dispatch_loss<float>(ent, a, V, s, &n_clusters);
   return st;  // the kernel's last cluster has added the loss into loss_accum
 }
