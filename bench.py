@@ -1103,6 +1103,51 @@ def profile_case(rows, workload="multiturn"):
     return 0 if word == 0 else 1
 
 
+def profile_segments(reps=3):
+    """The segmented reductions alone, for profiler captures (a few MB on the device): `reps`
+    calls of rl_group_advantages on the multi-turn batch's layout (traj_count_kernel,
+    group_adv_kernel), then on the tree workload's packed stream rl_group_advantages_by_owner
+    (owner_count_kernel, group_adv_kernel) and rl_sequence_is_weights (owner_logratio_kernel,
+    seq_weight_kernel; log-probs N(-2, 1) per token, rollout = old + N(0, 0.02^2))."""
+    import torch
+
+    from paper_2608_16798_gb300 import build as B
+
+    B.build()
+    import paper_2608_16798_gb300.rl_loss as R
+
+    dev = torch.device("cuda", 0)
+    t = torch
+    d = lambda x: t.from_numpy(np.ascontiguousarray(x)).to(dev)  # noqa: E731
+    lay = W.make_layout(WORKLOAD, 0)
+    params = R.make_params(W.CLIP_EPS_LOW, W.CLIP_EPS_HIGH, 0.0, 0, 0.0, 0.0, 1e-6, 0)
+    ws = R.new_workspace(0, 0, device=dev)
+    go, rw, to, mask, valid = (d(lay.group_offsets), d(lay.rewards), d(lay.traj_offsets), d(lay.mask),
+                               d(lay.traj_valid))
+    for _ in range(reps):
+        R.rl_group_advantages(go, rw, to, mask, params, ws, traj_valid=valid)
+    w = W.WORKLOADS["tree"]
+    prompts, calls, aux = W.tree_rollouts(w, seed=0)
+    out = R.rl_prefix_tree_build_batch(prompts, calls, aux, max_leaves=w.tree_max_leaves, n_threads=4)
+    n = len(prompts)
+    owner, tmask = d(out["owner"]), d(out["mask"])
+    T = len(out["tokens"])
+    tgo = d(np.arange(0, n + 1, w.group_size, dtype=np.int32))
+    trw = d((np.random.default_rng(0).random(n) < w.reward_p).astype(np.float32))
+    tvalid = d(np.array([st["valid"] for st in out["stats"]], np.uint8))
+    old_h = np.random.default_rng(1).normal(-2.0, 1.0, T).astype(np.float32)
+    old, roll = d(old_h), d(W.rollout_logp_from(old_h, 0, std=0.02))
+    for _ in range(reps):
+        R.rl_group_advantages_by_owner(tgo, trw, owner, tmask, params, ws, traj_valid=tvalid)
+    ws_tree = R.new_workspace(n, 0, device=dev)
+    for _ in range(reps):
+        R.rl_sequence_is_weights(owner, tmask, old, roll, n, ws_tree, cap=2.0)
+    word = R.rl_query_status(ws)[1] | R.rl_query_status(ws_tree)[1]
+    print(json.dumps({"profile_segments": reps, "multiturn_tokens": lay.n_tokens, "multiturn_traj": lay.n_traj,
+                      "tree_tokens": T, "tree_rollouts": n, "status": word}))
+    return 0 if word == 0 else 1
+
+
 def profile_ppo(steps):
     """The PPO step of the benchmark on the whole multi-turn batch, `steps` times without timing
     (for a profiler's launch list): advantages and coefficients, masked GAE, then per microbatch
@@ -1161,6 +1206,8 @@ def main():
                     help="workload of --profile-case (default: the benchmark's multiturn)")
     ap.add_argument("--profile-head", type=int, default=0, metavar="TOKENS",
                     help="run a small fused-head case for a profiler capture and exit")
+    ap.add_argument("--profile-segments", action="store_true",
+                    help="run the segmented-reduction kernels alone (a few MB) for a profiler capture and exit")
     ap.add_argument("--profile-ppo", type=int, default=0, metavar="STEPS",
                     help="run the PPO step on the batch STEPS times for a profiler's launch list and exit")
     ap.add_argument("--no-head", action="store_true", help="skip the fused-head measurement")
@@ -1174,6 +1221,8 @@ def main():
         return profile_head(args.profile_head)
     if args.profile_ppo:
         return profile_ppo(args.profile_ppo)
+    if args.profile_segments:
+        return profile_segments()
     if args.impl == "reference":
         return run_reference(args)
     args.warmup = max(3, args.warmup)
