@@ -127,6 +127,17 @@ __device__ __forceinline__ bool mbar_wait_sleep_bounded(uint64_t* bar, uint32_t 
   }
 }
 
+// The cluster-scope acquire form of mbar_try_wait_sleep / mbar_wait_sleep_bounded.
+__device__ __forceinline__ bool mbar_try_wait_cluster_sleep(uint64_t* bar, uint32_t parity, uint32_t hint_ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok) : "r"(smem_addr(bar)), "r"(parity), "r"(hint_ns) : "memory");
+  return ok != 0;
+}
+
 // Wait with cluster-scope acquire (data written into this CTA by peers with st.async).
 __device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
