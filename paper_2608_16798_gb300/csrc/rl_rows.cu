@@ -94,7 +94,11 @@ struct Vec<uint16_t> {  // bf16
     v[4] = bf16_lo(w.z); v[5] = bf16_hi(w.z); v[6] = bf16_lo(w.w); v[7] = bf16_hi(w.w);
   }
   static constexpr int NP = 4;  // float2 pairs per 16-byte vector
-  static constexpr uint32_t kPadWord = 0xFF7FFF7Fu;  // two most-negative finite bf16 values
+  // pad of register-held vectors past the slice: two bf16 values of about -1.5e38, at or below
+  // -1e38 (so they count as -inf for the maximum) yet far enough from -FLT_MAX that
+  // z log2(e) - m log2(e) stays finite: its exponential is 0 and, with the entropy on, e x is
+  // 0, not 0 x -inf = NaN (which would send every thread holding a pad down the slow path)
+  static constexpr uint32_t kPadWord = 0xFEE1FEE1u;
   static __device__ __forceinline__ void pairs(const uint4 w, float2 (&q)[4]) {
     q[0] = make_float2(bf16_lo(w.x), bf16_hi(w.x)); q[1] = make_float2(bf16_lo(w.y), bf16_hi(w.y));
     q[2] = make_float2(bf16_lo(w.z), bf16_hi(w.z)); q[3] = make_float2(bf16_lo(w.w), bf16_hi(w.w));
@@ -124,7 +128,7 @@ struct Vec<float> {
     v[0] = w.x; v[1] = w.y; v[2] = w.z; v[3] = w.w;
   }
   static constexpr int NP = 2;
-  static constexpr uint32_t kPadWord = 0xFF7FFFFFu;  // most-negative finite float
+  static constexpr uint32_t kPadWord = 0xFEE1B1E6u;  // -1.5e38: see Vec<uint16_t>::kPadWord
   static __device__ __forceinline__ void pairs(const uint4 w, float2 (&q)[2]) {
     q[0] = make_float2(__uint_as_float(w.x), __uint_as_float(w.y));
     q[1] = make_float2(__uint_as_float(w.z), __uint_as_float(w.w));
@@ -265,7 +269,7 @@ __device__ __forceinline__ void fold(SoftmaxPartial& ps, const float (&v)[EPV]) 
 }
 
 // Fold NV register-held 16-byte vectors into a partial, branch-free in the common
-// case. Vectors past the end of the data hold T's most-negative finite value, whose
+// case. Vectors past the end of the data hold about -1.5e38 (Vec<T>::kPadWord), whose
 // exponential is exactly 0. The reference is the partial's own maximum or, for a
 // fresh partial, the first vector's maximum; when the exponentials sum above 1e30
 // (a value far above the reference) everything is redone against the exact
@@ -1034,11 +1038,16 @@ static rl_status launch_rows(const RowArgs& args, const Plan& plan, cudaStream_t
 //     slices up to 40 KB (clusters of 8 at V = 151,936), 2 CTAs per SM: 12.84 ms per benchmark
 //     step against 12.96 with 7 warps of 11 vectors; wider clusters or 3 CTAs per SM were
 //     slower (13.6-18.5 ms);
-//   bf16 with the entropy: 7 warps of 11 vectors, clusters of 8, 2 CTAs per SM: 3.20 ms per
-//     32,768-row long-horizon microbatch, against 3.35-3.71 with 8, 9 or 11 warps and
-//     3.57-4.61 with clusters of 10, 12 or 16 at 3 CTAs per SM;
+//   bf16 with the entropy: the same 8 warps of 10 vectors: 2.72 ms per 32,768-row long-horizon
+//     microbatch, against 2.73 with 7 warps of 11 and 3.16 with 11 warps of 7;
 //   fp32: slices up to 30 KB (clusters of 5 at V = 32,000), 7 warps of up to 9 vectors, 3 CTAs
 //     per SM: 4.15 ms per 131,072-row edge batch against 4.35 with clusters of 4 at 2 per SM.
+#ifndef RL_ENT_NW
+#define RL_ENT_NW 8
+#endif
+#ifndef RL_ENT_HOLD
+#define RL_ENT_HOLD 10
+#endif
 template <typename T>
 struct LossShape;
 template <>
@@ -1074,7 +1083,8 @@ static rl_status dispatch_loss(bool ent, RowArgs args, int64_t V, cudaStream_t s
   const int64_t vecs_per_slice = plan.slice * static_cast<int64_t>(sizeof(T)) / 16;
   if constexpr (sizeof(T) == 2) {
     if (!ent && vecs_per_slice <= 10 * 8 * 32) return run(plan, launch_rows<T, 8, false, 10, 2>);
-    if (ent && vecs_per_slice <= 11 * 7 * 32) return run(plan, launch_rows<T, 7, true, 11, 2>);
+    if (ent && vecs_per_slice <= RL_ENT_HOLD * RL_ENT_NW * 32)
+      return run(plan, launch_rows<T, RL_ENT_NW, true, RL_ENT_HOLD, 2>);
   } else {
     if (vecs_per_slice <= 9 * 7 * 32)
       return ent ? run(plan, launch_rows<T, 7, true, 9, 3>) : run(plan, launch_rows<T, 7, false, 9, 3>);
