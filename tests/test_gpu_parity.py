@@ -281,15 +281,20 @@ def test_end_to_end_advantages_then_loss(R):
 
 # ----------------------------------------------------------------------------- logits at -inf
 
-def neg_inf_case(name, rows, seed=6, entropy=False):
+def neg_inf_case(name, rows, seed=6, entropy=False, fill="-inf"):
     """Rows with vocabulary entries masked to -inf (never the sampled one): 30% of the entries
     in half the rows, all but three entries in one row. old_logp and ref_logp follow from the
-    masked rows' log-probabilities, so the ratio band around the clip bounds still holds."""
+    masked rows' log-probabilities, so the ratio band around the clip bounds still holds.
+    fill="max_finite" masks with the most negative finite value instead (exp of it is 0 too;
+    x = (z - m) log2(e) overflows there, which the kernels must treat like -inf)."""
     c = make_case(name, seed=seed, rows=rows)
     raw = c.raw.copy()
     V = raw.shape[1]
     rng = np.random.default_rng(seed + 100)
-    ninf = np.uint16(0xFF80) if c.w.dtype == "bf16" else np.float32(-np.inf)
+    if fill == "-inf":
+        ninf = np.uint16(0xFF80) if c.w.dtype == "bf16" else np.float32(-np.inf)
+    else:
+        ninf = np.uint16(0xFF7F) if c.w.dtype == "bf16" else np.float32(-np.finfo(np.float32).max)
     for r in range(0, c.rows, 2):
         cols = rng.random(V) < 0.3
         cols[c.ids[r]] = False
@@ -305,18 +310,19 @@ def neg_inf_case(name, rows, seed=6, entropy=False):
     return dataclasses.replace(c, raw=raw, old=old, ref=ref, P=P)
 
 
-@pytest.mark.parametrize("name,entropy", [("longhorizon", False), ("multiturn", True), ("edge", True),
-                                          ("multiturn", False)])
-def test_policy_loss_neg_inf_logits(R, name, entropy):
-    case = neg_inf_case(name, 64, entropy=entropy)
+@pytest.mark.parametrize("name,entropy,fill", [("longhorizon", False, "-inf"), ("multiturn", True, "-inf"),
+                                               ("edge", True, "-inf"), ("multiturn", False, "-inf"),
+                                               ("longhorizon", True, "max_finite"), ("edge", True, "max_finite")])
+def test_policy_loss_neg_inf_logits(R, name, entropy, fill):
+    case = neg_inf_case(name, 64, entropy=entropy, fill=fill)
     out = run_loss(R, case)
-    compare(case, out, f"{name} -inf entries, entropy={entropy}")
+    compare(case, out, f"{name} {fill} entries, entropy={entropy}")
     assert np.isfinite(out["grad"]).all()
 
 
-@pytest.mark.parametrize("name", ["multiturn", "edge"])
-def test_token_logprobs_neg_inf_logits(R, name):
-    case = neg_inf_case(name, 48)
+@pytest.mark.parametrize("name,fill", [("multiturn", "-inf"), ("edge", "-inf"), ("multiturn", "max_finite")])
+def test_token_logprobs_neg_inf_logits(R, name, fill):
+    case = neg_inf_case(name, 48, fill=fill)
     V = case.raw.shape[1]
     ws = R.new_workspace(case.rows, V)
     logp, H, lse = R.rl_token_logprobs(logits_to_dev(case), to_dev(case.ids), ws, want_entropy=True, want_lse=True)
