@@ -1059,13 +1059,12 @@ struct LossShape<float> {
   static constexpr int64_t kSliceBytes[2] = {30 * 1024, 30 * 1024};
 };
 
-// The plan of the loss kernel for this path (the forward-only kernel has no clusters).
+// The plan of the loss kernel for this path (the forward-only kernel has no clusters); false
+// if no cluster of at most 16 CTAs of 100 KB holds the row (the callers check that first).
 template <typename T>
-static Plan loss_plan(int64_t V, bool ent) {
-  Plan plan;
-  if (!make_plan(V, static_cast<int>(sizeof(T)), &plan, LossShape<T>::kSliceBytes[ent ? 1 : 0]))
-    make_plan(V, static_cast<int>(sizeof(T)), &plan);
-  return plan;
+static bool loss_plan(int64_t V, bool ent, Plan* plan) {
+  return make_plan(V, static_cast<int>(sizeof(T)), plan, LossShape<T>::kSliceBytes[ent ? 1 : 0]) ||
+         make_plan(V, static_cast<int>(sizeof(T)), plan);
 }
 
 // Launches the loss kernel; *n_clusters receives the number of clusters, each of which leaves
@@ -1079,7 +1078,8 @@ static rl_status dispatch_loss(bool ent, RowArgs args, int64_t V, cudaStream_t s
     args.buf_elems = plan.buf_elems;
     return launcher(args, plan, s, n_clusters);
   };
-  const Plan plan = loss_plan<T>(V, ent);
+  Plan plan = {};
+  if (!loss_plan<T>(V, ent, &plan)) return set_error(RL_ERR_UNSUPPORTED, "rl_policy_loss_fwd_bwd: row too large");
   const int64_t vecs_per_slice = plan.slice * static_cast<int64_t>(sizeof(T)) / 16;
   if constexpr (sizeof(T) == 2) {
     if (!ent && vecs_per_slice <= 10 * 8 * 32) return run(plan, launch_rows<T, 8, false, 10, 2>);
@@ -1089,8 +1089,9 @@ static rl_status dispatch_loss(bool ent, RowArgs args, int64_t V, cudaStream_t s
     if (vecs_per_slice <= 9 * 7 * 32)
       return ent ? run(plan, launch_rows<T, 7, true, 9, 3>) : run(plan, launch_rows<T, 7, false, 9, 3>);
   }
-  Plan big;
-  make_plan(V, static_cast<int>(sizeof(T)), &big);
+  Plan big = {};
+  if (!make_plan(V, static_cast<int>(sizeof(T)), &big))
+    return set_error(RL_ERR_UNSUPPORTED, "rl_policy_loss_fwd_bwd: row too large");
   return ent ? run(big, launch_rows<T, 7, true, 0, 2>) : run(big, launch_rows<T, 7, false, 0, 2>);
 }
 
