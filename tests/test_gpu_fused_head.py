@@ -135,12 +135,12 @@ def test_fused_head_parity(R, T, D, V, agg, ent, tis):
     compare_head(c, out)
 
 
-@pytest.mark.parametrize("group_tokens", [0, 3 * 4096])
+@pytest.mark.parametrize("group_tokens", [0, 6000, 3 * 4096])
 def test_fused_head_three_chunks_bf16_grad(R, group_tokens):
     """More than 8,192 tokens, bf16 d_hidden. With the smallest workspace each chunk of 4,096 is
-    its own group: dH's contraction over V is split in two halves added in fp32 in the
-    workspace, then rounded to bf16, and dW is added three times. With room for three chunks
-    the group holds them all: dH is stored directly in bf16 and dW is added once."""
+    its own group and dW is added three times; with room for two chunks (6,000 tokens round up
+    to two) the groups are two chunks and a ragged last one; with room for three the group
+    holds them all and dW is added once."""
     c = make_head_case(8192 + 77, 128, 1100, seed=5, agg=2)
     out = run_head(R, c, dh_dtype=torch.bfloat16, group_tokens=group_tokens)
     compare_head(c, out, dh_bf16=True)
