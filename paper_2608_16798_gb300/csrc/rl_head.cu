@@ -329,6 +329,234 @@ __global__ void __launch_bounds__(kThreads, 1) head_kernel(const __grid_constant
   }
 }
 
+// ------------------------------------------------------------------ 256 x 512 tiles
+//
+// Wide form of the pair kernel: a CTA pair computes 256 tokens x 512 vocabulary entries per
+// tile with two cta_group::2 MMAs per K step that share the H operand, into one accumulator of
+// all 512 TMEM columns (4 stages of 48 KB: this CTA's 128 tokens of H and, per MMA, its 128
+// of the 256 W rows). The epilogue treats the tile as two 256-column halves with the same two
+// sweeps as the 256 x 256 form (so the tile maxima keep their 256-column granularity), but it
+// cannot overlap the next tile's MMAs: the single accumulator is handed back after both halves.
+constexpr uint32_t W_HALF = (BN / 2) * BK * 2;          // 16 KB
+constexpr uint32_t STAGEW_BYTES = A_BYTES + 2 * W_HALF;  // 48 KB
+constexpr int NSW = 4;
+constexpr size_t kSmemW = NSW * STAGEW_BYTES + 1024;
+
+// One 256-column half of a tile's epilogue: the row maximum of the valid columns and the
+// sampled id's logit (za), then e = exp(z - m), its sums and (STATS_P) e in bf16 at `out`.
+template <int MODE>
+__device__ __forceinline__ SoftmaxPartial epi_half(uint32_t tacc, int n0, int V, int32_t a, int ent, uint16_t* out,
+                                                   float& za, float& tm_out) {
+  const float kNegInf = -__int_as_float(0x7f800000);
+  float tm = kNegInf;
+#pragma unroll 1
+  for (int c = 0; c < BN; c += 32) {
+    const int col0 = n0 + c;
+    const int nvalid = min(32, V - col0);
+    if (nvalid <= 0) break;  // past the vocabulary (uniform across the warp)
+    float v[32];
+    tc::tmem_ld32(tacc + c, v);
+#pragma unroll
+    for (int j = 0; j < 32; ++j)
+      if (j < nvalid) tm = fmaxf(tm, v[j]);
+    const int ja = a - col0;
+    if (ja >= 0 && ja < 32) {
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (j == ja) za = v[j];
+    }
+  }
+  const float nm = -tm * kLog2e;
+  float s0 = 0.f, s1 = 0.f, u0 = 0.f;
+#pragma unroll 1
+  for (int c = 0; c < BN; c += 32) {
+    const int col0 = n0 + c;
+    const int nvalid = min(32, V - col0);
+    if (nvalid <= 0) break;
+    float v[32];
+    tc::tmem_ld32(tacc + c, v);
+    uint32_t w[16];
+#pragma unroll
+    for (int j = 0; j < 32; j += 2) {
+      float e2[2];
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const bool in = j + h < nvalid;
+        const float z = in ? v[j + h] : tm;
+        const float e = in ? ex2(fmaf(z, kLog2e, nm)) : 0.f;
+        if (h) s1 += e; else s0 += e;
+        if (ent) u0 = fmaf(e, z - tm, u0);
+        e2[h] = e;
+      }
+      w[j / 2] = pack_bf16x2(e2[0], e2[1]);
+    }
+    if (MODE == STATS_P && out) {
+      uint16_t* o = out + c;
+      if (nvalid == 32) {
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          *reinterpret_cast<uint4*>(o + 8 * j) = make_uint4(w[4 * j], w[4 * j + 1], w[4 * j + 2], w[4 * j + 3]);
+      } else {
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          if (j < nvalid) o[j] = static_cast<uint16_t>((w[j / 2] >> (16 * (j & 1))) & 0xFFFFu);
+      }
+    }
+  }
+  tm_out = tm;
+  return SoftmaxPartial{tm, s0 + s1, u0};
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(kThreads, 1) head_wide_kernel(const __grid_constant__ CUtensorMap tmH,
+                                                                const __grid_constant__ CUtensorMap tmW,
+                                                                const HeadArgs p) {
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t full[NSW], empty[NSW], accf, acce;
+  __shared__ uint32_t tbase;
+  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  const int unit = static_cast<int>(blockIdx.x >> 1);
+  const int n_units = static_cast<int>(gridDim.x >> 1);
+  constexpr int VB2 = VB_TILES / 2;  // 512-column tiles per vocabulary block
+  const int n_m = (p.Tc + 2 * BM - 1) / (2 * BM);
+  const int n_nt2 = (p.n_nt + 1) / 2;
+  const int n_items = n_m * p.n_vb;
+  const int nkb = p.D / BK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < NSW; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(&accf, 1);
+    mbar_init(&acce, 8);
+    fence_mbar_init();
+  }
+  if (warp == 1) tc::tmem_alloc_pair(&tbase, 2 * BN);
+  tc::fence_before_sync();
+  cluster_sync_all();
+  tc::fence_after_sync();
+  const uint32_t tmem = tbase;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      uint32_t g = 0;
+      bool ok = true;
+      for (int item = unit; item < n_items && ok; item += n_units) {
+        const int vb = item / n_m, m0 = (item % n_m) * 2 * BM + static_cast<int>(rank) * BM;
+        const int nt1 = min((vb + 1) * VB2, n_nt2);
+        for (int nt = vb * VB2; nt < nt1 && ok; ++nt) {
+          for (int kb = 0; kb < nkb; ++kb, ++g) {
+            const int s = g % NSW;
+            const uint32_t use = g / NSW;
+            if (use > 0 && !mbar_wait_bounded(&empty[s], (use - 1) & 1)) {
+              flag_status(p.status, RL_DEV_TIMEOUT);
+              ok = false;
+              break;
+            }
+            uint8_t* st = sm + s * STAGEW_BYTES;
+            if (rank == 0) mbar_arrive_expect_tx(&full[s], 2 * STAGEW_BYTES);  // both CTAs' bytes
+            const uint32_t bar = map_to_rank(smem_addr(&full[s]), 0);
+            tc::tma_load_2d_pair(st, &tmH, kb * BK, m0, bar);
+#pragma unroll
+            for (int h = 0; h < 2; ++h)
+              tc::tma_load_2d_pair(st + A_BYTES + h * W_HALF, &tmW, kb * BK,
+                                   nt * 2 * BN + h * BN + static_cast<int>(rank) * (BN / 2), bar);
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && rank == 0) {
+      constexpr uint32_t idesc = tc::idesc_bf16_f32(2 * BM, BN);
+      uint32_t g = 0, t = 0;
+      bool ok = true;
+      for (int item = unit; item < n_items && ok; item += n_units) {
+        const int vb = item / n_m;
+        const int nt1 = min((vb + 1) * VB2, n_nt2);
+        for (int nt = vb * VB2; nt < nt1 && ok; ++nt, ++t) {
+          if (t > 0 && !mbar_wait_cluster_bounded(&acce, (t - 1) & 1)) {
+            flag_status(p.status, RL_DEV_TIMEOUT);
+            ok = false;
+            break;
+          }
+          tc::fence_after_sync();
+          for (int kb = 0; kb < nkb; ++kb, ++g) {
+            const int s = g % NSW;
+            if (!mbar_wait_bounded(&full[s], (g / NSW) & 1)) {
+              flag_status(p.status, RL_DEV_TIMEOUT);
+              ok = false;
+              break;
+            }
+            tc::fence_after_sync();
+            const uint32_t a = smem_addr(sm + s * STAGEW_BYTES), b = a + A_BYTES;
+#pragma unroll
+            for (int k = 0; k < BK / 16; ++k) {
+              const uint64_t ad = tc::desc_kmajor_sw128(a + k * 32);
+#pragma unroll
+              for (int h = 0; h < 2; ++h)
+                tc::mma_bf16_pair(tmem + h * BN, ad, tc::desc_kmajor_sw128(b + h * W_HALF + k * 32), idesc,
+                                  (kb | k) != 0);
+            }
+            tc::mma_commit_pair(&empty[s], 0x3);
+          }
+          if (ok) tc::mma_commit_pair(&accf, 0x3);
+        }
+      }
+    }
+  } else {
+    const int q = warp & 3;
+    const int rl = 32 * q + lane;
+    const float kNegInf = -__int_as_float(0x7f800000);
+    const uint32_t tq = tmem + (static_cast<uint32_t>(32 * q) << 16);
+    uint32_t t = 0;
+    bool ok = true;
+    for (int item = unit; item < n_items && ok; item += n_units) {
+      const int vb = item / n_m, m0 = (item % n_m) * 2 * BM + static_cast<int>(rank) * BM;
+      const int r = m0 + rl;
+      const bool row_ok = r < p.Tc;
+      const int nt1 = min((vb + 1) * VB2, n_nt2);
+      SoftmaxPartial ps{kNegInf, 0.f, 0.f};
+      float za = 0.f;
+      const int32_t a = row_ok ? p.token_ids[p.t0 + r] : -1;
+      uint16_t* dz_row = (MODE == STATS_P && row_ok) ? p.dz + static_cast<int64_t>(r) * p.ldz : nullptr;
+      for (int nt = vb * VB2; nt < nt1; ++nt, ++t) {
+        if (!mbar_wait_sleep_bounded(&accf, t & 1)) {
+          if (lane == 0) flag_status(p.status, RL_DEV_TIMEOUT);
+          ok = false;
+          break;
+        }
+        tc::fence_after_sync();
+#pragma unroll 1
+        for (int h = 0; h < 2; ++h) {
+          const int j = nt * 2 + h;  // 256-column tile
+          if (j >= p.n_nt) break;
+          float tm;
+          const SoftmaxPartial half =
+              epi_half<MODE>(tq + h * BN, j * BN, p.V, a, p.ent, dz_row ? dz_row + j * BN : nullptr, za, tm);
+          if (MODE == STATS_P && row_ok) p.tmax[static_cast<int64_t>(r) * p.n_nt + j] = tm;
+          ps = merge(ps, half);
+        }
+        tc::fence_before_sync();
+        __syncwarp();
+        if (lane == 0) {
+          if (rank != 0) mbar_arrive_remote(map_to_rank(smem_addr(&acce), 0));
+          else mbar_arrive(&acce);
+        }
+      }
+      if (ok && row_ok) p.partials[static_cast<int64_t>(vb) * p.Tc + r] = make_float4(ps.m, ps.s, ps.u, za);
+    }
+  }
+  tc::fence_before_sync();
+  cluster_sync_all();
+  if (warp == 1) {
+    tc::fence_after_sync();
+    tc::tmem_dealloc_pair(tmem, 2 * BN);
+  }
+}
+
 struct MergeArgs {
   int64_t t0;
   int32_t Tc, V, n_vb, n_traj;
@@ -569,10 +797,20 @@ static Layout layout(int64_t max_rows, int64_t V, size_t ws_bytes = 0, int64_t w
   return L;
 }
 
+// Which passes use the 256 x 512 form: bit 0 the forward-only statistics (STATS), bit 1 the
+// loss call's statistics pass (STATS_P). Measured at 32,768 x 4,096 x 151,936 (back to back,
+// same box): the forward-only call 24.24-24.36 ms wide against 24.81 ms with 256 x 256 tiles;
+// the loss call 71.5-72.1 ms either way (its heavier epilogue, which stores the exponentials,
+// is hidden behind the MMAs only with two accumulators).
+#ifndef RL_HEAD_WIDE
+#define RL_HEAD_WIDE 1
+#endif
+
 template <int MODE>
 static rl_status launch_head(const CUtensorMap& mh, const CUtensorMap& mw, const HeadArgs& a, cudaStream_t s) {
-  auto kern = head_kernel<MODE, kPair>;
-  constexpr size_t smem = kPair ? kSmem2 : kSmem;
+  constexpr bool kWide = ((RL_HEAD_WIDE >> MODE) & 1) != 0;
+  auto kern = kWide ? head_wide_kernel<MODE> : head_kernel<MODE, kPair>;
+  constexpr size_t smem = kWide ? kSmemW : (kPair ? kSmem2 : kSmem);
   int dev = 0, sms = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
@@ -599,7 +837,7 @@ static rl_status launch_head(const CUtensorMap& mh, const CUtensorMap& mw, const
       e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
       if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(head_kernel)");
       int n = sms;
-      if constexpr (kPair) {
+      if constexpr (kPair || kWide) {
         cfg.gridDim = dim3(2);
         e = cudaOccupancyMaxActiveClusters(&n, kern, &cfg);
         if (e != cudaSuccess) return cuda_error(e, "cudaOccupancyMaxActiveClusters(head_kernel)");
@@ -609,7 +847,7 @@ static rl_status launch_head(const CUtensorMap& mh, const CUtensorMap& mw, const
     }
     max_pairs = it->second;
   }
-  if constexpr (kPair) {
+  if constexpr (kPair || kWide) {
     // persistent: one 2-CTA cluster per resident pair, work items of 256 tokens x one vocabulary block
     const int items = (a.Tc + 2 * BM - 1) / (2 * BM) * a.n_vb;
     const int pairs = std::max(1, std::min(items, max_pairs));
