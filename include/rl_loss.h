@@ -455,8 +455,9 @@ rl_status rl_sequence_is_weights(int32_t n_traj, int64_t n_tokens, const int32_t
  *   entropy_out  float [T] or NULL (entropy work is skipped when NULL)
  *   lse_out      float [T] or NULL
  *   ws, ws_bytes workspace; rl_workspace_size(T, V, D) bytes always suffice (the
- *                call uses the status word and 16 * ceil(V / 4096) * min(T, 4096)
- *                bytes of per-block softmax partials after it)
+ *                call uses the status word and 32 * ceil(V / 4096) * min(T, 4096)
+ *                bytes of softmax partials after it: two per token and 4,096-entry
+ *                vocabulary block)
  * One tensor-core pass per chunk of 4,096 tokens, then a per-token merge of the
  * vocabulary blocks' partials in fixed order (deterministic).
  */

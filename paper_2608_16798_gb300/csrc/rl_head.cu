@@ -8,7 +8,7 @@
 //      holds 128 of the tile's tokens). The epilogue reads each tile twice from TMEM: first
 //      its row maximum m_j, then e = exp(z - m_j), which it stores (bf16) in the chunk's
 //      dZ buffer, with m_j per token and tile, and folds into per-row online-softmax
-//      partials for its vocabulary block.
+//      partials: two per vocabulary block (its even and its odd tiles).
 //   2. head_merge_kernel    one thread per token: merges the partials into lse, entropy and
 //      logp, evaluates the objective's per-token terms (same readings as the logits path),
 //      writes the row's loss contribution and the coefficients of dZ.
@@ -23,7 +23,8 @@
 //      operands in their row-major layouts (dZ K-major for dH, MN-major for dW; W and H
 //      MN-major), dH tiles first and dW tiles after them, handed out by a work counter; dH is
 //      stored, dW added in fp32 by TMA reduce-add, once per group.
-// The forward-only call runs head_kernel<STATS> (no stores) and head_logp_merge_kernel.
+// The forward-only call runs head_wide_kernel<STATS> (256 x 512 tiles, no stores; the same two
+// partials per block) and head_logp_merge_kernel.
 // The objective (Sec. 2.3.2, Sec. 3.2.4) is the same as for rl_policy_loss_fwd_bwd; here
 // pi_theta's logits come from the hidden states times the vocabulary projection.
 #include <cuda.h>
@@ -68,6 +69,7 @@ constexpr uint32_t kWBoxRows = kPair ? BN / 2 : BN;  // rows of W per TMA box
 #define RL_HEAD_CHUNK 4096
 #endif
 constexpr int64_t kChunk = RL_HEAD_CHUNK;  // tokens per chunk (tuning knob, compile time)
+constexpr int64_t kParts = 2;               // partials per token and vocabulary block (even, odd tiles)
 
 enum Mode { STATS = 0, STATS_P = 1 };
 
@@ -88,7 +90,7 @@ struct HeadArgs {
   int32_t Tc, D, V, n_mt, n_vb, n_nt;
   int32_t ent;
   const int32_t* token_ids;
-  float4* partials;        // [n_vb][Tc] (m, s, u, z_a)
+  float4* partials;        // [2 n_vb][Tc] (m, s, u, z_a): a block's even tiles, then its odd tiles
   uint16_t* dz;            // [Tc x ldz] bf16: e = exp(z - m_j) (STATS_P)
   int64_t ldz;
   float* tmax;             // [Tc x n_nt]: m_j per token and tile (STATS_P)
@@ -237,7 +239,8 @@ __global__ void __launch_bounds__(kThreads, 1) head_kernel(const __grid_constant
       const int r = m0 + rl;  // token within the chunk
       const bool row_ok = r < p.Tc;
       const int nt1 = min((vb + 1) * VB_TILES, p.n_nt);
-      SoftmaxPartial ps{kNegInf, 0.f, 0.f};
+      // running partials of the block's even and odd tiles (the halves of its 256 x 512 tiles)
+      SoftmaxPartial ps0{kNegInf, 0.f, 0.f}, ps1{kNegInf, 0.f, 0.f};
       float za = 0.f;
       const int32_t a = row_ok ? p.token_ids[p.t0 + r] : -1;
       for (int nt = vb * VB_TILES; nt < nt1; ++nt, ++t) {
@@ -314,9 +317,14 @@ __global__ void __launch_bounds__(kThreads, 1) head_kernel(const __grid_constant
           else mbar_arrive(&acce[acc]);
         }
         if (MODE == STATS_P && row_ok) p.tmax[static_cast<int64_t>(r) * p.n_nt + nt] = tm;
-        ps = merge(ps, SoftmaxPartial{tm, s0 + s1, u0});
+        const SoftmaxPartial tile{tm, s0 + s1, u0};
+        if (nt & 1) ps1 = merge(ps1, tile);
+        else ps0 = merge(ps0, tile);
       }
-      if (ok && row_ok) p.partials[static_cast<int64_t>(vb) * p.Tc + r] = make_float4(ps.m, ps.s, ps.u, za);
+      if (ok && row_ok) {
+        p.partials[static_cast<int64_t>(2 * vb) * p.Tc + r] = make_float4(ps0.m, ps0.s, ps0.u, za);
+        p.partials[static_cast<int64_t>(2 * vb + 1) * p.Tc + r] = make_float4(ps1.m, ps1.s, ps1.u, 0.f);
+      }
     }
   }
   tc::fence_before_sync();
@@ -335,8 +343,11 @@ __global__ void __launch_bounds__(kThreads, 1) head_kernel(const __grid_constant
 // tile with two cta_group::2 MMAs per K step that share the H operand, into one accumulator of
 // all 512 TMEM columns (4 stages of 48 KB: this CTA's 128 tokens of H and, per MMA, its 128
 // of the 256 W rows). The epilogue treats the tile as two 256-column halves with the same two
-// sweeps as the 256 x 256 form (so the tile maxima keep their 256-column granularity), but it
-// cannot overlap the next tile's MMAs: the single accumulator is handed back after both halves.
+// sweeps as the 256 x 256 form (so the tile maxima keep their 256-column granularity), one
+// group of four warps per half, each with its own partial (the block's even or odd tiles, as
+// in the 256 x 256 form, so both forms give the same bits). It cannot overlap the next
+// tile's MMAs: the single accumulator is handed back after both halves; the second group
+// halves the time that takes.
 constexpr uint32_t W_HALF = (BN / 2) * BK * 2;          // 16 KB
 constexpr uint32_t STAGEW_BYTES = A_BYTES + 2 * W_HALF;  // 48 KB
 constexpr int NSW = 4;
@@ -407,8 +418,12 @@ __device__ __forceinline__ SoftmaxPartial epi_half(uint32_t tacc, int n0, int V,
   return SoftmaxPartial{tm, s0 + s1, u0};
 }
 
+// warp 0 TMA, warp 1 MMA, warps 2-9 epilogue: warps 2-5 read the tile's first 256 columns and
+// warps 6-9 its second 256, each group with its own running partial (two per vocabulary block)
+constexpr int kThreadsW = 320;
+
 template <int MODE>
-__global__ void __launch_bounds__(kThreads, 1) head_wide_kernel(const __grid_constant__ CUtensorMap tmH,
+__global__ void __launch_bounds__(kThreadsW, 1) head_wide_kernel(const __grid_constant__ CUtensorMap tmH,
                                                                 const __grid_constant__ CUtensorMap tmW,
                                                                 const HeadArgs p) {
   extern __shared__ uint8_t smem_raw[];
@@ -431,7 +446,7 @@ __global__ void __launch_bounds__(kThreads, 1) head_wide_kernel(const __grid_con
       mbar_init(&empty[s], 1);
     }
     mbar_init(&accf, 1);
-    mbar_init(&acce, 8);
+    mbar_init(&acce, 16);  // 8 epilogue warps in each CTA of the pair
     fence_mbar_init();
   }
   if (warp == 1) tc::tmem_alloc_pair(&tbase, 2 * BN);
@@ -507,7 +522,8 @@ __global__ void __launch_bounds__(kThreads, 1) head_wide_kernel(const __grid_con
       }
     }
   } else {
-    const int q = warp & 3;
+    const int q = warp & 3;            // TMEM lane quarter this warp may access
+    const int h = (warp - 2) >> 2;     // the 256-column half of each tile this warp reads
     const int rl = 32 * q + lane;
     const float kNegInf = -__int_as_float(0x7f800000);
     const uint32_t tq = tmem + (static_cast<uint32_t>(32 * q) << 16);
@@ -529,10 +545,8 @@ __global__ void __launch_bounds__(kThreads, 1) head_wide_kernel(const __grid_con
           break;
         }
         tc::fence_after_sync();
-#pragma unroll 1
-        for (int h = 0; h < 2; ++h) {
-          const int j = nt * 2 + h;  // 256-column tile
-          if (j >= p.n_nt) break;
+        const int j = nt * 2 + h;  // 256-column tile
+        if (j < p.n_nt) {
           float tm;
           const SoftmaxPartial half =
               epi_half<MODE>(tq + h * BN, j * BN, p.V, a, p.ent, dz_row ? dz_row + j * BN : nullptr, za, tm);
@@ -546,7 +560,8 @@ __global__ void __launch_bounds__(kThreads, 1) head_wide_kernel(const __grid_con
           else mbar_arrive(&acce);
         }
       }
-      if (ok && row_ok) p.partials[static_cast<int64_t>(vb) * p.Tc + r] = make_float4(ps.m, ps.s, ps.u, za);
+      if (ok && row_ok)
+        p.partials[static_cast<int64_t>(2 * vb + h) * p.Tc + r] = make_float4(ps.m, ps.s, ps.u, za);
     }
   }
   tc::fence_before_sync();
@@ -559,7 +574,7 @@ __global__ void __launch_bounds__(kThreads, 1) head_wide_kernel(const __grid_con
 
 struct MergeArgs {
   int64_t t0;
-  int32_t Tc, V, n_vb, n_traj;
+  int32_t Tc, V, n_part, n_traj;  // n_part partials per token (two per vocabulary block)
   const float4* partials;
   const int32_t* token_ids;
   const uint8_t* mask;
@@ -610,7 +625,7 @@ __global__ void __launch_bounds__(256) head_merge_kernel(const MergeArgs p) {
   }
   SoftmaxPartial q{-__int_as_float(0x7f800000), 0.f, 0.f};
   float za = 0.f;
-  for (int b = 0; b < p.n_vb; ++b) {
+  for (int b = 0; b < p.n_part; ++b) {
     const float4 w = p.partials[static_cast<int64_t>(b) * p.Tc + r];
     q = merge(q, SoftmaxPartial{w.x, w.y, w.z});
     za += w.w;
@@ -722,7 +737,7 @@ __global__ void __launch_bounds__(kDzThreads) head_dz_kernel(const DzArgs p) {
 
 struct LogpMergeArgs {
   int64_t t0;
-  int32_t Tc, V, n_vb;
+  int32_t Tc, V, n_part;  // n_part partials per token (two per vocabulary block)
   const float4* partials;
   const int32_t* token_ids;
   float* logp_out;
@@ -738,10 +753,10 @@ __global__ void __launch_bounds__(256) head_logp_merge_kernel(const LogpMergeArg
   const int64_t t = p.t0 + r;
   SoftmaxPartial q{-__int_as_float(0x7f800000), 0.f, 0.f};
   float za = 0.f;
-  for (int b = 0; b < p.n_vb; ++b) {
+  for (int b = 0; b < p.n_part; ++b) {
     const float4 w = p.partials[static_cast<int64_t>(b) * p.Tc + r];
     q = merge(q, SoftmaxPartial{w.x, w.y, w.z});
-    za += w.w;  // nonzero in the one block that holds the sampled id
+    za += w.w;  // nonzero in the one partial whose columns hold the sampled id
   }
   const float lnS = logf(q.s);
   const float lse = q.m + lnS;
@@ -782,7 +797,7 @@ static Layout layout(int64_t max_rows, int64_t V, size_t ws_bytes = 0, int64_t w
   auto al = al256;
   size_t off = kWsHeader + al(static_cast<size_t>(std::max<int64_t>(max_rows, 0)) * sizeof(double));
   L.off_partials = off;
-  off += al(static_cast<size_t>(L.n_vb * L.Tc) * sizeof(float4));
+  off += al(static_cast<size_t>(kParts * L.n_vb * L.Tc) * sizeof(float4));
   L.off_rc = off;
   off += al(static_cast<size_t>(L.Tc) * sizeof(RowCoef));
   L.off_tmax = off;
@@ -821,7 +836,7 @@ static rl_status launch_head(const CUtensorMap& mh, const CUtensorMap& mw, const
   attr[0].val.clusterDim.x = 2;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
-  cfg.blockDim = dim3(kThreads);
+  cfg.blockDim = dim3(kWide ? kThreadsW : kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cfg.attrs = attr;
@@ -885,7 +900,7 @@ size_t head_workspace_bytes_grouped(int64_t max_rows, int64_t V, int64_t D, int6
 // hidden states (256 MB) then evict W's tiles from the 129 MB L2.
 static size_t head_logp_workspace_bytes(int64_t T, int64_t V) {
   const head::Layout L = head::layout(T, V);
-  return kWsHeader + head::al256(static_cast<size_t>(L.n_vb * L.Tc) * sizeof(float4));
+  return kWsHeader + head::al256(static_cast<size_t>(head::kParts * L.n_vb * L.Tc) * sizeof(float4));
 }
 
 }  // namespace rl
@@ -970,7 +985,7 @@ extern "C" rl_status rl_fused_head_loss_fwd_bwd(
     ma.t0 = t0;
     ma.Tc = Tc;
     ma.V = static_cast<int>(V);
-    ma.n_vb = ha.n_vb;
+    ma.n_part = ha.n_vb * static_cast<int>(kParts);
     ma.n_traj = n_traj;
     ma.partials = partials;
     ma.token_ids = token_ids;
@@ -1074,7 +1089,7 @@ extern "C" rl_status rl_fused_head_token_logprobs(const void* hidden, const void
     ma.t0 = t0;
     ma.Tc = Tc;
     ma.V = static_cast<int>(V);
-    ma.n_vb = ha.n_vb;
+    ma.n_part = ha.n_vb * static_cast<int>(kParts);
     ma.partials = partials;
     ma.token_ids = token_ids;
     ma.logp_out = logp_out;

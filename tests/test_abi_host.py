@@ -202,12 +202,13 @@ def test_fused_head_logprobs_argument_checks(R):
     assert call(h=FAKE + 2) == 3
     assert call(ws=FAKE + 8) == 3
     assert call(T=0) == 0
-    # rl_workspace_size(T, V, D) always suffices; one chunk of partials is the minimum
-    # (logp=None makes a call that passed the workspace check stop at the next one)
+    # rl_workspace_size(T, V, D) always suffices; one chunk of partials (two per token and
+    # 4,096-entry vocabulary block) is the minimum (logp=None makes a call that passed the
+    # workspace check stop at the next one)
     big = dict(T=20000, V=151936, logp=None)
     assert call(ws_bytes=R.rl_workspace_size(20000, 151936, 4096), **big) == 1
-    assert call(ws_bytes=256 + 16 * 38 * 4096, **big) == 1
-    assert call(ws_bytes=256 + 16 * 38 * 4096 - 1, **big) == 4
+    assert call(ws_bytes=256 + 2 * 16 * 38 * 4096, **big) == 1
+    assert call(ws_bytes=256 + 2 * 16 * 38 * 4096 - 1, **big) == 4
 
 
 def test_masked_gae_argument_checks(R):
