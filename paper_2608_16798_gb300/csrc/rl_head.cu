@@ -814,9 +814,10 @@ static Layout layout(int64_t max_rows, int64_t V, size_t ws_bytes = 0, int64_t w
 
 // Which passes use the 256 x 512 form: bit 0 the forward-only statistics (STATS), bit 1 the
 // loss call's statistics pass (STATS_P). Measured at 32,768 x 4,096 x 151,936 (back to back,
-// same box): the forward-only call 24.24-24.36 ms wide against 24.81 ms with 256 x 256 tiles;
-// the loss call 71.5-72.1 ms either way (its heavier epilogue, which stores the exponentials,
-// is hidden behind the MMAs only with two accumulators).
+// same box): the forward-only call 24.24-24.36 ms wide (one epilogue group; 23.54-23.65 ms with
+// two) against 24.81 ms with 256 x 256 tiles; the loss call 70.9-71.9 ms with wide statistics
+// tiles (two epilogue groups) against 69.7-70.1 ms with 256 x 256 ones: its heavier epilogue,
+// which stores the exponentials, is hidden behind the MMAs only with two accumulators.
 #ifndef RL_HEAD_WIDE
 #define RL_HEAD_WIDE 1
 #endif
