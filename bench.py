@@ -217,12 +217,15 @@ def time_logits_extras(torch, R, batch, dev, peak, reps=20):
     return out
 
 
-def time_other_workloads(torch, R, dev, peak, reps=10):
+def time_other_workloads(torch, R, dev, peak, reps=10, oracle_slices=None):
     """rl_policy_loss_fwd_bwd on the long-horizon workload (bf16, entropy + k3 KL, two resident
     32,768-row microbatches: the first and the middle one) and the edge workload (fp32,
     V = 32,000, the whole 131,072-row batch as one microbatch), timed with CUDA events around
     `reps` launches after two warm-up launches. The logits stay resident (20 and 17 GB, far
-    above L2); pi_old comes from the library's forward pass plus the workload's noise."""
+    above L2); pi_old comes from the library's forward pass plus the workload's noise. With
+    `oracle_slices` (a dict), bounded spans of the same device rows are copied to the host for
+    the CPU oracle's timing: 4,096 rows of each long-horizon microbatch, the first 32,768 edge
+    rows, the whole tiny batch."""
     t = torch
     out = {}
     for name, picks in (("longhorizon", (0, None)), ("edge", (0,))):
@@ -249,6 +252,9 @@ def time_other_workloads(torch, R, dev, peak, reps=10):
             lp = logp.cpu().numpy()
             old = d(W.old_logp_from(lp, w, 0, lo))
             ref = d(W.ref_logp_from(lp, w, 0, lo)) if w.ref_noise_std else None
+            if oracle_slices is not None:
+                n_or = min(n, ORACLE_ROWS[name])
+                oracle_slices.setdefault(name, []).append((lo, logits[:n_or], ids[:n_or]))
             grad = t.empty_like(logits)
             trained = (lay.mask[lo:hi] != 0) & (coef_h[tt_h[lo:hi]] != 0)
             nbytes += int((trained.astype(np.int64) + 1).sum()) * w.vocab * es
@@ -276,17 +282,25 @@ def time_other_workloads(torch, R, dev, peak, reps=10):
         per_launch_bytes = nbytes / len(items)
         rows_per_launch = rows_total / len(items)
         gbs = per_launch_bytes / (ms * 1e-3) / 1e9
+        if oracle_slices is not None:
+            oracle_slices[name] = OracleSlice(w, oracle_slices[name], ORACLE_PARAMS[name])
         out[name] = {"rows_per_launch": rows_per_launch, "vocab": w.vocab, "dtype": w.dtype,
                      "entropy_coef": w.entropy_coef, "kl_coef": w.kl_coef, "ms_per_launch": ms,
                      "tokens_per_s": rows_per_launch / (ms * 1e-3), "algorithmic_bytes_per_launch": per_launch_bytes,
                      "achieved_gbs": gbs, "frac": gbs / peak, "reps": reps}
         del items
         t.cuda.empty_cache()
-    out["tiny"] = time_tiny(torch, R, dev)
+    out["tiny"] = time_tiny(torch, R, dev, oracle_slices=oracle_slices)
     return out
 
 
-def time_tiny(torch, R, dev, reps=100):
+# rows of each span the CPU oracle is timed on, and the objective's parameters there
+ORACLE_ROWS = {"longhorizon": 4096, "edge": 32768, "tiny": 512}
+ORACLE_PARAMS = {"longhorizon": {"kl_coef": 1e-3, "kl_estimator": 3, "entropy_coef": 1e-3}, "edge": {}, "tiny": {}}
+ORACLE_HEAD_TOKENS = 1024
+
+
+def time_tiny(torch, R, dev, reps=100, oracle_slices=None):
     """The tiny workload (one group of 8 trajectories x 64 tokens, V = 4,096 bf16): a whole step
     (advantages + the loss over the 512 rows) is 8.4 MB of logits and gradient, resident in the
     129 MB L2, so it is latency-bound and gets no HBM fraction. Timed as CUDA-graph replays (device
@@ -299,6 +313,8 @@ def time_tiny(torch, R, dev, reps=100):
     logits = t.empty((T, w.vocab), dtype=t.bfloat16, device=dev)
     W.logits_rows_torch(w, 0, 0, T, logits)
     ids = W.sample_tokens_torch(logits, 0, 0, w)
+    if oracle_slices is not None:
+        oracle_slices["tiny"] = OracleSlice(w, [(0, logits, ids)], ORACLE_PARAMS["tiny"])
     params = R.make_params(W.CLIP_EPS_LOW, W.CLIP_EPS_HIGH, 0.0, 0, 0.0, 0.0, 1e-6, 0)
     ws = R.new_workspace(T, w.vocab, device=dev)
     logp, _, _ = R.rl_token_logprobs(logits, ids, ws)
@@ -671,22 +687,41 @@ def _gen_rows(span):
     return hi - lo
 
 
-def _oracle_init(shm_name, shape, ids, mask, tt, adv, coef, old):
+def _oracle_init(shm_name, shape, dtype, inputs, params):
     from multiprocessing import shared_memory
 
     sys.path.insert(0, ROOT)
     shm = shared_memory.SharedMemory(name=shm_name)
-    _W.update(shm=shm, raw=np.ndarray(shape, dtype=np.uint16, buffer=shm.buf), ids=ids, mask=mask, tt=tt, adv=adv,
-              coef=coef, old=old)
+    raw = np.ndarray(shape, dtype=np.uint16 if dtype == "bf16" else np.float32, buffer=shm.buf)
+    _W.update(shm=shm, raw=raw, dtype=dtype, params=params, **inputs)
 
 
 def _oracle_rows(span):
     import oracle.grpo_objective as O
 
     lo, hi = span
-    O.policy_loss_fwd_bwd(_W["raw"][lo:hi], "bf16", _W["ids"][lo:hi], _W["mask"][lo:hi], _W["tt"][lo:hi], _W["adv"],
-                          _W["coef"], _W["old"][lo:hi], O.LossParams())
+    ref = None if _W["ref"] is None else _W["ref"][lo:hi]
+    O.policy_loss_fwd_bwd(_W["raw"][lo:hi], _W["dtype"], _W["ids"][lo:hi], _W["mask"][lo:hi], _W["tt"][lo:hi],
+                          _W["adv"], _W["coef"], _W["old"][lo:hi], O.LossParams(**_W["params"]), ref_logp=ref)
     return hi - lo
+
+
+def _logp_from_law(w, z_a):
+    """Log-probability of the sampled token from the logit law alone (lse ~ ln V + sigma^2 / 2 for
+    N(0, sigma^2) logits): places old_logp (and ref_logp) near it without using any output of the
+    CUDA library."""
+    return z_a - (math.log(w.vocab) + w.logit_std ** 2 / 2)
+
+
+def _oracle_layout_inputs(w, lay, gidx):
+    """Advantages, coefficients and trajectory ids of the whole batch (oracle), and the mask and
+    trajectory ids of the rows gidx."""
+    import oracle.grpo_objective as O
+
+    P = O.LossParams(loss_agg=0)
+    adv, coef, _, tt = O.advantages_and_coefficients(lay.rewards, lay.group_offsets, lay.traj_offsets, lay.mask,
+                                                     lay.traj_valid, P)
+    return adv, coef, lay.mask[gidx], tt[gidx]
 
 
 class OracleSample:
@@ -722,20 +757,61 @@ class OracleSample:
                 ids_shm.unlink()
             self.source = "numpy-drawn logits of the same law (no GPU used)"
 
-    def oracle_inputs(self):
-        """Inputs of the oracle for these rows. old_logp is placed near the sampled token's
-        log-probability from the logit law (lse ~ ln V + sigma^2 / 2 for N(0, sigma^2) logits),
-        which keeps the timing leg independent of the CUDA library's outputs."""
-        import oracle.grpo_objective as O
+    dtype = "bf16"
+    params = {}
 
+    def oracle_inputs(self):
+        """Inputs of the oracle for these rows; old_logp from the logit law (_logp_from_law)."""
         w, lay, rows = WORKLOAD, self.layout, self.rows
         z_a = (self.raw[np.arange(rows), self.ids].astype(np.uint32) << 16).view(np.float32).astype(np.float64)
-        logp_hat = z_a - (math.log(w.vocab) + w.logit_std ** 2 / 2)
-        old = W.old_logp_from(logp_hat, w, 0)
-        P = O.LossParams()
-        adv, coef, L, tt = O.advantages_and_coefficients(lay.rewards, lay.group_offsets, lay.traj_offsets, lay.mask,
-                                                         lay.traj_valid, P)
-        return self.ids, lay.mask[:rows], tt[:rows], adv, coef, old
+        old = W.old_logp_from(_logp_from_law(w, z_a), w, 0)
+        adv, coef, mask, tt = _oracle_layout_inputs(w, lay, np.arange(rows))
+        return {"ids": self.ids, "mask": mask, "tt": tt, "adv": adv, "coef": coef, "old": old, "ref": None}
+
+    def close(self):
+        self.shm.close()
+        self.shm.unlink()
+
+
+class OracleSlice:
+    """Spans of rows of a workload's device logits (rows the GPU timed), copied into host shared
+    memory for the float64 oracle, with the oracle's own inputs for them: the batch's advantages
+    and coefficients from the oracle, old_logp (and ref_logp) from the logit law."""
+
+    def __init__(self, w, pieces, params):
+        """pieces: (first global row, device logits [n x V], device ids [n]) per span."""
+        from multiprocessing import shared_memory
+
+        import torch
+
+        self.w, self.params, self.dtype = w, params, w.dtype
+        self.layout = W.make_layout(w, 0)
+        self.rows = sum(int(lg.shape[0]) for _, lg, _ in pieces)
+        es = 2 if w.dtype == "bf16" else 4
+        self.shm = shared_memory.SharedMemory(create=True, size=self.rows * w.vocab * es)
+        self.raw = np.ndarray((self.rows, w.vocab), dtype=np.uint16 if es == 2 else np.float32, buffer=self.shm.buf)
+        ids, old, ref, gidx, r = [], [], [], [], 0
+        for lo, lg, dids in pieces:
+            n = int(lg.shape[0])
+            view = torch.from_numpy(self.raw[r:r + n].view(np.int16 if es == 2 else np.int32))
+            view.copy_(lg.view(torch.int16 if es == 2 else torch.int32))
+            a = dids.cpu().numpy().astype(np.int32)
+            z = self.raw[np.arange(r, r + n), a]
+            z_a = ((z.astype(np.uint32) << 16).view(np.float32) if es == 2 else z).astype(np.float64)
+            lp = _logp_from_law(w, z_a)
+            ids.append(a)
+            old.append(W.old_logp_from(lp, w, 0, lo))
+            ref.append(W.ref_logp_from(lp, w, 0, lo) if w.ref_noise_std else None)
+            gidx.append(np.arange(lo, lo + n))
+            r += n
+        self.ids, self.old = np.concatenate(ids), np.concatenate(old)
+        self.ref = None if ref[0] is None else np.concatenate(ref)
+        self.gidx = np.concatenate(gidx)
+        self.spans = [(lo, lo + int(lg.shape[0])) for lo, lg, _ in pieces]
+
+    def oracle_inputs(self):
+        adv, coef, mask, tt = _oracle_layout_inputs(self.w, self.layout, self.gidx)
+        return {"ids": self.ids, "mask": mask, "tt": tt, "adv": adv, "coef": coef, "old": self.old, "ref": self.ref}
 
     def close(self):
         self.shm.close()
@@ -748,13 +824,12 @@ class OraclePool:
 
     CHUNK = 16
 
-    def __init__(self, sample: OracleSample):
+    def __init__(self, sample):
         self.cores = len(os.sched_getaffinity(0))
         self.sample = sample
-        ids, mask, tt, adv, coef, old = sample.oracle_inputs()
         self.pool = mp.get_context("spawn").Pool(self.cores, initializer=_oracle_init,
-                                                 initargs=(sample.shm.name, sample.raw.shape, ids, mask, tt, adv,
-                                                           coef, old))
+                                                 initargs=(sample.shm.name, sample.raw.shape, sample.dtype,
+                                                           sample.oracle_inputs(), sample.params))
         # imports and first touch of the workers (untimed)
         self.pool.map(_oracle_rows, [(i * self.CHUNK, (i + 1) * self.CHUNK) for i in range(self.cores)], chunksize=1)
 
@@ -784,6 +859,19 @@ def time_oracle(sample: OracleSample):
     return {"value": sample.rows / dt, "unit": UNIT, "cores": op.cores, "kind": "oracle", "seconds": dt,
             "sample": f"the first microbatch of the batch, all {sample.rows} rows ({trained} trained, the others "
                       f"masked), once, from {sample.source}; float64 numpy oracle on {op.cores} spawn workers"}
+
+
+def time_oracle_slice(sl: OracleSlice):
+    """The oracle over every row of a workload's slice, once, on all host cores."""
+    op = OraclePool(sl)
+    try:
+        dt = op.run(0, sl.rows)
+    finally:
+        op.close()
+    spans = ", ".join(f"[{lo}, {hi})" for lo, hi in sl.spans)
+    return {"rows": sl.rows, "seconds": dt, "tokens_per_s": sl.rows / dt, "cores": op.cores,
+            "sample": f"rows {spans} of the {sl.w.name} batch ({sl.w.dtype}, V = {sl.w.vocab}), the device rows the "
+                      f"GPU timed, once; float64 numpy oracle on {op.cores} spawn workers"}
 
 
 # ----------------------------------------------------------------------------- main
@@ -830,6 +918,8 @@ def compact_summary(value, ms_step, roofline, extras, head, ppo, tree, cpu, e2e)
                              "bound": "host"}
     if cpu:
         out["cpu_oracle"] = {"tokens_per_s": _r(cpu["value"]), "cores": cpu["cores"]}
+        for k, o in (cpu.get("workloads") or {}).items():
+            out["cpu_oracle"][f"{k}_tokens_per_s"] = _r(o["tokens_per_s"])
     if e2e:
         out["e2e"] = {"tokens_per_s": _r(e2e["value"])}
     return out
@@ -1003,8 +1093,40 @@ def _time_calls(torch, fn, warmup, reps):
     return a.elapsed_time(b) / reps
 
 
-def time_head(torch, R, dev, warmup=2, reps=5):
+class HeadSample:
+    """The first tokens of the fused-head workload (hidden rows, the whole W, ids) on the host for
+    the CPU oracle; old_logp as the device workload draws it (from a torch matmul of the set-up,
+    not from the library), the advantages and coefficients from the oracle."""
+
+    def __init__(self, torch, hb, n):
+        t = torch
+        self.n = n
+        self.hidden = hb.hidden[:n].view(t.int16).cpu().numpy().view(np.uint16)
+        self.weight = hb.weight.view(t.int16).cpu().numpy().view(np.uint16)
+        self.ids = hb.ids[:n].cpu().numpy()
+        self.old = hb.old[:n].cpu().numpy().astype(np.float64)
+        self.layout = W.make_layout(HEAD, 0)
+
+
+def time_oracle_head(hs: HeadSample):
+    """The float64 oracle of the fused head (Z = H W^T, the objective, dH = dZ W, dW = dZ^T H)
+    over the sample's tokens at the full D and V, once, in this process (numpy's BLAS threads)."""
+    import oracle.grpo_objective as O
+
+    adv, coef, mask, tt = _oracle_layout_inputs(HEAD, hs.layout, np.arange(hs.n))
+    t0 = time.perf_counter()
+    O.fused_head_loss_fwd_bwd(hs.hidden, hs.weight, hs.ids, mask, tt, adv, coef, hs.old, O.LossParams())
+    dt = time.perf_counter() - t0
+    V, D = hs.weight.shape
+    return {"rows": hs.n, "seconds": dt, "tokens_per_s": hs.n / dt, "flops": 6.0 * hs.n * D * V,
+            "threads": f"numpy BLAS, {len(os.sched_getaffinity(0))} host cores",
+            "sample": f"the first {hs.n} tokens of the fused-head workload at full D = {D} and V = {V} "
+                      "(W decoded to float64, Z, the objective, dH and dW in float64), from the device inputs"}
+
+
+def time_head(torch, R, dev, warmup=2, reps=5, oracle_tokens=0):
     hb = HeadBatch(torch, R, dev)
+    hs = HeadSample(torch, hb, oracle_tokens) if oracle_tokens else None
     ms = _time_calls(torch, lambda: hb.call(R), warmup, reps)
     ms_fwd = _time_calls(torch, lambda: hb.call_logprobs(R), warmup, reps)
     st, word = R.rl_query_status(hb.ws)
@@ -1032,7 +1154,7 @@ def time_head(torch, R, dev, warmup=2, reps=5):
             "note": "6 T D V (Z once, dH, dW), all on hand-written tcgen05 kernels (head_kernel: logits tiles and "
                     "softmax partials; head_grad_kernel: dH and dW in one launch), smallest workspace "
                     f"({hb.ws.numel() / 1e9:.2f} GB: one 4,096-token chunk of the logits gradient)",
-            "logprobs": fwd}
+            "logprobs": fwd}, hs
 
 
 def profile_head(T):
@@ -1293,9 +1415,11 @@ def main():
         ts = [kern_ms[s * n_mb + k] for s in range(args.steps)]
         per_mb.append({"rows": batch.mbs[k][1] - batch.mbs[k][0], "median_ms": statistics.median(ts),
                        "best_ms": min(ts), "median_gbs": batch.mb_bytes[k] / (statistics.median(ts) * 1e-3) / 1e9})
+    want_cpu = rank == 0 and world == 1 and not args.no_cpu_baseline
+    oracle_slices = {} if want_cpu else None  # host copies of device rows for the CPU oracle
     extras = time_logits_extras(torch, R, batch, dev, peak)
     if not args.no_other:
-        extras["other_workloads"] = time_other_workloads(torch, R, dev, peak)
+        extras["other_workloads"] = time_other_workloads(torch, R, dev, peak, oracle_slices=oracle_slices)
     extras["loss_batch_sum_ms"] = sum(m["median_ms"] for m in per_mb)
     extras["loss_microbatch_median_ms"] = [round(m["median_ms"], 4) for m in per_mb]
 
@@ -1309,20 +1433,27 @@ def main():
                "note": "per step: metadata and every microbatch's logits from pinned host memory, loss read "
                        "back; the gradient stays in HBM for the model's backward"}
 
-    cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        sample = OracleSample(batch.mbs[0][1] - batch.mbs[0][0], batch.logits, batch.ids)
-        try:
-            cpu = time_oracle(sample)
-        finally:
-            sample.close()
-
     ppo = None if args.no_ppo else time_ppo(torch, R, batch, dev)
     tree = None if args.no_tree else time_tree(torch, R, dev)
 
-    head = None
+    head, head_sample = None, None
     if not args.no_head:
-        head = time_head(torch, R, dev)
+        head, head_sample = time_head(torch, R, dev, oracle_tokens=ORACLE_HEAD_TOKENS if want_cpu else 0)
+
+    cpu = None
+    if want_cpu:
+        # the CPU oracle (float64, as it stands): the benchmark's first microbatch, then bounded
+        # samples of the other workloads' device rows
+        sample = OracleSample(batch.mbs[0][1] - batch.mbs[0][0], batch.logits, batch.ids)
+        try:
+            cpu = time_oracle(sample)
+            cpu["workloads"] = {name: time_oracle_slice(sl) for name, sl in oracle_slices.items()}
+            if head_sample is not None:
+                cpu["workloads"]["fusedhead"] = time_oracle_head(head_sample)
+        finally:
+            sample.close()
+            for sl in oracle_slices.values():
+                sl.close()
 
     if rank == 0:
         summary = compact_summary(value, ms_step, roofline, extras, head, ppo, tree, cpu, e2e)
