@@ -284,7 +284,9 @@ rl_status rl_policy_loss_fwd_bwd(const void* logits, rl_dtype dtype, int64_t row
  * rescale turns the kept values into the logits' gradient. After the last chunk of
  * each group (each chunk, with the smallest workspace), two tensor-core products give
  * the group's dH and add its dW (fp32, one addition per element and group, in chunk
- * order: deterministic). The logits of all T tokens are never held at once.
+ * order: deterministic). The groups follow ws_bytes, so the rounding of d_weight and
+ * d_hidden (not their values up to rounding) depends on the workspace size; calls with
+ * the same ws_bytes give the same bits. The logits of all T tokens are never held at once.
  */
 rl_status rl_fused_head_loss_fwd_bwd(const void* hidden, const void* weight, int64_t T, int64_t D, int64_t V,
                                      const int32_t* token_ids, const uint8_t* mask, const int32_t* token_traj,
