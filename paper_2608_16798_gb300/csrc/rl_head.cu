@@ -592,9 +592,31 @@ struct MergeArgs {
   int32_t* status;
 };
 
+// Token r's partials merged in index order (the same order in both merge kernels, so that the
+// forward-only call and the loss call agree bit for bit); the loads run 8 ahead of the merges.
+__device__ __forceinline__ void merge_partials(const float4* partials, int64_t Tc, int r, int n_part,
+                                               SoftmaxPartial& q, float& za) {
+  constexpr int kAhead = 8;
+  for (int b0 = 0; b0 < n_part; b0 += kAhead) {
+    float4 w[kAhead];
+#pragma unroll
+    for (int k = 0; k < kAhead; ++k)
+      if (b0 + k < n_part) w[k] = partials[static_cast<int64_t>(b0 + k) * Tc + r];
+#pragma unroll
+    for (int k = 0; k < kAhead; ++k)
+      if (b0 + k < n_part) {
+        q = merge(q, SoftmaxPartial{w[k].x, w[k].y, w[k].z});
+        za += w[k].w;  // nonzero in the one partial whose columns hold the sampled id
+      }
+  }
+}
+
+// threads per CTA of the merge kernels: small CTAs spread a chunk's tokens over many SMs
+constexpr int kMergeThreads = 64;
+
 // One thread per token of the chunk: merge the vocabulary blocks' partials (fixed order)
 // and evaluate the per-token objective terms.
-__global__ void __launch_bounds__(256) head_merge_kernel(const MergeArgs p) {
+__global__ void __launch_bounds__(kMergeThreads) head_merge_kernel(const MergeArgs p) {
   const int r = blockIdx.x * blockDim.x + threadIdx.x;
   if (r >= p.Tc) return;
   const int64_t t = p.t0 + r;
@@ -625,11 +647,7 @@ __global__ void __launch_bounds__(256) head_merge_kernel(const MergeArgs p) {
   }
   SoftmaxPartial q{-__int_as_float(0x7f800000), 0.f, 0.f};
   float za = 0.f;
-  for (int b = 0; b < p.n_part; ++b) {
-    const float4 w = p.partials[static_cast<int64_t>(b) * p.Tc + r];
-    q = merge(q, SoftmaxPartial{w.x, w.y, w.z});
-    za += w.w;
-  }
+  merge_partials(p.partials, p.Tc, r, p.n_part, q, za);
   const float lnS = logf(q.s);
   const float lse = q.m + lnS;
   const float H = lnS - q.u / q.s;
@@ -747,17 +765,13 @@ struct LogpMergeArgs {
 };
 
 // Forward-only merge: one thread per token of the chunk writes logp, H and lse.
-__global__ void __launch_bounds__(256) head_logp_merge_kernel(const LogpMergeArgs p) {
+__global__ void __launch_bounds__(kMergeThreads) head_logp_merge_kernel(const LogpMergeArgs p) {
   const int r = blockIdx.x * blockDim.x + threadIdx.x;
   if (r >= p.Tc) return;
   const int64_t t = p.t0 + r;
   SoftmaxPartial q{-__int_as_float(0x7f800000), 0.f, 0.f};
   float za = 0.f;
-  for (int b = 0; b < p.n_part; ++b) {
-    const float4 w = p.partials[static_cast<int64_t>(b) * p.Tc + r];
-    q = merge(q, SoftmaxPartial{w.x, w.y, w.z});
-    za += w.w;  // nonzero in the one partial whose columns hold the sampled id
-  }
+  merge_partials(p.partials, p.Tc, r, p.n_part, q, za);
   const float lnS = logf(q.s);
   const float lse = q.m + lnS;
   const int32_t a = p.token_ids[t];
@@ -1007,7 +1021,7 @@ extern "C" rl_status rl_fused_head_loss_fwd_bwd(
     ma.row_loss = row_loss;
     ma.token_stats = token_stats;
     ma.status = status;
-    head_merge_kernel<<<(Tc + 255) / 256, 256, 0, s>>>(ma);
+    head_merge_kernel<<<(Tc + kMergeThreads - 1) / kMergeThreads, kMergeThreads, 0, s>>>(ma);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_error(e, "head_merge_kernel launch");
 
@@ -1097,7 +1111,7 @@ extern "C" rl_status rl_fused_head_token_logprobs(const void* hidden, const void
     ma.entropy_out = entropy_out;
     ma.lse_out = lse_out;
     ma.status = status;
-    head_logp_merge_kernel<<<(Tc + 255) / 256, 256, 0, s>>>(ma);
+    head_logp_merge_kernel<<<(Tc + kMergeThreads - 1) / kMergeThreads, kMergeThreads, 0, s>>>(ma);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_error(e, "head_logp_merge_kernel launch");
   }
