@@ -124,6 +124,7 @@ def compare_head(c, out, dh_bf16=False):
     (256, 128, 8292, 0, False, False),     # three vocabulary blocks
     (200, 192, 700, 2, True, False),       # entropy + k3 KL
     (130, 64, 513, 1, False, True),        # TIS, token-mean, smallest D
+    (260, 128, 2000, 0, True, True),       # entropy + k3 KL + TIS together
     (100, 128, 777, 0, True, False),       # one CTA pair whose odd CTA's 128 tokens all lie past T
     (5, 64, 300, 2, False, False),         # a handful of tokens
     (40, 64, 524_288, 2, False, False),    # the largest vocabulary (128 blocks of 4,096)
