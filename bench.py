@@ -283,7 +283,7 @@ def time_other_workloads(torch, R, dev, peak, reps=10, oracle_slices=None):
         rows_per_launch = rows_total / len(items)
         gbs = per_launch_bytes / (ms * 1e-3) / 1e9
         if oracle_slices is not None:
-            oracle_slices[name] = OracleSlice(w, oracle_slices[name], ORACLE_PARAMS[name])
+            oracle_slices[name] = make_oracle_slice(w, oracle_slices[name], ORACLE_PARAMS[name])
         out[name] = {"rows_per_launch": rows_per_launch, "vocab": w.vocab, "dtype": w.dtype,
                      "entropy_coef": w.entropy_coef, "kl_coef": w.kl_coef, "ms_per_launch": ms,
                      "tokens_per_s": rows_per_launch / (ms * 1e-3), "algorithmic_bytes_per_launch": per_launch_bytes,
@@ -314,7 +314,7 @@ def time_tiny(torch, R, dev, reps=100, oracle_slices=None):
     W.logits_rows_torch(w, 0, 0, T, logits)
     ids = W.sample_tokens_torch(logits, 0, 0, w)
     if oracle_slices is not None:
-        oracle_slices["tiny"] = OracleSlice(w, [(0, logits, ids)], ORACLE_PARAMS["tiny"])
+        oracle_slices["tiny"] = make_oracle_slice(w, [(0, logits, ids)], ORACLE_PARAMS["tiny"])
     params = R.make_params(W.CLIP_EPS_LOW, W.CLIP_EPS_HIGH, 0.0, 0, 0.0, 0.0, 1e-6, 0)
     ws = R.new_workspace(T, w.vocab, device=dev)
     logp, _, _ = R.rl_token_logprobs(logits, ids, ws)
@@ -818,6 +818,15 @@ class OracleSlice:
         self.shm.unlink()
 
 
+def make_oracle_slice(w, pieces, params):
+    """An OracleSlice, or the reason it could not be made (host or shared memory short): the
+    CPU leg's extra samples never cost the benchmark its line."""
+    try:
+        return OracleSlice(w, pieces, params)
+    except (OSError, MemoryError) as e:
+        return f"{type(e).__name__}: {e}"
+
+
 class OraclePool:
     """The float64 oracle, as it stands, over a spawn pool of all host cores. Each job is a
     16-row span of the sample; ``run(lo, hi)`` times the oracle over rows [lo, hi) once."""
@@ -861,8 +870,11 @@ def time_oracle(sample: OracleSample):
                       f"masked), once, from {sample.source}; float64 numpy oracle on {op.cores} spawn workers"}
 
 
-def time_oracle_slice(sl: OracleSlice):
-    """The oracle over every row of a workload's slice, once, on all host cores."""
+def time_oracle_slice(sl):
+    """The oracle over every row of a workload's slice, once, on all host cores (or the reason
+    the slice is missing)."""
+    if isinstance(sl, str):
+        return {"unavailable": sl}
     op = OraclePool(sl)
     try:
         dt = op.run(0, sl.rows)
@@ -919,7 +931,7 @@ def compact_summary(value, ms_step, roofline, extras, head, ppo, tree, cpu, e2e)
     if cpu:
         out["cpu_oracle"] = {"tokens_per_s": _r(cpu["value"]), "cores": cpu["cores"]}
         for k, o in (cpu.get("workloads") or {}).items():
-            out["cpu_oracle"][f"{k}_tokens_per_s"] = _r(o["tokens_per_s"])
+            out["cpu_oracle"][f"{k}_tokens_per_s"] = _r(o.get("tokens_per_s"))
     if e2e:
         out["e2e"] = {"tokens_per_s": _r(e2e["value"])}
     return out
@@ -1449,11 +1461,15 @@ def main():
             cpu = time_oracle(sample)
             cpu["workloads"] = {name: time_oracle_slice(sl) for name, sl in oracle_slices.items()}
             if head_sample is not None:
-                cpu["workloads"]["fusedhead"] = time_oracle_head(head_sample)
+                try:
+                    cpu["workloads"]["fusedhead"] = time_oracle_head(head_sample)
+                except MemoryError as e:
+                    cpu["workloads"]["fusedhead"] = {"unavailable": f"MemoryError: {e}"}
         finally:
             sample.close()
             for sl in oracle_slices.values():
-                sl.close()
+                if not isinstance(sl, str):
+                    sl.close()
 
     if rank == 0:
         summary = compact_summary(value, ms_step, roofline, extras, head, ppo, tree, cpu, e2e)

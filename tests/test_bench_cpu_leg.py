@@ -52,3 +52,14 @@ def test_oracle_head_timing():
     assert hs.hidden.shape == (8, D) and hs.weight.shape == (V, D)
     r = bench.time_oracle_head(hs)
     assert r["rows"] == 8 and r["flops"] == 6.0 * 8 * D * V and r["tokens_per_s"] > 0
+
+
+def test_oracle_slice_failure_is_reported_not_raised(monkeypatch):
+    """A slice that cannot be made (shared memory short) is reported as unavailable."""
+    def no_room(*a, **k):
+        raise OSError(28, "No space left on device")
+
+    monkeypatch.setattr(bench, "OracleSlice", no_room)
+    sl = bench.make_oracle_slice(W.WORKLOADS["tiny"], [], {})
+    assert isinstance(sl, str) and "OSError" in sl
+    assert bench.time_oracle_slice(sl) == {"unavailable": sl}
