@@ -1,8 +1,8 @@
 """The entry points inside CUDA graphs and on concurrent streams.
 
 Every entry point enqueues work on the caller's stream and allocates nothing, so a whole
-step (advantages, then the loss over the microbatches; the fused head with its cuBLASLt
-products) can be captured once and replayed; replays give the eager results bit for bit
+step (advantages, then the loss over the microbatches; the fused head with its tensor-core
+backward products and their work counter) can be captured once and replayed; replays give the eager results bit for bit
 (the reductions have a fixed order). Host threads calling the library on their own streams
 with their own workspaces get the same bits as serial calls.
 """
