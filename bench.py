@@ -46,13 +46,13 @@ KERNEL_SRC = os.path.join(ROOT, "paper_2608_16798_gb300", "csrc", "rl_rows.cu")
 FALLBACK_HBM_GBS = 6800.0
 
 
-def workload_config(T, n_mb, inputs_sha256=None):
+def workload_config(T, n_mb):
     w = WORKLOAD
     return {"workload": f"multiturn: {w.n_groups} groups x {w.group_size} trajectories, lengths U{{256..2048}}, "
                         f"~40% masked in spans, V={w.vocab}, bf16 logits N(0,2^2), {w.microbatch}-row microbatches",
             "tokens_per_step": int(T), "microbatches": int(n_mb), "vocab": w.vocab, "logits": "bf16",
             "l2": "no flush: resident inputs (logits + gradient) far larger than L2",
-            "parallelism": "replicas", "seed": 0, "inputs_sha256": inputs_sha256}
+            "parallelism": "replicas", "seed": 0}
 
 
 def measured_peaks():
@@ -1475,8 +1475,8 @@ def main():
         summary = compact_summary(value, ms_step, roofline, extras, head, ppo, tree, cpu, e2e)
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
-                "vs_baseline": None, "dtype": "f32", "data": "synthetic", "config": workload_config(batch.T, n_mb, batch.inputs_sha256),
-                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks, "logits_path": extras, "fused_head": head, "ppo": ppo, "tree": tree,
+                "vs_baseline": None, "dtype": "f32", "data": "synthetic", "config": workload_config(batch.T, n_mb),
+                "inputs_sha256": batch.inputs_sha256, "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks, "logits_path": extras, "fused_head": head, "ppo": ppo, "tree": tree,
                 "gpu_launches": batch.launches_per_step() * args.steps,
                 "loss_per_step": float(batch.loss.item()) / (args.warmup + args.steps),
                 "summary": summary}
