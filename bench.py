@@ -1241,8 +1241,11 @@ def profile_segments(reps=3):
     """The segmented reductions alone, for profiler captures (a few MB on the device): `reps`
     calls of rl_group_advantages on the multi-turn batch's layout (traj_count_kernel,
     group_adv_kernel), then on the tree workload's packed stream rl_group_advantages_by_owner
-    (owner_count_kernel, group_adv_kernel) and rl_sequence_is_weights (owner_logratio_kernel,
-    seq_weight_kernel; log-probs N(-2, 1) per token, rollout = old + N(0, 0.02^2))."""
+    (owner_count_kernel, group_adv_kernel), rl_sequence_is_weights (owner_logratio_kernel,
+    seq_weight_kernel; log-probs N(-2, 1) per token, rollout = old + N(0, 0.02^2)), the same with
+    per-token advantages scaled in place (token_scale_kernel) and rl_rollout_value_advantages
+    (rollout_adv_kernel; values N(0, 1) per token); and rl_token_stats_summary over the multi-turn
+    batch's rows (stats_summary_kernel; per-token statistics uniform on [0, 1))."""
     import torch
 
     from paper_2608_16798_gb300 import build as B
@@ -1259,7 +1262,10 @@ def profile_segments(reps=3):
     go, rw, to, mask, valid = (d(lay.group_offsets), d(lay.rewards), d(lay.traj_offsets), d(lay.mask),
                                d(lay.traj_valid))
     for _ in range(reps):
-        R.rl_group_advantages(go, rw, to, mask, params, ws, traj_valid=valid)
+        _, coef, _, tt = R.rl_group_advantages(go, rw, to, mask, params, ws, traj_valid=valid)
+    stats = d(np.random.default_rng(2).random(lay.n_tokens * 5, dtype=np.float32))
+    for _ in range(reps):
+        R.rl_token_stats_summary(stats, mask, tt, coef, ws)
     w = W.WORKLOADS["tree"]
     prompts, calls, aux = W.tree_rollouts(w, seed=0)
     out = R.rl_prefix_tree_build_batch(prompts, calls, aux, max_leaves=w.tree_max_leaves, n_threads=4)
@@ -1276,6 +1282,12 @@ def profile_segments(reps=3):
     ws_tree = R.new_workspace(n, 0, device=dev)
     for _ in range(reps):
         R.rl_sequence_is_weights(owner, tmask, old, roll, n, ws_tree, cap=2.0)
+    tok_adv = d(np.random.default_rng(3).normal(0.0, 1.0, T).astype(np.float32))
+    for _ in range(reps):
+        R.rl_sequence_is_weights(owner, tmask, old, roll, n, ws_tree, cap=2.0, token_adv_inout=tok_adv)
+    values = d(np.random.default_rng(4).normal(0.0, 1.0, T).astype(np.float32))
+    for _ in range(reps):
+        R.rl_rollout_value_advantages(owner, tmask, values, trw, ws_tree)
     word = R.rl_query_status(ws)[1] | R.rl_query_status(ws_tree)[1]
     print(json.dumps({"profile_segments": reps, "multiturn_tokens": lay.n_tokens, "multiturn_traj": lay.n_traj,
                       "tree_tokens": T, "tree_rollouts": n, "status": word}))

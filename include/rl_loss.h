@@ -309,7 +309,8 @@ rl_status rl_fused_head_loss_fwd_bwd(const void* hidden, const void* weight, int
  *   mask, token_traj, n_traj, coef   as for rl_policy_loss_fwd_bwd
  *   summary_accum      double [5] on the device
  *   ws, ws_bytes       rl_workspace_size(0, 0, 0) bytes suffice (status word)
- * One CTA in a fixed order, in double precision: deterministic.
+ * One launch of one 8-CTA cluster, a fixed assignment of rows to threads and a fixed order of
+ * the partial sums, in double precision: deterministic.
  */
 rl_status rl_token_stats_summary(int64_t rows, const float* token_stats, const uint8_t* mask,
                                  const int32_t* token_traj, int32_t n_traj, const float* coef,

@@ -359,6 +359,30 @@ def test_nan_logits_stay_in_their_rows(R):
     check_grad(out["grad"][rows], g_ref, case.w.dtype, "rows without NaN")
 
 
+@pytest.mark.parametrize("rows", [1, 8191, 8193, 77881, 155959])
+def test_stats_summary_sizes(R, rows):
+    """The summary over batches that span the cluster's 8,192 threads several times with a
+    ragged tail (and the multi-turn batch's size): counts exact, sums within 1e-12 of the float64
+    sums of the same float32 values, and the same bits on a second call."""
+    rng = np.random.default_rng(rows)
+    n_traj = 97
+    stats = rng.random((rows, 5), dtype=np.float32)
+    stats[:, 2] = (rng.random(rows) < 0.1).astype(np.float32)  # clipped flags
+    mask = (rng.random(rows) < 0.6).astype(np.uint8)
+    tt = rng.integers(0, n_traj, rows).astype(np.int32)
+    coef = rng.random(n_traj).astype(np.float32)
+    coef[::7] = 0.0
+    ws = R.new_workspace(0, 0)
+    args = (torch.from_numpy(stats.reshape(-1)).cuda(), to_dev(mask), to_dev(tt), to_dev(coef), ws)
+    a = R.rl_token_stats_summary(*args).cpu().numpy()
+    b = R.rl_token_stats_summary(*args).cpu().numpy()
+    assert R.rl_query_status(ws)[1] == 0
+    ref = O.stats_summary(stats.astype(np.float64), mask, tt, coef)
+    assert a[0] == ref[0] and a[1] == ref[1]
+    assert np.allclose(a[2:], ref[2:], rtol=1e-12, atol=1e-12)
+    assert np.array_equal(a, b)
+
+
 def test_stats_summary(R):
     """Summaries of the loss call's statistics: counts exact, sums equal the float64 sum of the
     same float32 values (order-independent to 1e-12), and within the statistics' own tolerances
