@@ -221,7 +221,8 @@ def time_other_workloads(torch, R, dev, peak, reps=10, oracle_slices=None):
     """rl_policy_loss_fwd_bwd on the long-horizon workload (bf16, entropy + k3 KL, two resident
     32,768-row microbatches: the first and the middle one) and the edge workload (fp32,
     V = 32,000, the whole 131,072-row batch as one microbatch), timed with CUDA events around
-    `reps` launches after two warm-up launches. The logits stay resident (20 and 17 GB, far
+    `reps` launches after two warm-up launches; and rl_group_advantages over each workload's
+    whole batch (512 trajectories in 32 groups; 16,384 in 4,096 groups) as CUDA-graph replays. The logits stay resident (20 and 17 GB, far
     above L2); pi_old comes from the library's forward pass plus the workload's noise. With
     `oracle_slices` (a dict), bounded spans of the same device rows are copied to the host for
     the CPU oracle's timing: 4,096 rows of each long-horizon microbatch, the first 32,768 edge
@@ -239,9 +240,14 @@ def time_other_workloads(torch, R, dev, peak, reps=10, oracle_slices=None):
         kl = 3 if w.kl_coef else 0
         params = R.make_params(W.CLIP_EPS_LOW, W.CLIP_EPS_HIGH, w.kl_coef, kl, w.entropy_coef, 0.0, 1e-6, 0)
         ws = R.new_workspace(w.microbatch, w.vocab, device=dev)
-        adv, coef, n_tok, tt = R.rl_group_advantages(d(lay.group_offsets), d(lay.rewards), d(lay.traj_offsets),
-                                                     d(lay.mask), params, ws, traj_valid=d(lay.traj_valid))
+        go, rw, to, mk, va = (d(lay.group_offsets), d(lay.rewards), d(lay.traj_offsets), d(lay.mask),
+                              d(lay.traj_valid))
+        adv, coef, n_tok, tt = R.rl_group_advantages(go, rw, to, mk, params, ws, traj_valid=va)
         coef_h, tt_h = coef.cpu().numpy(), tt.cpu().numpy()
+        # the advantages over the workload's whole batch, alone (CUDA-graph replays)
+        ms_adv = _time_graph(torch, lambda: R.rl_group_advantages(go, rw, to, mk, params, ws, traj_valid=va,
+                                                                  adv_out=adv, coef_out=coef, n_tok_out=n_tok,
+                                                                  token_traj_out=tt), 20)
         items, nbytes, rows_total = [], 0, 0
         for lo, hi in chosen:
             n = hi - lo
@@ -287,7 +293,9 @@ def time_other_workloads(torch, R, dev, peak, reps=10, oracle_slices=None):
         out[name] = {"rows_per_launch": rows_per_launch, "vocab": w.vocab, "dtype": w.dtype,
                      "entropy_coef": w.entropy_coef, "kl_coef": w.kl_coef, "ms_per_launch": ms,
                      "tokens_per_s": rows_per_launch / (ms * 1e-3), "algorithmic_bytes_per_launch": per_launch_bytes,
-                     "achieved_gbs": gbs, "frac": gbs / peak, "reps": reps}
+                     "achieved_gbs": gbs, "frac": gbs / peak, "reps": reps,
+                     "group_advantages_us": ms_adv * 1e3, "trajectories": int(lay.n_traj),
+                     "groups": int(len(lay.group_offsets) - 1), "batch_tokens": int(lay.n_tokens)}
         del items
         t.cuda.empty_cache()
     out["tiny"] = time_tiny(torch, R, dev, oracle_slices=oracle_slices)
@@ -902,7 +910,7 @@ def compact_summary(value, ms_step, roofline, extras, head, ppo, tree, cpu, e2e)
         o = (extras.get("other_workloads") or {}).get(k)
         if o:
             out[f"{k}_loss"] = {"ms": _r(o["ms_per_launch"]), "tokens_per_s": _r(o["tokens_per_s"]),
-                                "frac": _r(o["frac"]), "bound": "hbm"}
+                                "frac": _r(o["frac"]), "bound": "hbm", "adv_us": _r(o["group_advantages_us"])}
     tiny = (extras.get("other_workloads") or {}).get("tiny")
     if tiny:
         out["tiny_step"] = {"us_graph": _r(tiny["us_per_step_graph"]), "tokens_per_s": _r(tiny["tokens_per_s_graph"]),
@@ -1239,9 +1247,10 @@ def profile_case(rows, workload="multiturn"):
 
 def profile_segments(reps=3):
     """The segmented reductions alone, for profiler captures (a few MB on the device): `reps`
-    calls of rl_group_advantages on the multi-turn batch's layout (traj_count_kernel,
-    group_adv_kernel), then on the tree workload's packed stream rl_group_advantages_by_owner
-    (owner_count_kernel, group_adv_kernel), rl_sequence_is_weights (owner_logratio_kernel,
+    calls of rl_group_advantages (count_adv_kernel, coef_kernel) on the multi-turn batch's layout
+    and on the edge workload's (16,384 trajectories in 4,096 groups), then on the tree workload's
+    packed stream rl_group_advantages_by_owner (the same kernels, counting by owner),
+    rl_sequence_is_weights (owner_logratio_kernel,
     seq_weight_kernel; log-probs N(-2, 1) per token, rollout = old + N(0, 0.02^2)), the same with
     per-token advantages scaled in place (token_scale_kernel) and rl_rollout_value_advantages
     (rollout_adv_kernel; values N(0, 1) per token); and rl_token_stats_summary over the multi-turn
@@ -1263,6 +1272,10 @@ def profile_segments(reps=3):
                                d(lay.traj_valid))
     for _ in range(reps):
         _, coef, _, tt = R.rl_group_advantages(go, rw, to, mask, params, ws, traj_valid=valid)
+    el = W.make_layout(W.WORKLOADS["edge"], 0)
+    eargs = (d(el.group_offsets), d(el.rewards), d(el.traj_offsets), d(el.mask), params, ws)
+    for _ in range(reps):
+        R.rl_group_advantages(*eargs, traj_valid=d(el.traj_valid))
     stats = d(np.random.default_rng(2).random(lay.n_tokens * 5, dtype=np.float32))
     for _ in range(reps):
         R.rl_token_stats_summary(stats, mask, tt, coef, ws)

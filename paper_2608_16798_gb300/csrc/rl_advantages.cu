@@ -1,18 +1,26 @@
 // Group-relative advantages and loss coefficients over ragged trajectories.
 //
-//   traj_count_kernel   L_i = sum_t M_t over trajectory i's span of the packed
-//                       stream, and token_traj[t] = i (one warp per trajectory).
-//                       The 1 / sum_t M_{i,t} normaliser of the masked GRPO
-//                       objective (Sec. 2.3.2).
-//   group_adv_kernel    one CTA: per group (one warp each) the mean and
+//   count_adv_kernel    one launch, two kinds of CTA: the first count L_i, the
+//                       trainable tokens of each trajectory (one warp per
+//                       trajectory span, writing token_traj[t] = i; or, by owner,
+//                       a grid-stride pass over tokens in any order), the 1 /
+//                       sum_t M_{i,t} normaliser of the masked GRPO objective
+//                       (Sec. 2.3.2); the others form A_i = (R_i - mu_g) /
+//                       (sigma_g + eps) per group (one warp per group: mean and
 //                       population standard deviation of the valid members'
-//                       rewards, A_i = (R_i - mu) / (sigma + eps) (Sec. 2.3.2
-//                       GRPO advantage; Sec. 3.2.3; discarded rollouts leave
-//                       the statistics, Sec. 3.4); then N = #{valid, L_i > 0}
-//                       and the coefficients c_i.
+//                       rewards in double precision; Sec. 2.3.2 GRPO advantage,
+//                       Sec. 3.2.3; discarded rollouts leave the statistics and
+//                       get A = 0, Sec. 3.4). Counts and advantages do not depend
+//                       on each other.
+//   coef_kernel         N = #{valid i : L_i > 0} and S = sum of their L_i (every
+//                       CTA forms both, integer sums, so any order gives the same
+//                       values), then c_i for its share of the trajectories, and
+//                       A = 0 for trajectories outside every group.
 //
-// Both are latency-bound: they touch ~T + 30 n bytes, well under 0.1% of the
-// logits stream of one microbatch.
+// Every kind of work is spread over the GPU: a batch of many small groups (4,096
+// groups of 4) costs no more than a few large ones. Both kernels are
+// latency-bound: they touch ~T + 30 n bytes, well under 0.1% of the logits
+// stream of one microbatch.
 #include <cstdint>
 
 #include "rl_device.cuh"
@@ -20,16 +28,15 @@
 
 namespace rl {
 
-__global__ void __launch_bounds__(256) traj_count_kernel(int32_t n_traj, int64_t n_tokens,
-                                                         const int64_t* __restrict__ traj_offsets,
-                                                         const uint8_t* __restrict__ mask,
-                                                         int32_t* __restrict__ n_tok_out,
-                                                         int32_t* __restrict__ token_traj_out,
-                                                         int32_t* status) {
-  const int lane = threadIdx.x & 31;
-  const int64_t i = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
-  if (i >= n_traj) return;
-  int64_t s = traj_offsets[i], e = traj_offsets[i + 1];
+constexpr int kAdvThreads = 256;
+constexpr int kAdvWarps = kAdvThreads / 32;
+
+// L_i over trajectory i's span [traj_offsets[i], traj_offsets[i + 1]) and the owner of each of
+// its tokens (one warp)
+__device__ __forceinline__ void count_span(int64_t i, int lane, int64_t n_tokens, const int64_t* traj_offsets,
+                                           const uint8_t* mask, int32_t* n_tok_out, int32_t* token_traj_out,
+                                           int32_t* status) {
+  const int64_t s = traj_offsets[i], e = traj_offsets[i + 1];
   if (s < 0 || e < s || e > n_tokens) {
     if (lane == 0) {
       flag_status(status, RL_DEV_BAD_OFFSETS);
@@ -49,13 +56,11 @@ __global__ void __launch_bounds__(256) traj_count_kernel(int32_t n_traj, int64_t
 // L_i by owner, for tokens in any order (tree-packed batches, Sec. 3.2.3: each shared prefix
 // token is one token of its rollout): lanes of a warp with the same owner are counted together
 // and one integer atomic per owner and warp adds them (the counts are exact in any order).
-__global__ void __launch_bounds__(256) owner_count_kernel(int64_t n_tokens, const int32_t* __restrict__ token_traj,
-                                                          const uint8_t* __restrict__ mask, int32_t n_traj,
-                                                          int32_t* __restrict__ n_tok_out, int32_t* status) {
-  const int lane = threadIdx.x & 31;
-  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  for (int64_t base = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x - lane; base < n_tokens;
-       base += stride) {
+// Warp w of `warps` takes the 32-token runs w, w + warps, ... (n_tok_out zeroed before).
+__device__ __forceinline__ void count_owners(int64_t w, int64_t warps, int lane, int64_t n_tokens,
+                                             const int32_t* token_traj, const uint8_t* mask, int32_t n_traj,
+                                             int32_t* n_tok_out, int32_t* status) {
+  for (int64_t base = w * 32; base < n_tokens; base += warps * 32) {
     const int64_t t = base + lane;
     int32_t who = -1;
     if (t < n_tokens && mask[t] != 0) {
@@ -68,68 +73,108 @@ __global__ void __launch_bounds__(256) owner_count_kernel(int64_t n_tokens, cons
   }
 }
 
-constexpr int kAdvThreads = 1024;
-
-__global__ void __launch_bounds__(kAdvThreads) group_adv_kernel(
-    int32_t n_traj, int32_t n_groups, const int32_t* __restrict__ group_offsets,
-    const float* __restrict__ rewards, const uint8_t* __restrict__ traj_valid,
-    const int32_t* __restrict__ n_tok, double adv_eps, int32_t loss_agg, float* __restrict__ adv_out,
-    float* __restrict__ coef_out, int32_t* status) {
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  constexpr int kWarps = kAdvThreads / 32;
-
-  // trajectories outside every group keep A = 0
-  for (int i = tid; i < n_traj; i += kAdvThreads) adv_out[i] = 0.f;
-  __syncthreads();
-
-  for (int g = warp; g < n_groups; g += kWarps) {
-    const int b = group_offsets[g], e = group_offsets[g + 1];
-    if (b < 0 || e < b || e > n_traj) {
-      if (lane == 0) flag_status(status, RL_DEV_BAD_OFFSETS);
-      continue;
-    }
-    // pass 1: count, sum, and min / max (all-equal test) over valid members
-    int k = 0;
-    double sum = 0.0;
-    float lo = __int_as_float(0x7f800000), hi = -__int_as_float(0x7f800000);
-    for (int i = b + lane; i < e; i += 32) {
-      if (traj_valid && traj_valid[i] == 0) continue;
-      const float r = rewards[i];
-      ++k;
-      sum += static_cast<double>(r);
-      lo = fminf(lo, r);
-      hi = fmaxf(hi, r);
-    }
-    k = warp_sum(k);
-    sum = warp_sum(sum);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
-      hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
-    }
-    if (k == 0 || lo == hi) continue;  // nothing valid, or all valid rewards equal: A = 0
-    const double mu = sum / k;
-    double sq = 0.0;
-    for (int i = b + lane; i < e; i += 32) {
-      if (traj_valid && traj_valid[i] == 0) continue;
-      const double d = static_cast<double>(rewards[i]) - mu;
-      sq += d * d;
-    }
-    sq = warp_sum(sq);
-    const double denom = sqrt(sq / k) + adv_eps;
-    for (int i = b + lane; i < e; i += 32) {
-      if (traj_valid && traj_valid[i] == 0) continue;
-      adv_out[i] = static_cast<float>((static_cast<double>(rewards[i]) - mu) / denom);
-    }
+// A_i for the members of group g (one warp): mean and population standard deviation of the
+// valid members' rewards in double precision, each A_i rounded once to float. Invalid members,
+// and every member of a group with no valid member or whose valid rewards are all equal, get 0.
+__device__ __forceinline__ void group_advantage(int64_t g, int lane, int32_t n_traj, const int32_t* group_offsets,
+                                                const float* rewards, const uint8_t* traj_valid, double adv_eps,
+                                                float* adv_out, int32_t* status) {
+  const int b = group_offsets[g], e = group_offsets[g + 1];
+  if (b < 0 || e < b || e > n_traj) {
+    if (lane == 0) flag_status(status, RL_DEV_BAD_OFFSETS);
+    return;
   }
+  // pass 1: count, sum, and min / max (all-equal test) over valid members
+  int k = 0;
+  double sum = 0.0;
+  float lo = __int_as_float(0x7f800000), hi = -__int_as_float(0x7f800000);
+  for (int i = b + lane; i < e; i += 32) {
+    if (traj_valid && traj_valid[i] == 0) continue;
+    const float r = rewards[i];
+    ++k;
+    sum += static_cast<double>(r);
+    lo = fminf(lo, r);
+    hi = fmaxf(hi, r);
+  }
+  k = warp_sum(k);
+  sum = warp_sum(sum);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+    hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+  }
+  if (k == 0 || lo == hi) {  // nothing valid, or all valid rewards equal: A = 0
+    for (int i = b + lane; i < e; i += 32) adv_out[i] = 0.f;
+    return;
+  }
+  const double mu = sum / k;
+  double sq = 0.0;
+  for (int i = b + lane; i < e; i += 32) {
+    if (traj_valid && traj_valid[i] == 0) continue;
+    const double d = static_cast<double>(rewards[i]) - mu;
+    sq += d * d;
+  }
+  sq = warp_sum(sq);
+  const double denom = sqrt(sq / k) + adv_eps;
+  for (int i = b + lane; i < e; i += 32) {
+    const bool valid = !traj_valid || traj_valid[i] != 0;
+    adv_out[i] = valid ? static_cast<float>((static_cast<double>(rewards[i]) - mu) / denom) : 0.f;
+  }
+}
 
-  // N = number of valid trajectories with L_i > 0; S = sum of their L_i
-  __shared__ long long red_n[kWarps], red_s[kWarps];
+struct CountAdvArgs {
+  int32_t n_traj, n_groups;
+  int64_t n_tokens;
+  int64_t count_blocks;            // CTAs [0, count_blocks) count, the rest form advantages
+  const int64_t* traj_offsets;     // spans (rl_group_advantages)
+  const int32_t* token_traj;       // owners (rl_group_advantages_by_owner)
+  const uint8_t* mask;
+  const int32_t* group_offsets;
+  const float* rewards;
+  const uint8_t* traj_valid;
+  double adv_eps;
+  float* adv_out;
+  float* coef_out;
+  int32_t* n_tok_out;
+  int32_t* token_traj_out;
+  int32_t* status;
+};
+
+template <bool BY_OWNER>
+__global__ void __launch_bounds__(kAdvThreads) count_adv_kernel(const CountAdvArgs a) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (blockIdx.x < a.count_blocks) {
+    const int64_t w = static_cast<int64_t>(blockIdx.x) * kAdvWarps + warp;
+    if (BY_OWNER) {
+      count_owners(w, a.count_blocks * kAdvWarps, lane, a.n_tokens, a.token_traj, a.mask, a.n_traj, a.n_tok_out,
+                   a.status);
+    } else if (w < a.n_traj) {
+      count_span(w, lane, a.n_tokens, a.traj_offsets, a.mask, a.n_tok_out, a.token_traj_out, a.status);
+    }
+  } else {
+    const int64_t g = (static_cast<int64_t>(blockIdx.x) - a.count_blocks) * kAdvWarps + warp;
+    if (g < a.n_groups)
+      group_advantage(g, lane, a.n_traj, a.group_offsets, a.rewards, a.traj_valid, a.adv_eps, a.adv_out, a.status);
+  }
+}
+
+// Coefficients c_i (Sec. 2.3.2: 1 / (N L_i) under seq-mean-token-mean; 1 / S under token-mean;
+// 1 under token-sum) for valid trajectories with L_i > 0, else 0; A = 0 for trajectories
+// before the first group or after the last.
+__global__ void __launch_bounds__(kAdvThreads) coef_kernel(int32_t n_traj, int32_t n_groups,
+                                                           const int32_t* __restrict__ group_offsets,
+                                                           const uint8_t* __restrict__ traj_valid,
+                                                           const int32_t* __restrict__ n_tok, int32_t loss_agg,
+                                                           float* __restrict__ adv_out, float* __restrict__ coef_out) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  __shared__ long long red_n[kAdvWarps], red_s[kAdvWarps];
   long long cnt = 0, tok = 0;
+#pragma unroll 4
   for (int i = tid; i < n_traj; i += kAdvThreads) {
-    const bool counted = (!traj_valid || traj_valid[i] != 0) && n_tok[i] > 0;
+    const int32_t L = n_tok[i];
+    const bool counted = (!traj_valid || traj_valid[i] != 0) && L > 0;
     cnt += counted;
-    tok += counted ? n_tok[i] : 0;
+    tok += counted ? L : 0;
   }
   cnt = warp_sum(cnt);
   tok = warp_sum(tok);
@@ -139,11 +184,18 @@ __global__ void __launch_bounds__(kAdvThreads) group_adv_kernel(
   }
   __syncthreads();
   long long N = 0, S = 0;
-  for (int w = 0; w < kWarps; ++w) {
+  for (int w = 0; w < kAdvWarps; ++w) {
     N += red_n[w];
     S += red_s[w];
   }
-  for (int i = tid; i < n_traj; i += kAdvThreads) {
+  int32_t first = n_traj, last = n_traj;  // trajectories [first, last) belong to groups
+  if (n_groups > 0) {
+    first = min(max(group_offsets[0], 0), n_traj);
+    last = min(max(group_offsets[n_groups], first), n_traj);
+  }
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * kAdvThreads + tid; i < n_traj;
+       i += static_cast<int64_t>(gridDim.x) * kAdvThreads) {
+    if (i < first || i >= last) adv_out[i] = 0.f;
     const int32_t L = n_tok[i];
     const bool counted = (!traj_valid || traj_valid[i] != 0) && L > 0;
     float c = 0.f;
@@ -157,6 +209,29 @@ __global__ void __launch_bounds__(kAdvThreads) group_adv_kernel(
     }
     coef_out[i] = c;
   }
+}
+
+// Launches count_adv_kernel (count_blocks counting CTAs, then one warp per group) and
+// coef_kernel on stream s.
+template <bool BY_OWNER>
+static rl_status launch_advantages(CountAdvArgs a, int64_t count_blocks, const rl_loss_params* params, const char* fn,
+                                   cudaStream_t s) {
+  a.count_blocks = count_blocks;
+  const int64_t adv_blocks = (static_cast<int64_t>(a.n_groups) + kAdvWarps - 1) / kAdvWarps;
+  const int64_t blocks = count_blocks + adv_blocks;
+  if (blocks > 0) {
+    count_adv_kernel<BY_OWNER><<<static_cast<unsigned>(blocks), kAdvThreads, 0, s>>>(a);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_error(e, (std::string(fn) + ": count_adv_kernel launch").c_str());
+  }
+  // every CTA reads all n_tok once for N and S: a few CTAs per wave of the GPU at most
+  int64_t cb = (static_cast<int64_t>(a.n_traj) + kAdvThreads - 1) / kAdvThreads;
+  if (cb > 152) cb = 152;
+  coef_kernel<<<static_cast<unsigned>(cb), kAdvThreads, 0, s>>>(a.n_traj, a.n_groups, a.group_offsets, a.traj_valid,
+                                                                 a.n_tok_out, params->loss_agg, a.adv_out, a.coef_out);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_error(e, (std::string(fn) + ": coef_kernel launch").c_str());
+  return RL_OK;
 }
 
 }  // namespace rl
@@ -184,19 +259,24 @@ extern "C" rl_status rl_group_advantages(int32_t n_traj, int32_t n_groups, const
     return set_error(RL_ERR_INVALID_ARG, "rl_group_advantages: NULL array argument");
   if (n_tokens > 0 && !mask) return set_error(RL_ERR_INVALID_ARG, "rl_group_advantages: mask is NULL");
   if (n_tokens > INT32_MAX) return set_error(RL_ERR_UNSUPPORTED, "rl_group_advantages: more than 2^31 - 1 tokens");
-  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  int32_t* status = reinterpret_cast<int32_t*>(ws);
-  const int warps_per_block = 256 / 32;
-  const unsigned blocks = static_cast<unsigned>((static_cast<int64_t>(n_traj) + warps_per_block - 1) / warps_per_block);
-  traj_count_kernel<<<blocks, 256, 0, s>>>(n_traj, n_tokens, traj_offsets, mask, n_tok_out, token_traj_out, status);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return cuda_error(e, "rl_group_advantages: traj_count_kernel launch");
-  group_adv_kernel<<<1, kAdvThreads, 0, s>>>(n_traj, n_groups, group_offsets, rewards, traj_valid, n_tok_out,
-                                             static_cast<double>(params->adv_eps), params->loss_agg, adv_out,
-                                             coef_out, status);
-  e = cudaGetLastError();
-  if (e != cudaSuccess) return cuda_error(e, "rl_group_advantages: group_adv_kernel launch");
-  return RL_OK;
+  CountAdvArgs a = {};
+  a.n_traj = n_traj;
+  a.n_groups = n_groups;
+  a.n_tokens = n_tokens;
+  a.traj_offsets = traj_offsets;
+  a.mask = mask;
+  a.group_offsets = group_offsets;
+  a.rewards = rewards;
+  a.traj_valid = traj_valid;
+  a.adv_eps = static_cast<double>(params->adv_eps);
+  a.adv_out = adv_out;
+  a.coef_out = coef_out;
+  a.n_tok_out = n_tok_out;
+  a.token_traj_out = token_traj_out;
+  a.status = reinterpret_cast<int32_t*>(ws);
+  const int64_t count_blocks = (static_cast<int64_t>(n_traj) + kAdvWarps - 1) / kAdvWarps;  // a warp per span
+  return launch_advantages<false>(a, count_blocks, params, "rl_group_advantages",
+                                  reinterpret_cast<cudaStream_t>(stream));
 }
 
 extern "C" rl_status rl_group_advantages_by_owner(int32_t n_traj, int32_t n_groups, const int32_t* group_offsets,
@@ -222,21 +302,24 @@ extern "C" rl_status rl_group_advantages_by_owner(int32_t n_traj, int32_t n_grou
   if (!rewards || !adv_out || !coef_out || !n_tok_out || (n_tokens > 0 && (!token_traj || !mask)))
     return set_error(RL_ERR_INVALID_ARG, "rl_group_advantages_by_owner: NULL array argument");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  int32_t* status = reinterpret_cast<int32_t*>(ws);
   cudaError_t e = cudaMemsetAsync(n_tok_out, 0, static_cast<size_t>(n_traj) * sizeof(int32_t), s);
   if (e != cudaSuccess) return cuda_error(e, "rl_group_advantages_by_owner: cudaMemsetAsync");
-  if (n_tokens > 0) {
-    int64_t blocks = (n_tokens + 255) / 256;
-    if (blocks > 152 * 8) blocks = 152 * 8;
-    owner_count_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(n_tokens, token_traj, mask, n_traj, n_tok_out,
-                                                                     status);
-    e = cudaGetLastError();
-    if (e != cudaSuccess) return cuda_error(e, "rl_group_advantages_by_owner: owner_count_kernel launch");
-  }
-  group_adv_kernel<<<1, kAdvThreads, 0, s>>>(n_traj, n_groups, group_offsets, rewards, traj_valid, n_tok_out,
-                                             static_cast<double>(params->adv_eps), params->loss_agg, adv_out,
-                                             coef_out, status);
-  e = cudaGetLastError();
-  if (e != cudaSuccess) return cuda_error(e, "rl_group_advantages_by_owner: group_adv_kernel launch");
-  return RL_OK;
+  CountAdvArgs a = {};
+  a.n_traj = n_traj;
+  a.n_groups = n_groups;
+  a.n_tokens = n_tokens;
+  a.token_traj = token_traj;
+  a.mask = mask;
+  a.group_offsets = group_offsets;
+  a.rewards = rewards;
+  a.traj_valid = traj_valid;
+  a.adv_eps = static_cast<double>(params->adv_eps);
+  a.adv_out = adv_out;
+  a.coef_out = coef_out;
+  a.n_tok_out = n_tok_out;
+  a.status = reinterpret_cast<int32_t*>(ws);
+  // grid-stride over 32-token runs: at most 8 CTAs per SM
+  int64_t count_blocks = (n_tokens + kAdvThreads - 1) / kAdvThreads;
+  if (count_blocks > 152 * 8) count_blocks = 152 * 8;
+  return launch_advantages<true>(a, count_blocks, params, "rl_group_advantages_by_owner", s);
 }

@@ -115,6 +115,32 @@ def test_group_advantages_parity(R, name, n_groups, invalid, agg):
     assert np.all(a[lay.traj_valid == 0] == 0) and np.all(c[lay.traj_valid == 0] == 0)
 
 
+@pytest.mark.parametrize("go", [[2, 5, 8], [0], [0, 10], [0, 1, 2, 3, 4, 5, 6, 7, 8, 9, 10]])
+def test_group_advantages_outside_groups_and_one_member_groups(R, go):
+    """Trajectories before the first group or after the last keep A = 0 (also with no group at
+    all), one-member groups give A = 0, and the coefficients count every trajectory."""
+    rng = np.random.default_rng(len(go))
+    n = 10
+    rewards = rng.random(n).astype(np.float32)
+    traj_offsets = np.cumsum([0] + list(rng.integers(0, 6, n))).astype(np.int64)
+    mask = (rng.random(int(traj_offsets[-1])) < 0.7).astype(np.uint8)
+    group_offsets = np.array(go, np.int32)
+    P = O.LossParams(loss_agg=0)
+    adv, coef, L, tt = O.advantages_and_coefficients(rewards, group_offsets, traj_offsets, mask, None, P)
+    ws = R.new_workspace(0, 0)
+    a, c, n_tok, tt_d = R.rl_group_advantages(to_dev(group_offsets), to_dev(rewards), to_dev(traj_offsets),
+                                              to_dev(mask), cuda_params(R, P), ws)
+    assert R.rl_query_status(ws)[1] == 0
+    assert np.array_equal(n_tok.cpu().numpy(), L) and np.array_equal(tt_d.cpu().numpy(), tt)
+    a, c = a.cpu().numpy().astype(np.float64), c.cpu().numpy().astype(np.float64)
+    assert np.all(np.abs(a - adv) <= 2.0 ** -23 * np.abs(adv)), (a, adv)
+    assert np.all(np.abs(c - coef) <= 2.0 ** -23 * np.abs(coef)), (c, coef)
+    inside = np.zeros(n, bool)
+    if len(go):
+        inside[go[0]:go[-1]] = True
+    assert np.all(a[~inside] == 0.0)
+
+
 def test_group_advantages_bad_offsets_flagged(R):
     go = to_dev(np.array([0, 3, 2], np.int32))   # decreasing
     rw = to_dev(np.zeros(3, np.float32))
