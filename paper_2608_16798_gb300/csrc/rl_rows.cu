@@ -20,6 +20,9 @@
 // from HBM exactly once and its gradient written once; masked rows (and rows of
 // trajectories with c_i = 0) are not read at all, only zero-filled.
 //
+// Rows of at most 8 KB (V <= 4,096 bf16 or 2,048 fp32) take a lighter form of the
+// loss kernel, a warp per row with the row held in registers (small_rows_kernel).
+//
 // The kernels are persistent: the grid holds as many clusters as fit on the
 // GPU at once, and cluster j processes rows j, j + n_clusters, ... . Each
 // cluster adds its rows' loss contributions in row order and leaves one partial
@@ -763,6 +766,178 @@ __global__ void __launch_bounds__((NW + 1) * 32, MINB) rows_kernel(const RowArgs
   if (C > 1) cluster_sync_all();
 }
 
+// ------------------------------------------------------------------ short rows
+//
+// For rows of at most kSmallRowBytes (V <= 4,096 bf16 or 2,048 fp32) a cluster of CTAs per row
+// costs more in set-up and exchange than the row's own data. Here one warp owns a row: its lanes
+// hold the row in registers (vector j = lane + 32 k in x[k]), fold it with the same online
+// softmax as the cluster kernel, merge the 32 partials by shuffles, and write the gradient from
+// registers. Warps take rows w, w + (all warps), ...; each warp adds its rows' loss terms in row
+// order, the CTA adds its warps' sums in warp order into one partial, and the last CTA to finish
+// (the same workspace counter as the cluster kernel's) adds the CTAs' partials, in order, into
+// the caller's total.
+constexpr int64_t kSmallRowBytes = 8192;
+constexpr int kSmallWarps = 8;
+
+template <typename T, bool ENT>
+__global__ void __launch_bounds__(kSmallWarps * 32, 2) small_rows_kernel(const RowArgs p) {
+  constexpr int EPV = Vec<T>::N;
+  constexpr int NV = static_cast<int>(kSmallRowBytes / 16 / 32);  // 16-byte vectors a lane holds
+  __shared__ double warp_loss[kSmallWarps];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t all_warps = static_cast<int64_t>(gridDim.x) * kSmallWarps;
+  const int64_t V = p.V, ld = p.ld;
+  const int nv = static_cast<int>(V / EPV);  // full vectors of a row
+  const uint32_t pad = Vec<T>::kPadWord;
+  const T* logits = static_cast<const T*>(p.logits);
+  T* grad = static_cast<T*>(p.grad);
+  double w_loss = 0.0;  // lane 0: this warp's rows' c l, in row order
+  for (int64_t r = static_cast<int64_t>(blockIdx.x) * kSmallWarps + warp; r < p.rows; r += all_warps) {
+    // ---- which rows are trained on (the same tests, in the same order, as the cluster kernel).
+    // The row's own words are loaded at once; then its owner's coefficient and advantage together
+    // with the row's logits (when the row is masked in and its owner in range), so that a row
+    // costs two dependent trips to memory before its arithmetic.
+    const int32_t a = p.token_ids[r];
+    const uint32_t mk = p.mask[r];
+    const int32_t i = p.token_traj[r];
+    const float old = p.old_logp[r];
+    const float ref = p.ref_logp ? p.ref_logp[r] : 0.f;
+    const float roll = p.rollout_logp ? p.rollout_logp[r] : 0.f;
+    const float A_row = p.adv_per_row ? p.adv[r] : 0.f;
+    const bool owner_ok = i >= 0 && i < p.n_traj;
+    const bool fetch = mk != 0 && owner_ok;
+    const T* row = logits + r * ld;
+    auto reload = [&](int k) {
+      const int j = lane + k * 32;
+      return j < nv ? reinterpret_cast<const uint4*>(row)[j] : make_uint4(pad, pad, pad, pad);
+    };
+    uint4 x[NV];
+    float c = 0.f, A = 0.f;
+    if (fetch) {
+      c = p.coef[i];
+      A = p.adv_per_row ? A_row : p.adv[i];
+#pragma unroll
+      for (int k = 0; k < NV; ++k) x[k] = reload(k);
+    }
+    bool active = fetch && c != 0.f;
+    if (mk != 0 && !owner_ok && lane == 0) flag_status(p.status, RL_DEV_BAD_TRAJ);
+    if (active && (a < 0 || a >= V)) {
+      if (lane == 0) flag_status(p.status, RL_DEV_BAD_TOKEN);
+      active = false;
+    }
+    T* g_row = grad + r * ld;
+    if (!active) {
+      for (int j = lane; j < nv; j += 32) st_global_16(g_row + j * EPV, make_uint4(0u, 0u, 0u, 0u));
+      for (int64_t e = static_cast<int64_t>(nv) * EPV + lane; e < V; e += 32) g_row[e] = T(0);
+      if (lane == 0 && p.token_stats)
+        for (int k = 0; k < 5; ++k) p.token_stats[r * 5 + k] = 0.f;
+      continue;
+    }
+    const float za = Vec<T>::to_f(row[a]);
+    // ---- pass 1: the lane's partial, then the warp's (lane 0's merge, broadcast)
+    SoftmaxPartial ps{RL_NEG_INF, 0.f, 0.f};
+    fold_block<T, ENT>(ps, x, reload);
+    float tail_z = 0.f;
+    const int64_t te = static_cast<int64_t>(nv) * EPV + lane;  // ragged tail: one element per lane at most
+    if (te < V) {
+      const float z = Vec<T>::to_f(row[te]);
+      tail_z = z;
+      if (z != RL_NEG_INF) {
+        raise_max<ENT>(ps, z);
+        accumulate<ENT>(ps, z, -ps.m * kLog2e);
+      }
+    }
+    SoftmaxPartial q = warp_merge(ps);
+    q.m = __shfl_sync(0xffffffffu, q.m, 0);
+    q.s = __shfl_sync(0xffffffffu, q.s, 0);
+    q.u = __shfl_sync(0xffffffffu, q.u, 0);
+    const float lnS = logf(q.s);
+    const float lse = q.m + lnS;
+    const float H = lnS - q.u / q.s;
+    // ---- per-token scalars (every lane computes the same values)
+    const float logp = za - lse;
+    const float rho = expf((za - old) - lse);  // large operands differenced first
+    const float crho = fminf(fmaxf(rho, p.clip_lo), p.clip_hi);
+    const float surr = fminf(rho * A, crho * A);
+    const bool cut = (A > 0.f && rho > p.clip_hi) || (A < 0.f && rho < p.clip_lo);
+    const float w = (p.tis_cap > 0.f && p.rollout_logp) ? fminf(expf(old - roll), p.tis_cap) : 1.f;
+    float kl = 0.f, dkl = 0.f;
+    if (p.beta != 0.f && p.ref_logp) {
+      const float d = (ref - za) + lse;  // r - logp
+      const float ed = expf(d);
+      kl = ed - d - 1.f;
+      dkl = 1.f - ed;
+    }
+    const float ell = -w * surr + p.beta * kl - p.alpha * H;
+    const float g = (cut ? 0.f : -w * A * rho) + p.beta * dkl;
+    const float cg = c * g, ca0 = c * p.alpha;
+    // p_v = 2^(z_v log2(e) + nl), the rounding of nl folded into the coefficients (as in the
+    // cluster kernel)
+    const float nl = -lse * kLog2e;
+    const float fl = fmaf(fmaf(-lse, kLog2e, -nl), kLn2, 1.f);
+    const float Kp = -cg * fl;
+    const float ca = ca0 * fl;
+    const float Ke = (-cg + ca0 * (H - lse)) * fl;
+    if (lane == 0) {
+      w_loss += static_cast<double>(c) * static_cast<double>(ell);
+      if (p.token_stats) {
+        float* st = p.token_stats + r * 5;
+        st[0] = logp; st[1] = rho; st[2] = cut ? 1.f : 0.f; st[3] = H; st[4] = kl;
+      }
+    }
+    __syncwarp();  // every lane has read z_a before any lane overwrites it (in-place gradients)
+    // ---- pass 2: gradient from the registers
+    constexpr int NP = Vec<T>::NP;
+    const float2 l2 = make_float2(kLog2e, kLog2e), nl2 = make_float2(nl, nl);
+    const float2 kp2 = make_float2(Kp, Kp), ca2 = make_float2(ca, ca), ke2 = make_float2(Ke, Ke);
+#pragma unroll
+    for (int k = 0; k < NV; ++k) {
+      const int j = lane + k * 32;
+      float2 qv[NP], o[NP];
+      Vec<T>::pairs(x[k], qv);
+#pragma unroll
+      for (int i = 0; i < NP; ++i) {
+        const float2 xx = __ffma2_rn(qv[i], l2, nl2);
+        const float2 pk = make_float2(ex2(xx.x), ex2(xx.y));
+        if (ENT) {
+          const float2 zc = make_float2(fmaxf(qv[i].x, -1e30f), fmaxf(qv[i].y, -1e30f));
+          o[i] = __fmul2_rn(pk, __ffma2_rn(ca2, zc, ke2));
+        } else {
+          o[i] = __fmul2_rn(kp2, pk);
+        }
+      }
+      if (j < nv) st_global_16(g_row + j * EPV, Vec<T>::pack_pairs(o));
+    }
+    if (te < V) {
+      const float pk = ex2(fmaf(tail_z, kLog2e, nl));
+      Vec<T>::store_scalar(g_row + te, ENT ? pk * fmaf(ca, fmaxf(tail_z, -1e30f), Ke) : Kp * pk);
+    }
+    // the sampled token's element gets + c g; rewritten by the lane that stored it
+    const int writer = a < nv * EPV ? (a / EPV) % 32 : (a - nv * EPV);
+    if (lane == writer) {
+      const float pk = ex2(fmaf(za, kLog2e, nl));
+      Vec<T>::store_scalar(g_row + a, (ENT ? pk * fmaf(ca, fmaxf(za, -1e30f), Ke) : Kp * pk) + cg);
+    }
+  }
+  // ---- the loss: warps in order into one partial per CTA; the last CTA adds the partials
+  if (lane == 0) warp_loss[warp] = w_loss;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double t = 0.0;
+    for (int k = 0; k < kSmallWarps; ++k) t += warp_loss[k];
+    p.row_loss[blockIdx.x] = t;
+    __threadfence();
+    const bool last = atomicAdd(p.done, 1u) == gridDim.x - 1;
+    if (last) {
+      __threadfence();
+      double sum = 0.0;
+      for (unsigned k = 0; k < gridDim.x; ++k) sum += __ldcg(p.row_loss + k);
+      *p.loss_accum += sum;
+      *p.done = 0u;
+    }
+  }
+}
+
 // ------------------------------------------------------------------ forward-only stream
 //
 // rl_token_logprobs reads each row exactly once and keeps nothing on chip, so it
@@ -1071,8 +1246,48 @@ static bool loss_plan(int64_t V, bool ent, Plan* plan) {
 // one loss partial at the head of the per-row loss area (the last one also adds them up).
 // Registers hold the slice when it fits the path's held vectors; otherwise the slice stays in
 // shared memory (7 warps, 2 CTAs per SM, slices up to 40 KB).
+// Launches the short-row kernel: as many CTAs as fit on the GPU at once, at most one warp per row.
+template <typename T, bool ENT>
+static rl_status launch_small(const RowArgs& args, cudaStream_t s) {
+  auto kern = small_rows_kernel<T, ENT>;
+  constexpr int kThreads = kSmallWarps * 32;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_error(e, "cudaGetDevice");
+  static std::mutex mu;
+  static std::map<std::pair<const void*, int>, int64_t> grid_cache;
+  int64_t grid = 0;
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    auto key = std::make_pair(reinterpret_cast<const void*>(kern), dev);
+    auto it = grid_cache.find(key);
+    if (it != grid_cache.end()) {
+      grid = it->second;
+    } else {
+      int per_sm = 0, sms = 0;
+      e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, 0);
+      if (e != cudaSuccess) return cuda_error(e, "cudaOccupancyMaxActiveBlocksPerMultiprocessor");
+      e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+      if (e != cudaSuccess) return cuda_error(e, "cudaDeviceGetAttribute");
+      if (per_sm <= 0) return set_error(RL_ERR_UNSUPPORTED, "small_rows_kernel does not fit on an SM");
+      grid = static_cast<int64_t>(per_sm) * sms;
+      grid_cache[key] = grid;
+    }
+  }
+  const int64_t blocks = std::min<int64_t>(grid, (args.rows + kSmallWarps - 1) / kSmallWarps);
+  kern<<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(args);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_error(e, "small_rows_kernel launch");
+  return RL_OK;
+}
+
 template <typename T>
 static rl_status dispatch_loss(bool ent, RowArgs args, int64_t V, cudaStream_t s, int64_t* n_clusters) {
+  // rows of at most 8 KB (16-byte aligned): a warp per row
+  if (args.tma && V * static_cast<int64_t>(sizeof(T)) <= kSmallRowBytes) {
+    *n_clusters = 0;
+    return ent ? launch_small<T, true>(args, s) : launch_small<T, false>(args, s);
+  }
   auto run = [&](const Plan& plan, auto launcher) {
     args.slice = plan.slice;
     args.buf_elems = plan.buf_elems;

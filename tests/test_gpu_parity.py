@@ -115,14 +115,15 @@ def test_group_advantages_parity(R, name, n_groups, invalid, agg):
     assert np.all(a[lay.traj_valid == 0] == 0) and np.all(c[lay.traj_valid == 0] == 0)
 
 
+@pytest.mark.parametrize("scale", [1, 20000])  # a few tokens per trajectory, or tens of thousands
 @pytest.mark.parametrize("go", [[2, 5, 8], [0], [0, 10], [0, 1, 2, 3, 4, 5, 6, 7, 8, 9, 10]])
-def test_group_advantages_outside_groups_and_one_member_groups(R, go):
+def test_group_advantages_outside_groups_and_one_member_groups(R, go, scale):
     """Trajectories before the first group or after the last keep A = 0 (also with no group at
     all), one-member groups give A = 0, and the coefficients count every trajectory."""
     rng = np.random.default_rng(len(go))
     n = 10
     rewards = rng.random(n).astype(np.float32)
-    traj_offsets = np.cumsum([0] + list(rng.integers(0, 6, n))).astype(np.int64)
+    traj_offsets = np.cumsum([0] + list(rng.integers(0, 6, n) * scale)).astype(np.int64)
     mask = (rng.random(int(traj_offsets[-1])) < 0.7).astype(np.uint8)
     group_offsets = np.array(go, np.int32)
     P = O.LossParams(loss_agg=0)
@@ -212,6 +213,21 @@ def test_policy_loss_ragged_shapes(R, vocab, ld_pad, dtype_case):
     compare(case, out, f"V={vocab} ld=V+{ld_pad}")
 
 
+@pytest.mark.parametrize("name,vocab,ld_pad,rows,agg,tis", [
+    ("longhorizon", 4096, 0, 3000, 2, True),  # entropy + k3 KL + TIS; many rows per warp
+    ("multiturn", 4096, 0, 6000, 0, False),   # 40% masked rows, the paper's weighting
+    ("edge", 2048, 0, 2000, 2, False),        # fp32 at the 8 KB limit
+    ("tiny", 37, 3, 200, 2, False),           # four vectors and a ragged tail of five
+    ("longhorizon", 4104, 0, 300, 2, False),  # bf16 rows just over 8 KB: one CTA per row
+    ("edge", 2049, 3, 300, 2, True)])         # fp32 rows just over 8 KB, 16-byte aligned
+def test_policy_loss_short_rows(R, name, vocab, ld_pad, rows, agg, tis):
+    """Rows of at most 8 KB (aligned) take the warp-per-row kernel; rows just over it take the
+    cluster kernel with one CTA per row. Both against the oracle, with the workloads' masks."""
+    case = make_case(name, seed=21, row0=0, rows=rows, vocab=vocab, loss_agg=agg, tis=tis)
+    out = run_loss(R, case, ld=vocab + ld_pad)
+    compare(case, out, f"{name} V={vocab} ld=V+{ld_pad} rows={rows}")
+
+
 @pytest.mark.parametrize("name,row0,rows", [("tiny", 0, 1), ("multiturn", 100, 1), ("edge", 3, 2), ("multiturn", 0, 3)])
 def test_policy_loss_fewest_rows(R, name, row0, rows):
     """One to three rows: a single cluster (or as many as rows), whose last one sums the loss."""
@@ -225,8 +241,9 @@ def test_policy_loss_fewest_rows(R, name, row0, rows):
     assert np.all(np.abs(H.cpu().numpy() - H_ref) <= 5e-5 + 2e-5 * np.abs(H_ref))
 
 
-def test_policy_loss_in_place_and_deterministic(R):
-    case = make_case("multiturn", seed=5, row0=300, rows=64, loss_agg=2)
+@pytest.mark.parametrize("name,row0,rows", [("multiturn", 300, 64), ("tiny", 0, 512)])
+def test_policy_loss_in_place_and_deterministic(R, name, row0, rows):
+    case = make_case(name, seed=5, row0=row0, rows=rows, loss_agg=2)
     a = run_loss(R, case)
     b = run_loss(R, case, in_place=True)
     c = run_loss(R, case)
@@ -235,12 +252,14 @@ def test_policy_loss_in_place_and_deterministic(R):
     compare(case, b, "in place")
 
 
-def test_policy_loss_microbatch_split(R):
-    case = make_case("longhorizon", seed=6, row0=2000, rows=80, loss_agg=0)
+@pytest.mark.parametrize("name,row0,rows,vocab", [("longhorizon", 2000, 80, None), ("longhorizon", 100, 2000, 4096)])
+def test_policy_loss_microbatch_split(R, name, row0, rows, vocab):
+    case = make_case(name, seed=6, row0=row0, rows=rows, vocab=vocab, loss_agg=0)
     whole = run_loss(R, case)
     parts = []
-    for lo, hi in ((0, 33), (33, 80)):
-        sub = make_case("longhorizon", seed=6, row0=2000 + lo, rows=hi - lo, loss_agg=0)
+    cut = rows * 2 // 5 + 1
+    for lo, hi in ((0, cut), (cut, rows)):
+        sub = make_case(name, seed=6, row0=row0 + lo, rows=hi - lo, vocab=vocab, loss_agg=0)
         # the same rows: the generator is keyed by row, only the noise streams differ -> reuse the parent's
         sub.raw, sub.ids, sub.old = case.raw[lo:hi], case.ids[lo:hi], case.old[lo:hi]
         sub.ref = None if case.ref is None else case.ref[lo:hi]
@@ -338,7 +357,8 @@ def neg_inf_case(name, rows, seed=6, entropy=False, fill="-inf"):
 
 @pytest.mark.parametrize("name,entropy,fill", [("longhorizon", False, "-inf"), ("multiturn", True, "-inf"),
                                                ("edge", True, "-inf"), ("multiturn", False, "-inf"),
-                                               ("longhorizon", True, "max_finite"), ("edge", True, "max_finite")])
+                                               ("longhorizon", True, "max_finite"), ("edge", True, "max_finite"),
+                                               ("tiny", True, "-inf"), ("tiny", False, "max_finite")])
 def test_policy_loss_neg_inf_logits(R, name, entropy, fill):
     case = neg_inf_case(name, 64, entropy=entropy, fill=fill)
     out = run_loss(R, case)
