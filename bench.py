@@ -225,15 +225,20 @@ def time_other_workloads(torch, R, dev, peak, reps=10, oracle_slices=None):
     whole batch (512 trajectories in 32 groups; 16,384 in 4,096 groups) as CUDA-graph replays. The logits stay resident (20 and 17 GB, far
     above L2); pi_old comes from the library's forward pass plus the workload's noise. With
     `oracle_slices` (a dict), bounded spans of the same device rows are copied to the host for
-    the CPU oracle's timing: 4,096 rows of each long-horizon microbatch, the first 32,768 edge
-    rows, the whole tiny batch."""
+    the CPU oracle's timing: 4,096 rows at the start of each of the two timed long-horizon
+    microbatches and of the last (partial) one, drawn on the device like the others, the whole
+    edge batch, the whole tiny batch."""
     t = torch
     out = {}
-    for name, picks in (("longhorizon", (0, None)), ("edge", (0,))):
+    # (microbatch, timed): the last long-horizon microbatch is partial (18,951 rows), so only the
+    # CPU oracle's sample takes rows from it
+    for name, picks in (("longhorizon", (("first", True), ("middle", True), ("last", False))),
+                        ("edge", (("first", True),))):
         w = W.WORKLOADS[name]
         lay = W.make_layout(w, 0)
         mbs = W.microbatches(lay, w.microbatch)
-        chosen = [mbs[0] if k == 0 else mbs[len(mbs) // 2] for k in picks]
+        where = {"first": mbs[0], "middle": mbs[len(mbs) // 2], "last": mbs[-1]}
+        chosen = [(where[k], timed) for k, timed in picks]
         dt = t.bfloat16 if w.dtype == "bf16" else t.float32
         es = 2 if w.dtype == "bf16" else 4
         d = lambda x: t.from_numpy(np.ascontiguousarray(x)).to(dev)  # noqa: E731
@@ -249,8 +254,10 @@ def time_other_workloads(torch, R, dev, peak, reps=10, oracle_slices=None):
                                                                   adv_out=adv, coef_out=coef, n_tok_out=n_tok,
                                                                   token_traj_out=tt), 20)
         items, nbytes, rows_total = [], 0, 0
-        for lo, hi in chosen:
-            n = hi - lo
+        for (lo, hi), timed in chosen:
+            if not timed and oracle_slices is None:
+                continue
+            n = hi - lo if timed else min(hi - lo, ORACLE_ROWS[name])
             logits = t.empty((n, w.vocab), dtype=dt, device=dev)
             W.logits_rows_torch(w, 0, lo, n, logits)
             ids = W.sample_tokens_torch(logits, 0, lo, w)
@@ -261,6 +268,8 @@ def time_other_workloads(torch, R, dev, peak, reps=10, oracle_slices=None):
             if oracle_slices is not None:
                 n_or = min(n, ORACLE_ROWS[name])
                 oracle_slices.setdefault(name, []).append((lo, logits[:n_or], ids[:n_or]))
+            if not timed:
+                continue
             grad = t.empty_like(logits)
             trained = (lay.mask[lo:hi] != 0) & (coef_h[tt_h[lo:hi]] != 0)
             nbytes += int((trained.astype(np.int64) + 1).sum()) * w.vocab * es
@@ -303,7 +312,7 @@ def time_other_workloads(torch, R, dev, peak, reps=10, oracle_slices=None):
 
 
 # rows of each span the CPU oracle is timed on, and the objective's parameters there
-ORACLE_ROWS = {"longhorizon": 4096, "edge": 32768, "tiny": 512}
+ORACLE_ROWS = {"longhorizon": 4096, "edge": 131072, "tiny": 512}
 ORACLE_PARAMS = {"longhorizon": {"kl_coef": 1e-3, "kl_estimator": 3, "entropy_coef": 1e-3}, "edge": {}, "tiny": {}}
 ORACLE_HEAD_TOKENS = 1024
 
@@ -826,13 +835,20 @@ class OracleSlice:
         self.shm.unlink()
 
 
-def make_oracle_slice(w, pieces, params):
+def make_oracle_slice(w, pieces, params, fallback_rows=32768):
     """An OracleSlice, or the reason it could not be made (host or shared memory short): the
-    CPU leg's extra samples never cost the benchmark its line."""
+    CPU leg's extra samples never cost the benchmark its line. When the whole span does not fit,
+    the first `fallback_rows` rows of the first span are tried instead."""
     try:
         return OracleSlice(w, pieces, params)
     except (OSError, MemoryError) as e:
-        return f"{type(e).__name__}: {e}"
+        if not pieces or int(pieces[0][1].shape[0]) <= fallback_rows:
+            return f"{type(e).__name__}: {e}"
+        lo, lg, ids = pieces[0]
+        try:
+            return OracleSlice(w, [(lo, lg[:fallback_rows], ids[:fallback_rows])], params)
+        except (OSError, MemoryError) as e2:
+            return f"{type(e2).__name__}: {e2}"
 
 
 class OraclePool:
@@ -890,8 +906,9 @@ def time_oracle_slice(sl):
         op.close()
     spans = ", ".join(f"[{lo}, {hi})" for lo, hi in sl.spans)
     return {"rows": sl.rows, "seconds": dt, "tokens_per_s": sl.rows / dt, "cores": op.cores,
-            "sample": f"rows {spans} of the {sl.w.name} batch ({sl.w.dtype}, V = {sl.w.vocab}), the device rows the "
-                      f"GPU timed, once; float64 numpy oracle on {op.cores} spawn workers"}
+            "sample": f"rows {spans} of the {sl.w.name} batch ({sl.w.dtype}, V = {sl.w.vocab}), drawn on the "
+                      f"device as the GPU's workload draws them, once; float64 numpy oracle on {op.cores} spawn "
+                      f"workers"}
 
 
 # ----------------------------------------------------------------------------- main

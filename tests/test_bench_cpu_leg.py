@@ -63,3 +63,23 @@ def test_oracle_slice_failure_is_reported_not_raised(monkeypatch):
     sl = bench.make_oracle_slice(W.WORKLOADS["tiny"], [], {})
     assert isinstance(sl, str) and "OSError" in sl
     assert bench.time_oracle_slice(sl) == {"unavailable": sl}
+
+
+def test_oracle_slice_falls_back_to_fewer_rows(monkeypatch):
+    """A span too large for shared memory is retried as its first rows; only when that fails
+    too is the slice reported as unavailable."""
+    made = []
+
+    class Tight:
+        def __init__(self, w, pieces, params):
+            n = sum(int(lg.shape[0]) for _, lg, _ in pieces)
+            if n > 8:
+                raise OSError(28, "No space left on device")
+            made.append(n)
+
+    monkeypatch.setattr(bench, "OracleSlice", Tight)
+    lg, ids = torch.zeros((20, 4)), torch.zeros(20, dtype=torch.int32)
+    sl = bench.make_oracle_slice(W.WORKLOADS["tiny"], [(0, lg, ids)], {}, fallback_rows=8)
+    assert isinstance(sl, Tight) and made == [8]
+    sl = bench.make_oracle_slice(W.WORKLOADS["tiny"], [(0, lg, ids)], {}, fallback_rows=12)
+    assert isinstance(sl, str) and "OSError" in sl
