@@ -213,17 +213,20 @@ def test_policy_loss_ragged_shapes(R, vocab, ld_pad, dtype_case):
     compare(case, out, f"V={vocab} ld=V+{ld_pad}")
 
 
-@pytest.mark.parametrize("name,vocab,ld_pad,rows,agg,tis", [
-    ("longhorizon", 4096, 0, 3000, 2, True),  # entropy + k3 KL + TIS; many rows per warp
-    ("multiturn", 4096, 0, 6000, 0, False),   # 40% masked rows, the paper's weighting
-    ("edge", 2048, 0, 2000, 2, False),        # fp32 at the 8 KB limit
-    ("tiny", 37, 3, 200, 2, False),           # four vectors and a ragged tail of five
-    ("longhorizon", 4104, 0, 300, 2, False),  # bf16 rows just over 8 KB: one CTA per row
-    ("edge", 2049, 3, 300, 2, True)])         # fp32 rows just over 8 KB, 16-byte aligned
-def test_policy_loss_short_rows(R, name, vocab, ld_pad, rows, agg, tis):
+@pytest.mark.parametrize("name,vocab,ld_pad,rows,agg,tis,ent", [
+    ("longhorizon", 4096, 0, 3000, 2, True, None),  # entropy + k3 KL + TIS; many rows per warp
+    ("multiturn", 4096, 0, 6000, 0, False, None),   # 40% masked rows, the paper's weighting
+    ("edge", 2048, 0, 2000, 2, False, None),        # fp32 at the 8 KB limit
+    ("edge", 1536, 4, 800, 2, False, 1e-2),         # fp32 with the entropy term
+    ("tiny", 37, 3, 200, 2, False, None),           # four vectors and a ragged tail of five
+    ("longhorizon", 4104, 0, 300, 2, False, None),  # bf16 rows just over 8 KB: one CTA per row
+    ("edge", 2049, 3, 300, 2, True, None)])         # fp32 rows just over 8 KB, 16-byte aligned
+def test_policy_loss_short_rows(R, name, vocab, ld_pad, rows, agg, tis, ent):
     """Rows of at most 8 KB (aligned) take the warp-per-row kernel; rows just over it take the
     cluster kernel with one CTA per row. Both against the oracle, with the workloads' masks."""
     case = make_case(name, seed=21, row0=0, rows=rows, vocab=vocab, loss_agg=agg, tis=tis)
+    if ent is not None:
+        case = dataclasses.replace(case, P=dataclasses.replace(case.P, entropy_coef=ent))
     out = run_loss(R, case, ld=vocab + ld_pad)
     compare(case, out, f"{name} V={vocab} ld=V+{ld_pad} rows={rows}")
 
