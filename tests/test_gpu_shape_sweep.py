@@ -96,3 +96,72 @@ def test_loss_shape_sweep(R, k, name, V, ld_pad, rows, agg, tis, ent, seed):
         case = dataclasses.replace(case, P=dataclasses.replace(case.P, entropy_coef=ent))
     out = run_loss(R, case, ld=V + ld_pad)
     compare(case, out, f"case {k}: {name} V={V} ld=V+{ld_pad} rows={rows} agg={agg} tis={tis} ent={ent}")
+
+
+def _draw_head(n=12, seed=7):
+    """Fused-head shapes: tokens 1-5,000 (ragged 128-row tiles, one or two 4,096-token chunks),
+    hidden sizes 64-1,024 (multiples of 64), vocabularies up to 20,000 (ragged 256-wide tiles,
+    up to five 4,096-wide blocks), with T D V at most 4e9 so the oracle stays quick."""
+    rng = np.random.default_rng(seed)
+    cases = []
+    for k in range(n):
+        D = 64 * int(rng.integers(1, 17))
+        V = int(rng.integers(1, 20_001))
+        T = int(min(rng.integers(1, 5_001), max(1, 4_000_000_000 // (D * V))))
+        cases.append((k, T, D, V, int(rng.integers(0, 3)), bool(rng.random() < 0.4), bool(rng.random() < 0.3)))
+    return cases
+
+
+HEAD_CASES = _draw_head()
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("k,T,D,V,agg,ent,tis", HEAD_CASES,
+                         ids=[f"{c[0]}-T{c[1]}-D{c[2]}-V{c[3]}" for c in HEAD_CASES])
+def test_fused_head_shape_sweep(R, k, T, D, V, agg, ent, tis):
+    from test_gpu_fused_head import compare_head, make_head_case, run_head
+
+    if T < 8:
+        pytest.skip("the case builder cuts at least four trajectories inside the token range")
+    c = make_head_case(T, D, V, seed=1000 + k, agg=agg, ent=ent, tis=tis)
+    compare_head(c, run_head(R, c))
+
+
+def _draw_fwd(n=16, seed=11):
+    """Forward log-probs shapes: bf16 or fp32 rows up to 400,000 entries, padded leading
+    dimensions, with and without the entropy and lse outputs."""
+    rng = np.random.default_rng(seed)
+    cases = []
+    for k in range(n):
+        fp32 = rng.random() < 0.4
+        V = int(np.exp(rng.uniform(0.0, np.log(400_000))))
+        if fp32:  # the edge workload's generator (spikes, half-masked rows) needs two entries
+            V = max(V, 2)
+        rows = int(max(1, min(64, 8_000_000 // V)))
+        cases.append((k, "edge" if fp32 else "multiturn", V, int(rng.integers(0, 9)), rows, bool(rng.random() < 0.5),
+                      int(rng.integers(0, 1 << 30))))
+    return cases
+
+
+FWD_CASES = _draw_fwd()
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("k,name,V,ld_pad,rows,ent,seed", FWD_CASES,
+                         ids=[f"{c[0]}-{c[1]}-V{c[2]}-ld{c[3]}-r{c[4]}" for c in FWD_CASES])
+def test_token_logprobs_shape_sweep(R, k, name, V, ld_pad, rows, ent, seed):
+    import oracle.grpo_objective as O
+    from parity_cases import logits_to_dev, to_dev
+
+    case = make_case(name, seed=seed % 1000, rows=rows, vocab=V)
+    ws = R.new_workspace(case.rows, V)
+    logp, H, lse = R.rl_token_logprobs(logits_to_dev(case, V + ld_pad), to_dev(case.ids), ws, want_entropy=ent,
+                                       want_lse=True)
+    assert R.rl_query_status(ws)[1] == 0
+    lp_ref, H_ref, lse_ref = O.token_logprobs(case.raw, case.w.dtype, case.ids)
+    lp, ls = logp.cpu().numpy().astype(np.float64), lse.cpu().numpy().astype(np.float64)
+    assert np.all(np.abs(lp - lp_ref) <= 1e-5 + 2.0 ** -22 * np.abs(lp_ref)), np.abs(lp - lp_ref).max()
+    assert np.all(np.abs(ls - lse_ref) <= 1e-5 + 2.0 ** -22 * np.abs(lse_ref)), np.abs(ls - lse_ref).max()
+    if ent:
+        Hd = H.cpu().numpy().astype(np.float64)
+        assert np.all(np.abs(Hd - H_ref) <= 5e-5 + 2e-5 * np.abs(H_ref)), np.abs(Hd - H_ref).max()
