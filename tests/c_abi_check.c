@@ -101,14 +101,19 @@ static int tree_checks(void) {
   return fails;
 }
 
-static int gpu_checks(void) {
-  enum { G = 2, PER = 4, N = G * PER, LEN = 24, T = N * LEN, V = 1000 };
+/* The advantages and the loss on uniform fp32 logits with old_logp = logp (-ln V), where the loss
+ * is -sum_i c_i L_i A_i (0 for complete groups) and every trained gradient row is
+ * -c_i A_i (onehot - 1/V); at V = 1,000 (rows of 4 KB: a warp per row) and V = 24,000 (rows of
+ * 96 KB: clusters of CTAs). */
+static int loss_checks(int V) {
+  enum { G = 2, PER = 4, N = G * PER, LEN = 24, T = N * LEN };
   const int32_t go[G + 1] = {0, PER, 2 * PER};
   float rewards[N];
   int64_t offs[N + 1];
   uint8_t mask[T];
   int32_t ids[T];
   float old[T];
+  int fails = 0;
   for (int i = 0; i < N; ++i) rewards[i] = (float)((i * 7) % 3);
   for (int i = 0; i <= N; ++i) offs[i] = (int64_t)i * LEN;
   for (int t = 0; t < T; ++t) {
@@ -150,7 +155,7 @@ static int gpu_checks(void) {
         "rl_group_advantages: %s", rl_last_error_message());
   CHECK(rl_policy_loss_fwd_bwd(d_logits, RL_F32, T, V, V, d_ids, d_mask, d_tt, N, d_adv, d_coef, d_old, NULL, NULL,
                                &p, d_grad, d_loss, NULL, d_ws, ws_bytes, NULL) == RL_OK,
-        "rl_policy_loss_fwd_bwd: %s", rl_last_error_message());
+        "rl_policy_loss_fwd_bwd (V = %d): %s", V, rl_last_error_message());
   int32_t word = -1;
   CHECK(rl_query_status(d_ws, NULL, &word) == RL_OK && word == 0, "device status %d", word);
 
@@ -166,18 +171,18 @@ static int gpu_checks(void) {
     expect -= (double)coef[i] * ntok[i] * adv[i];
     scale += fabs((double)coef[i] * ntok[i] * adv[i]);
   }
-  CHECK(fabs(loss - expect) <= 1e-5 * scale + 1e-12, "loss %.9g, closed form %.9g", loss, expect);
+  CHECK(fabs(loss - expect) <= 1e-5 * scale + 1e-12, "V = %d: loss %.9g, closed form %.9g", V, loss, expect);
   CHECK(fabs(expect) <= 1e-6 * scale + 1e-12, "complete groups: the closed form is 0 (%.3g)", expect);
   /* gradient rows: -c A (onehot - 1/V) on trained tokens, zero elsewhere */
-  float* row = (float*)malloc(V * sizeof(float));
+  float* row = (float*)malloc((size_t)V * sizeof(float));
   for (int t = 0; t < T; t += 7) {
-    cudaMemcpy(row, (char*)d_grad + (size_t)t * V * 4, V * sizeof(float), D2H);
+    cudaMemcpy(row, (char*)d_grad + (size_t)t * V * 4, (size_t)V * sizeof(float), D2H);
     const int i = t / LEN;
     const double g = mask[t] ? -(double)coef[i] * adv[i] : 0.0;
     for (int v = 0; v < V; ++v) {
       const double ref = g * ((v == ids[t] ? 1.0 : 0.0) - 1.0 / V);
       if (fabs(row[v] - ref) > 1e-6 * fabs(g) + 1e-12) {
-        fprintf(stderr, "FAIL: grad[%d][%d] = %.9g, closed form %.9g\n", t, v, row[v], ref);
+        fprintf(stderr, "FAIL: V = %d: grad[%d][%d] = %.9g, closed form %.9g\n", V, t, v, row[v], ref);
         ++fails;
         break;
       }
@@ -188,6 +193,8 @@ static int gpu_checks(void) {
   for (size_t k = 0; k < sizeof all / sizeof all[0]; ++k) cudaFree(all[k]);
   return fails;
 }
+
+static int gpu_checks(void) { return loss_checks(1000) + loss_checks(24000); }
 
 /* The fused head with all hidden states 0 (so every logits row is 0: uniform), the masked GAE at
  * gamma = lambda = 1 in the skip reading, and the value loss, each against its closed form:
