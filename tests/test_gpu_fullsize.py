@@ -123,6 +123,77 @@ def test_full_microbatch(R, name, mb):
     check_grad(g_dev, g_ref, w.dtype, f"{name} mb {mb} sampled rows", row_scale=scale)
 
 
+def test_whole_multiturn_batch(R):
+    """The benchmark's whole step as bench.py calls it: rl_group_advantages over the 155,959-token
+    multi-turn batch, then rl_policy_loss_fwd_bwd on each of its ten 16,384-row microbatches into
+    one loss accumulator (V = 151,936 bf16). The oracle computes every row's log-probability,
+    entropy and log-sum-exp in float64 and, with its own advantages and coefficients, the batch
+    loss. Checked: token counts and owners (bit-exact), advantages and coefficients (one float32
+    ulp), the total loss, every row's statistics, every inactive row exactly zero, and gradients
+    on sampled rows of every microbatch."""
+    w = W.WORKLOADS["multiturn"]
+    seed = 0
+    lay = W.make_layout(w, seed)
+    T = lay.n_tokens
+    logits = torch.empty((T, w.vocab), dtype=torch.bfloat16, device="cuda")
+    W.logits_rows_torch(w, seed, 0, T, logits)
+    ids = W.sample_tokens_torch(logits, seed, 0, w)
+    ids_np = ids.cpu().numpy()
+    logp, H, lse = np.empty(T), np.empty(T), np.empty(T)
+    for b0 in range(0, T, BLOCK):
+        b1 = min(T, b0 + BLOCK)
+        logp[b0:b1], H[b0:b1], lse[b0:b1] = token_logprobs_parallel(_host_raw(logits[b0:b1], "bf16"), "bf16",
+                                                                    ids_np[b0:b1])
+    old = W.old_logp_from(logp, w, seed)
+    P = loss_params(w)
+    adv, coef, L, tt = O.advantages_and_coefficients(lay.rewards, lay.group_offsets, lay.traj_offsets, lay.mask,
+                                                     lay.traj_valid, P)
+
+    # the CUDA path: advantages over the batch, then the microbatches
+    ws = R.new_workspace(w.microbatch, w.vocab)
+    a_d, c_d, n_d, tt_d = R.rl_group_advantages(to_dev(lay.group_offsets), to_dev(lay.rewards),
+                                                to_dev(lay.traj_offsets), to_dev(lay.mask), cuda_params(R, P), ws,
+                                                traj_valid=to_dev(lay.traj_valid))
+    mbs = W.microbatches(lay, w.microbatch)
+    assert len(mbs) == 10
+    loss = torch.zeros(1, dtype=torch.float64, device="cuda")
+    st = torch.zeros(T * 5, dtype=torch.float32, device="cuda")
+    grad = torch.empty_like(logits)
+    mask_d, old_d = to_dev(lay.mask), to_dev(old.astype(np.float32))
+    for lo, hi in mbs:
+        R.rl_policy_loss_fwd_bwd(logits[lo:hi], ids[lo:hi], mask_d[lo:hi], tt_d[lo:hi], a_d, c_d, old_d[lo:hi],
+                                 cuda_params(R, P), ws, loss, grad_out=grad[lo:hi], token_stats=st[lo * 5:hi * 5])
+    assert R.rl_query_status(ws)[1] == 0
+    assert np.array_equal(n_d.cpu().numpy(), L) and np.array_equal(tt_d.cpu().numpy(), tt)
+    a32, c32 = a_d.cpu().numpy().astype(np.float64), c_d.cpu().numpy().astype(np.float64)
+    assert np.all(np.abs(a32 - adv) <= 2.0 ** -23 * np.abs(adv)) and np.all(np.abs(c32 - coef) <= 2.0 ** -23 * coef)
+
+    adv_o, coef_o = adv.astype(np.float32).astype(np.float64), coef.astype(np.float32).astype(np.float64)
+    z_a = O.decode_logits(_host_raw(logits.gather(1, ids.long()[:, None])[:, 0].contiguous(), "bf16"), "bf16")
+    terms = O.token_terms(z_a, lse, H, old, adv_o[tt], P)
+    c_row = coef_o[tt]
+    active = (lay.mask != 0) & (c_row != 0)
+    contrib = np.where(active, c_row * terms["ell"], 0.0)
+    check_loss(loss.item(), math.fsum(contrib.tolist()), contrib, "whole multi-turn batch loss")
+    stats_ref = np.stack([terms["logp"], terms["rho"], terms["cut"], H, terms["kl"]], axis=1)
+    stats_ref[~active] = 0.0
+    check_stats(st.view(-1, 5).cpu().numpy(), stats_ref, active, "whole multi-turn batch stats")
+
+    inactive_idx = torch.from_numpy(np.nonzero(~active)[0]).cuda()
+    assert int(torch.count_nonzero(grad.index_select(0, inactive_idx)).item()) == 0
+    rng = np.random.default_rng(321)
+    sample = []
+    for lo, hi in mbs:
+        act = np.nonzero(active[lo:hi])[0] + lo
+        sample.extend(rng.choice(act, size=min(3, len(act)), replace=False).tolist())
+    sample = np.array(sorted(sample))
+    sel = torch.from_numpy(sample).cuda()
+    _, g_ref, _, _ = O.policy_loss_fwd_bwd(_host_raw(logits.index_select(0, sel), "bf16"), "bf16", ids_np[sample],
+                                           lay.mask[sample], tt[sample], adv_o, coef_o, old[sample], P)
+    scale = (np.abs(c_row[sample]) * np.abs(adv_o[tt][sample]) * stats_ref[sample, 1])[:, None]
+    check_grad(grad_to_np(grad.index_select(0, sel)), g_ref, "bf16", "whole batch sampled rows", row_scale=scale)
+
+
 def test_fused_head_full_size(R):
     """The fused LM head at 32,768 x 4,096 x 151,936 (four chunks), as the benchmark calls it.
 
