@@ -1,0 +1,91 @@
+"""Properties of the CUDA path that need no oracle (needs a GB300).
+
+Reordering whole groups in the packed batch (each group's trajectories and their tokens move
+together) changes nothing a row or a trajectory sees: its own logits, its group's rewards, and
+N, S over the batch. So after the reordering every row's gradient and statistics and every
+trajectory's advantage, coefficient and count must be the same bits, and the loss the same up
+to the order of its sum.
+"""
+
+import dataclasses
+
+import numpy as np
+import pytest
+import torch
+
+from parity_cases import cuda_params, loss_params, to_dev
+from paper_2608_16798_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def R():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_16798_gb300 import build
+
+    build.build()
+    import paper_2608_16798_gb300.rl_loss as R
+
+    R.lib()
+    return R
+
+
+def _reorder_groups(lay, perm):
+    """The layout with its groups in the order perm; returns (group offsets, trajectory offsets,
+    rewards, validity, mask) of the new packing, the old trajectory of each new one and the old
+    token of each new one."""
+    go, to = lay.group_offsets, lay.traj_offsets
+    traj_order = np.concatenate([np.arange(go[g], go[g + 1]) for g in perm]).astype(np.int64)
+    sizes = np.array([go[g + 1] - go[g] for g in perm])
+    new_go = np.concatenate([[0], np.cumsum(sizes)]).astype(np.int32)
+    lens = (to[1:] - to[:-1])[traj_order]
+    new_to = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    tok_order = np.concatenate([np.arange(to[i], to[i + 1]) for i in traj_order]).astype(np.int64)
+    return (new_go, new_to, lay.rewards[traj_order], lay.traj_valid[traj_order], lay.mask[tok_order], traj_order,
+            tok_order)
+
+
+def _step(R, P, go, to, rewards, valid, mask, logits, ids, old):
+    T, V = logits.shape
+    ws = R.new_workspace(T, V)
+    adv, coef, n_tok, tt = R.rl_group_advantages(to_dev(go), to_dev(rewards), to_dev(to), to_dev(mask),
+                                                 cuda_params(R, P), ws, traj_valid=to_dev(valid))
+    loss = torch.zeros(1, dtype=torch.float64, device="cuda")
+    st = torch.zeros(T * 5, dtype=torch.float32, device="cuda")
+    grad = R.rl_policy_loss_fwd_bwd(logits, ids, to_dev(mask), tt, adv, coef, old, cuda_params(R, P), ws, loss,
+                                    token_stats=st)
+    assert R.rl_query_status(ws)[1] == 0
+    return adv, coef, n_tok, grad, st.view(T, 5), loss.item()
+
+
+@pytest.mark.parametrize("name,vocab", [("multiturn", 4096), ("edge", None)])  # warp-per-row, cluster kernel
+def test_reordering_groups_changes_nothing(R, name, vocab):
+    w = W.WORKLOADS[name] if vocab is None else dataclasses.replace(W.WORKLOADS[name], vocab=vocab)
+    lay = W.make_layout(w, 3)
+    T = lay.n_tokens
+    dt = torch.bfloat16 if w.dtype == "bf16" else torch.float32
+    logits = torch.empty((T, w.vocab), dtype=dt, device="cuda")
+    W.logits_rows_torch(w, 3, 0, T, logits)
+    ids = W.sample_tokens_torch(logits, 3, 0, w)
+    logp, _, _ = R.rl_token_logprobs(logits, ids, R.new_workspace(T, w.vocab))
+    old = to_dev(W.old_logp_from(logp.cpu().numpy().astype(np.float64), w, 3))
+    P = loss_params(w, loss_agg=0)
+
+    a0, c0, n0, g0, s0, l0 = _step(R, P, lay.group_offsets, lay.traj_offsets, lay.rewards, lay.traj_valid, lay.mask,
+                                   logits, ids, old)
+    perm = np.random.default_rng(4).permutation(len(lay.group_offsets) - 1)
+    go, to, rw, va, mk, traj_order, tok_order = _reorder_groups(lay, perm)
+    t_ord = torch.from_numpy(tok_order).cuda()
+    j_ord = torch.from_numpy(traj_order).cuda()
+    a1, c1, n1, g1, s1, l1 = _step(R, P, go, to, rw, va, mk, logits.index_select(0, t_ord).contiguous(),
+                                   ids.index_select(0, t_ord).contiguous(), old.index_select(0, t_ord).contiguous())
+
+    assert torch.equal(a1, a0.index_select(0, j_ord)) and torch.equal(c1, c0.index_select(0, j_ord))
+    assert torch.equal(n1, n0.index_select(0, j_ord))
+    assert torch.equal(s1, s0.index_select(0, t_ord))
+    view = torch.int16 if dt == torch.bfloat16 else torch.int32
+    assert torch.equal(g1.view(view), g0.index_select(0, t_ord).view(view))
+    # the loss terms are the same; only the order of the double-precision sum changes
+    assert abs(l1 - l0) <= 1e-9 * max(abs(l0), 1e-30) + 1e-15, (l0, l1)
