@@ -89,3 +89,27 @@ def test_reordering_groups_changes_nothing(R, name, vocab):
     assert torch.equal(g1.view(view), g0.index_select(0, t_ord).view(view))
     # the loss terms are the same; only the order of the double-precision sum changes
     assert abs(l1 - l0) <= 1e-9 * max(abs(l0), 1e-30) + 1e-15, (l0, l1)
+
+
+def test_fused_head_token_order(R):
+    """The fused head with its tokens reordered (each with its id, mask, owner and old_logp):
+    every token's d_hidden row and statistics are the same bits, the loss the same up to the
+    order of its sum, and d_W, a sum over tokens that the products now group differently, the
+    same up to float32 rounding of its terms."""
+    from test_gpu_fused_head import make_head_case, run_head
+
+    c = make_head_case(4096 + 515, 192, 3000, seed=31, agg=0, ent=True)
+    a = run_head(R, c)
+    perm = np.random.default_rng(5).permutation(c["T"])
+    p = dict(c)
+    p["h"] = c["h"][perm]
+    for k in ("ids", "mask", "tt", "old", "ref"):
+        p[k] = c[k][perm]
+    b = run_head(R, p)
+    assert a["word"] == 0 and b["word"] == 0
+    assert np.array_equal(b["dH"], a["dH"][perm]), "d_hidden rows differ after reordering the tokens"
+    assert np.array_equal(b["stats"], a["stats"][perm])
+    assert abs(b["loss"] - a["loss"]) <= 1e-9 * max(abs(a["loss"]), 1e-30) + 1e-15
+    scale = np.abs(a["dW"]).max()
+    assert np.all(np.abs(b["dW"] - a["dW"]) <= 1e-3 * scale + 1e-5 * np.abs(a["dW"])), \
+        np.abs(b["dW"] - a["dW"]).max() / scale
