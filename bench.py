@@ -471,8 +471,9 @@ class StagedPinned:
     """Host memory for the end-to-end leg: a HostStagingBuffer (one mapping with transparent huge
     pages, registered with the CUDA runtime). Once filled, its units are qualified by timing a
     copy from each to the device; units that copy far below the median are replaced and refilled
-    before any timed work. On the box, a few physical huge pages in some processes copy at 3-72
-    GB/s against 210 GB/s from the rest, and pages can turn slow when first written. Falls back to
+    before any timed work. On the Grace host of a GB300, a few physical huge pages in some
+    processes were measured to copy at 3-72 GB/s against 210 GB/s from the rest, and pages can
+    turn slow when first written. Falls back to
     torch's pinned allocator when the mapping or registration is refused."""
 
     def __init__(self, torch, rows, cols, dtype, dev):
@@ -647,8 +648,8 @@ def e2e_run(torch, R, batch, dev, steps, warmup, slots=4, repeats=3):
             out.append((hi - lo) * V * 2 / a0.elapsed_time(a1) / 1e6)
         return out
 
-    # repetitions of `steps` timed steps; before each, the staging buffer is qualified again (on
-    # the box, pages of a qualified buffer were seen to turn slow later in the same process)
+    # repetitions of `steps` timed steps; before each, the staging buffer is qualified again
+    # (pages of a qualified buffer have been seen to turn slow later in the same process)
     runs = []
     for rep in range(repeats):
         if rep > 0 and (whole or len(batch.mbs) >= 2):
