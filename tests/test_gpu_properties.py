@@ -113,3 +113,60 @@ def test_fused_head_token_order(R):
     scale = np.abs(a["dW"]).max()
     assert np.all(np.abs(b["dW"] - a["dW"]) <= 1e-3 * scale + 1e-5 * np.abs(a["dW"])), \
         np.abs(b["dW"] - a["dW"]).max() / scale
+
+
+@pytest.mark.parametrize("name,vocab", [("multiturn", 4096), ("multiturn", None), ("edge", None)])
+def test_statistics_request_changes_no_bit(R, name, vocab):
+    """Asking for the per-token statistics selects the kernel form that also sums the entropy;
+    with no entropy bonus (alpha = 0) the loss is the same bits and every gradient element the
+    same value as without the statistics (the warp-per-row kernel and the cluster kernel, bf16
+    and fp32), logits at -inf included. Zeros may differ in sign: in a row whose surrogate
+    weight c g is 0 and whose log-sum-exp lies below its entropy (the edge workload's rows at
+    -1e4), the entropy form's coefficient is -0 + 0 (H - lse) = +0 where the other's is -0."""
+    from parity_cases import make_case, logits_to_dev
+
+    case = make_case(name, seed=41, row0=500, rows=300, vocab=vocab, loss_agg=2)
+    raw = case.raw.copy()
+    ninf = np.uint16(0xFF80) if case.w.dtype == "bf16" else np.float32(-np.inf)
+    for r in range(0, case.rows, 3):  # a few entries at -inf (never the sampled one)
+        cols = np.random.default_rng(r).choice(raw.shape[1], size=max(1, raw.shape[1] // 50), replace=False)
+        cols = cols[cols != case.ids[r]]
+        raw[r, cols] = ninf
+    case = dataclasses.replace(case, raw=raw)
+    logits = logits_to_dev(case)
+    args = (to_dev(case.ids), to_dev(case.mask), to_dev(case.tt.astype(np.int32)),
+            to_dev(case.adv64.astype(np.float32)), to_dev(case.coef64.astype(np.float32)), to_dev(case.old),
+            cuda_params(R, case.P))
+    assert case.P.entropy_coef == 0.0
+    outs = []
+    for stats in (None, torch.zeros(case.rows * 5, dtype=torch.float32, device="cuda")):
+        ws = R.new_workspace(case.rows, raw.shape[1])
+        loss = torch.zeros(1, dtype=torch.float64, device="cuda")
+        g = R.rl_policy_loss_fwd_bwd(logits, *args, ws, loss, ref_logp=None if case.ref is None else to_dev(case.ref),
+                                     token_stats=stats)
+        assert R.rl_query_status(ws)[1] == 0
+        outs.append((loss.item(), g))
+    assert outs[0][0] == outs[1][0]
+    assert torch.equal(outs[0][1], outs[1][1])  # values: -0 == +0
+
+
+def test_stats_summary_skips_bad_owners(R):
+    """Rows whose owner is outside [0, n_traj) set RL_DEV_BAD_TRAJ and are left out of the sums."""
+    import oracle.grpo_objective as O
+
+    rng = np.random.default_rng(8)
+    rows, n_traj = 20000, 50
+    stats = rng.random((rows, 5), dtype=np.float32)
+    mask = (rng.random(rows) < 0.7).astype(np.uint8)
+    tt = rng.integers(0, n_traj, rows).astype(np.int32)
+    bad = rng.choice(rows, size=37, replace=False)
+    tt[bad] = np.where(np.arange(37) % 2 == 0, -3, n_traj + 5)
+    coef = rng.random(n_traj).astype(np.float32)
+    ws = R.new_workspace(0, 0)
+    got = R.rl_token_stats_summary(torch.from_numpy(stats.reshape(-1)).cuda(), to_dev(mask), to_dev(tt),
+                                   to_dev(coef), ws).cpu().numpy()
+    assert R.rl_query_status(ws)[1] & R.RL_DEV_BAD_TRAJ
+    keep = np.ones(rows, bool)
+    keep[bad] = False
+    ref = O.stats_summary(stats[keep].astype(np.float64), mask[keep], tt[keep], coef)
+    assert got[0] == ref[0] and got[1] == ref[1] and np.allclose(got[2:], ref[2:], rtol=1e-12, atol=1e-12)
