@@ -919,7 +919,10 @@ __global__ void __launch_bounds__(kSmallWarps * 32, 2) small_rows_kernel(const R
       Vec<T>::store_scalar(g_row + a, (ENT ? pk * fmaf(ca, fmaxf(za, -1e30f), Ke) : Kp * pk) + cg);
     }
   }
-  // ---- the loss: warps in order into one partial per CTA; the last CTA adds the partials
+  // ---- the loss: warps in order into one partial per CTA; the last CTA adds the partials, all
+  // its threads loading them at once (thread k takes partials k, k + 256, ...), then combined
+  // by shuffles and the warps in order: a fixed order for a given grid
+  __shared__ uint32_t is_last;
   if (lane == 0) warp_loss[warp] = w_loss;
   __syncthreads();
   if (threadIdx.x == 0) {
@@ -927,11 +930,19 @@ __global__ void __launch_bounds__(kSmallWarps * 32, 2) small_rows_kernel(const R
     for (int k = 0; k < kSmallWarps; ++k) t += warp_loss[k];
     p.row_loss[blockIdx.x] = t;
     __threadfence();
-    const bool last = atomicAdd(p.done, 1u) == gridDim.x - 1;
-    if (last) {
-      __threadfence();
+    is_last = atomicAdd(p.done, 1u) == gridDim.x - 1 ? 1u : 0u;
+  }
+  __syncthreads();
+  if (is_last) {
+    __threadfence();
+    double t = 0.0;
+    for (unsigned k = threadIdx.x; k < gridDim.x; k += kSmallWarps * 32) t += __ldcg(p.row_loss + k);
+    t = warp_sum(t);
+    if (lane == 0) warp_loss[warp] = t;
+    __syncthreads();
+    if (threadIdx.x == 0) {
       double sum = 0.0;
-      for (unsigned k = 0; k < gridDim.x; ++k) sum += __ldcg(p.row_loss + k);
+      for (int k = 0; k < kSmallWarps; ++k) sum += warp_loss[k];
       *p.loss_accum += sum;
       *p.done = 0u;
     }
