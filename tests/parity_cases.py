@@ -239,3 +239,60 @@ def check_stats(st_dev, st_ref, active, what="", zerr=None):
     assert np.all(d[:, 3] <= 5e-5 + 2e-5 * np.abs(b[:, 3]) + 2 * z), f"{what}: entropy max diff {d[:, 3].max()}"
     assert np.all(d[:, 4] <= 1e-6 + 1e-4 * np.abs(b[:, 4]) + 2 * z * (1 + np.abs(b[:, 4]))), \
         f"{what}: KL max diff {d[:, 4].max()}"
+
+
+# ----------------------------------------------------------------------------- the loss call and its comparison
+
+def run_loss(R, case, adv32=None, coef32=None, ld=None, in_place=False, stats=True, ws=None):
+    dev = "cuda"
+    logits = logits_to_dev(case, ld)
+    adv32 = case.adv64.astype(np.float32) if adv32 is None else adv32
+    coef32 = case.coef64.astype(np.float32) if coef32 is None else coef32
+    ws = R.new_workspace(case.rows, case.raw.shape[1]) if ws is None else ws
+    loss = torch.zeros(1, dtype=torch.float64, device=dev)
+    st = torch.full((case.rows * 5,), float("nan"), dtype=torch.float32, device=dev) if stats else None
+    # the gradient buffer starts as NaN everywhere (padding columns included): an element the
+    # library should write and does not stays NaN and fails the comparison
+    poison = torch.full_like(logits, float("nan")) if logits.is_contiguous() else None
+    if not in_place and poison is None:
+        full = torch.full((case.rows, logits.stride(0)), float("nan"), dtype=logits.dtype, device=dev)
+        poison = full[:, :logits.shape[1]]
+    g = R.rl_policy_loss_fwd_bwd(logits, to_dev(case.ids), to_dev(case.mask), to_dev(case.tt.astype(np.int32)),
+                                 to_dev(adv32), to_dev(coef32), to_dev(case.old), cuda_params(R, case.P), ws, loss,
+                                 grad_out=logits if in_place else poison,
+                                 ref_logp=None if case.ref is None else to_dev(case.ref),
+                                 rollout_logp=None if case.roll is None else to_dev(case.roll), token_stats=st)
+    status, word = R.rl_query_status(ws)
+    if not in_place and not logits.is_contiguous():  # columns past V are never written
+        assert torch.isnan(full[:, logits.shape[1]:]).all()
+    return dict(loss=float(loss.item()), grad=grad_to_np(g), stats=None if st is None else st.view(-1, 5).cpu().numpy(),
+                status=status, word=word)
+
+
+def grad_scale(case, stats, adv, coef):
+    """Per-row size of the gradient's coefficients |c| (w |A| rho + beta |1 - e^(r - logp)| + alpha (1 + |H|)),
+    the scale of the float32 rounding in a row (used only as an error floor)."""
+    c = np.abs(coef[case.tt])
+    A = np.abs(adv[case.tt])
+    rho, H, logp = stats[:, 1], stats[:, 3], stats[:, 0]
+    w = np.ones_like(rho)
+    if case.roll is not None and case.P.tis_cap > 0:
+        w = np.minimum(np.exp(case.old.astype(np.float64) - case.roll), case.P.tis_cap)
+    kl = 0.0
+    if case.ref is not None and case.P.kl_coef:
+        kl = case.P.kl_coef * np.abs(1 - np.exp(np.clip(case.ref - logp, -50, 50)))
+    return (c * (w * A * rho + kl + case.P.entropy_coef * (1 + np.abs(H))))[:, None]
+
+
+def compare(case, out, what):
+    adv32 = case.adv64.astype(np.float32).astype(np.float64)
+    coef32 = case.coef64.astype(np.float32).astype(np.float64)
+    loss, grad, stats, contrib = oracle_loss(case, adv32, coef32)
+    check_loss(out["loss"], loss, contrib, what)
+    check_grad(out["grad"], grad, case.w.dtype, what, row_scale=grad_scale(case, stats, adv32, coef32),
+               absolute=case.P.loss_agg != O.AGG_TOKEN_SUM)
+    active = (case.mask != 0) & (coef32[case.tt] != 0)
+    assert np.all(out["grad"][~active] == 0.0), f"{what}: inactive rows not exactly zero"
+    if out["stats"] is not None:
+        check_stats(out["stats"], stats, active, what)
+    assert out["word"] == 0, f"{what}: device status {out['word']}"

@@ -15,9 +15,8 @@ import numpy as np
 import pytest
 import torch
 
-from parity_cases import make_case
+from parity_cases import compare, make_case, run_loss
 from paper_2608_16798_gb300 import workloads as W
-from test_gpu_parity import compare, run_loss
 
 
 def _draw(n=40, seed=2026):
